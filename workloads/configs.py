@@ -1,0 +1,162 @@
+"""The five workload recipes (tiny expression grammar, SQL admin, SQL
+SELECT-only headline, long/deep flatness sweep, cold schema).
+
+Each recipe returns a plain dict of inputs; seeds default to 1000 + index.
+Prefixes are lists of token ids obtained by rendering a random sentence,
+tokenizing it greedily and truncating it (at a byte offset for the tiny
+grammar, at a token count for the SQL workloads)."""
+from __future__ import annotations
+
+import numpy as np
+
+from . import grammar_text, grammar_keywords
+from .gen import (GreedyTokenizer, SqlGen, expr_sentence, expr_vocab, make_schema,
+                  render, sql_vocab)
+
+SQL_V_HEADLINE = 151_936
+SQL_V_SWEEP = 128_256
+SQL_V_ADMIN = 32_000
+
+_cache: dict = {}
+
+
+def _sql_vocab_cached(V: int, seed: int, multiword: float):
+    key = ("vocab", V, seed, multiword)
+    if key not in _cache:
+        kws = grammar_keywords(grammar_text("sql"))
+        src = None
+        if multiword > 0:
+            rng = np.random.default_rng(seed + 77)
+            tables, cols, _ = make_schema(seed + 78, 50, 12, kws, col_pool=300)
+            g = SqlGen(rng, tables, cols, dml=True)
+            src = [render(g.statement(2), rng).encode() for _ in range(3000)]
+        _cache[key] = sql_vocab(seed, V, kws, multiword_frac=multiword, sentence_src=src)
+    return _cache[key]
+
+
+def tiny_expr(seed: int = 1001, B: int = 64, V: int = 512):
+    """Expression grammar, V=512 vocab over [a-z0-9+*() ], 64 prefixes truncated
+    at a uniformly random byte offset of a random derivation (nesting <= 8)."""
+    rng = np.random.default_rng(seed)
+    toks, eos, specials = expr_vocab(seed, V)
+    tk = GreedyTokenizer(toks, specials + [eos])
+    prefixes, texts = [], []
+    for _ in range(B):
+        s = expr_sentence(rng, 8).encode()
+        cut = int(rng.integers(0, len(s) + 1))
+        texts.append(s[:cut])
+        prefixes.append(tk.encode(s[:cut]))
+    return dict(name="tiny_expr", grammar=grammar_text("expr"), role=None, lexicons={},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
+                seed=seed)
+
+
+def _sql_prefixes(rng, gen: SqlGen, tk: GreedyTokenizer, lens):
+    prefixes, texts = [], []
+    for n in lens:
+        preds = max(1, n // 10)
+        while True:
+            text = render(gen.statement(2, where_preds=preds), rng, comment_rate=0.01).encode()
+            ids = tk.encode(text)
+            if len(ids) >= n or preds > 4 * n:
+                break
+            preds *= 2
+        ids = ids[:n]
+        prefixes.append(ids)
+        texts.append(b"".join(tk_tokens(tk, ids)))
+    return prefixes, texts
+
+
+def tk_tokens(tk: GreedyTokenizer, ids):
+    inv = getattr(tk, "_inv", None)
+    if inv is None:
+        inv = {v: k for k, v in tk.map.items()}
+        tk._inv = inv
+    return [inv[i] for i in ids]
+
+
+def sql_admin(seed: int = 1002, B: int = 32, V: int = SQL_V_ADMIN):
+    """SQL grammar, admin role (all productions), schema 20 x 10, V=32,000,
+    32 prefixes of U[20,200] tokens."""
+    kws = grammar_keywords(grammar_text("sql"))
+    tables, cols, words = make_schema(seed, 20, 10, kws, col_pool=120)
+    toks, eos, specials = _sql_vocab_cached(V, seed, 0.0)
+    tk = GreedyTokenizer(toks, specials + [eos])
+    rng = np.random.default_rng(seed + 1)
+    lens = [int(x) for x in rng.integers(20, 201, size=B)]
+    prefixes, texts = _sql_prefixes(rng, SqlGen(rng, tables, cols, dml=True), tk, lens)
+    return dict(name="sql_admin", grammar=grammar_text("sql"), role=["dml"],
+                lexicons={"TABLE_NAME": tables, "COLUMN_NAME": words},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
+                seed=seed)
+
+
+def sql_select_only(seed: int = 1003, B: int = 32, V: int = SQL_V_HEADLINE,
+                    lo: int = 50, hi: int = 2000):
+    """Headline workload: SQL grammar under the SELECT-only projection (DML
+    productions removed), schema 200 x 30, V=151,936 with ~3% multi-word tokens,
+    B=32 prefixes of U[50,2000] tokens, fp32 logits N(0,3)."""
+    kws = grammar_keywords(grammar_text("sql"))
+    tables, cols, words = make_schema(seed, 200, 30, kws, col_pool=3000)
+    toks, eos, specials = _sql_vocab_cached(V, 1003, 0.03)
+    tk = GreedyTokenizer(toks, specials + [eos])
+    rng = np.random.default_rng(seed + 1)
+    lens = [int(x) for x in rng.integers(lo, hi + 1, size=B)]
+    prefixes, texts = _sql_prefixes(rng, SqlGen(rng, tables, cols, dml=False), tk, lens)
+    return dict(name="sql_select_only", grammar=grammar_text("sql"), role=[],
+                lexicons={"TABLE_NAME": tables, "COLUMN_NAME": words},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
+                seed=seed, logits_dtype="f32", logits_std=3.0)
+
+
+def sql_sweep_cell(n: int, depth: int, seed: int = 1004, B: int = 32, V: int = SQL_V_SWEEP):
+    """One cell of the flatness sweep: admin role, schema 200 x 30, V=128,256,
+    B=32 prefixes of exactly ``n`` tokens whose first part opens ``depth``
+    nesting levels (parentheses or IN-subqueries) and whose rest is a
+    left-recursive AND/OR chain, truncated mid-chain."""
+    kws = grammar_keywords(grammar_text("sql"))
+    tables, cols, words = make_schema(seed, 200, 30, kws, col_pool=3000)
+    toks, eos, specials = _sql_vocab_cached(V, seed, 0.0)
+    tk = GreedyTokenizer(toks, specials + [eos])
+    rng = np.random.default_rng(seed * 1000 + n * 7 + depth)
+    gen = SqlGen(rng, tables, cols, dml=True)
+    prefixes, texts = [], []
+    for _ in range(B):
+        preds = max(2, n // 6)
+        while True:
+            text = render(gen.nested_chain(depth, preds), rng).encode()
+            ids = tk.encode(text, limit=n + 1)
+            if len(ids) > n:
+                break
+            preds *= 2
+        ids = ids[:n]
+        prefixes.append(ids)
+        texts.append(b"".join(tk_tokens(tk, ids)))
+    return dict(name="sql_sweep_n%d_d%d" % (n, depth), grammar=grammar_text("sql"), role=["dml"],
+                lexicons={"TABLE_NAME": tables, "COLUMN_NAME": words},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
+                seed=seed, n=n, depth=depth)
+
+
+def sql_cold_schema(seed: int = 1005, B: int = 256, V: int = SQL_V_HEADLINE,
+                    lo: int = 50, hi: int = 2000):
+    """Cold-schema workload: a fresh schema of 1,000 tables x 50 distinct
+    columns (50k identifiers), SELECT-only role, the headline V=151,936
+    vocabulary, B=256 prefixes of U[50,2000] tokens, bf16 logits N(0,3)."""
+    kws = grammar_keywords(grammar_text("sql"))
+    tables, cols, words = make_schema(seed, 1000, 50, kws, col_pool=None)
+    toks, eos, specials = _sql_vocab_cached(V, 1003, 0.03)
+    tk = GreedyTokenizer(toks, specials + [eos])
+    rng = np.random.default_rng(seed + 1)
+    lens = [int(x) for x in rng.integers(lo, hi + 1, size=B)]
+    prefixes, texts = _sql_prefixes(rng, SqlGen(rng, tables, cols, dml=False), tk, lens)
+    return dict(name="sql_cold_schema", grammar=grammar_text("sql"), role=[],
+                lexicons={"TABLE_NAME": tables, "COLUMN_NAME": words},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
+                seed=seed, logits_dtype="bf16", logits_std=3.0)
+
+
+def logits(seed: int, B: int, V: int, std: float = 3.0):
+    """fp32 logits ~ N(0, std^2), shape [B, V], as a numpy array."""
+    rng = np.random.default_rng(seed + 99)
+    return (rng.standard_normal((B, V), dtype=np.float32) * np.float32(std)).astype(np.float32)
