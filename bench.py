@@ -1,0 +1,345 @@
+"""Benchmark of the cold full-vocabulary mask step on GB300.
+
+Workload (default): SQL SELECT-only projection, schema 200 x 30, vocabulary
+V = 151,936 (seeded, BPE-like, ~3% multi-word tokens), batch B = 32 parser
+configurations at prefixes of U[50, 2000] tokens, fp32 logits N(0, 3).
+
+One step = the whole per-token hot path for one batch, through the C ABI:
+  grid_advance (out-of-place, one admitted token per row)
+  -> grid_masks (allowed sets + EOS gate, trie walk, id-order packing)
+  -> grid_apply_mask (in-place -inf fill of the fp32 logits).
+Steps rotate over 16 distinct pre-built batches (512 prefixes); their logits
+(16 x 19.45 MB = 311 MB) exceed the 129 MB L2, so every step reads cold logits.
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+N_BATCHES = 16
+METRIC = "cold full-vocab masks/s (batch-32 mask step at V=151,936)"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = "clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown," \
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown," \
+             "clocks_event_reasons.sw_power_cap"
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) == 7:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=2)
+        except Exception:
+            self.proc.kill()
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in self.rows for k in range(4) if r[3 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args):
+    """The CPU oracle as it stands, on the host cores: each step is a bounded
+    sample (one configuration of the workload, ``--ref-tokens`` token ids,
+    split over a spawn pool of all cores)."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    import numpy as np
+    from tests.harness import _init_worker, _oracle_rows
+    from workloads import configs
+    import multiprocessing as mp
+    wl = configs.sql_select_only()
+    V = len(wl["tokens"])
+    cores = os.cpu_count() or 1
+    S = args.ref_tokens
+    rng = np.random.default_rng(0)
+    ctx = mp.get_context("spawn")
+    times = []
+    with ctx.Pool(cores, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])) as pool:
+        def step(k):
+            row = k % len(wl["prefixes"])
+            ids = rng.choice(V, S, replace=False)
+            parts = np.array_split(ids, cores)
+            jobs = [(wl["prefixes"][row], wl["tokens"], wl["eos"], wl["specials"], list(p)) for p in parts]
+            t0 = time.perf_counter()
+            pool.map(_oracle_rows, jobs, chunksize=1)
+            return time.perf_counter() - t0
+        for k in range(args.warmup):
+            step(k)
+        for k in range(args.steps):
+            times.append(step(k))
+    tot = sum(times)
+    value = args.steps * S / V / tot
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "masks/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+            "data": "synthetic",
+            "config": {"workload": "sql_select_only", "B": 32, "V": V},
+            "cpu_baseline": {"value": value, "unit": "masks/s", "cores": cores, "kind": "oracle",
+                             "sample": "per step: %d random token ids of one configuration (rows rotate), "
+                                       "split over %d spawn workers" % (S, cores)},
+            "e2e": {"value": value, "unit": "masks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def cpu_baseline_sample(wl, seconds_target=15.0):
+    """Time the oracle on a bounded sample of the workload: whole rows split
+    across a spawn pool of all host cores; scaled to masks/s."""
+    import numpy as np
+    import multiprocessing as mp
+    from tests.harness import _init_worker, _oracle_rows
+    V = len(wl["tokens"])
+    cores = os.cpu_count() or 1
+    ctx = mp.get_context("spawn")
+    rng = np.random.default_rng(1)
+    n_ids = 24000
+    done = 0
+    with ctx.Pool(cores, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])) as pool:
+        pool.map(_oracle_rows, [(wl["prefixes"][0], wl["tokens"], wl["eos"], wl["specials"], [0])] * cores)
+        t0 = time.perf_counter()
+        rows = 0
+        while time.perf_counter() - t0 < seconds_target / cores * 2 and rows < 8:
+            ids = rng.choice(V, n_ids, replace=False)
+            parts = np.array_split(ids, cores * 2)
+            jobs = [(wl["prefixes"][rows % len(wl["prefixes"])], wl["tokens"], wl["eos"], wl["specials"],
+                     list(p)) for p in parts]
+            pool.map(_oracle_rows, jobs, chunksize=1)
+            done += n_ids
+            rows += 1
+        dt = time.perf_counter() - t0
+    return {"value": done / V / dt, "unit": "masks/s", "cores": cores, "kind": "oracle",
+            "sample": "%d rows x %d random token ids of the headline workload (%.1f s wall on %d spawn "
+                      "workers), scaled to full-vocabulary masks" % (rows, n_ids, dt, cores)}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--ref-tokens", type=int, default=8192)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    args.warmup = max(3, args.warmup)
+
+    import numpy as np
+    import torch
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if ws > 1 else 0)
+    torch.cuda.set_device(dev)
+
+    from paper_2607_11951_gb300 import grid as G
+    from workloads import configs
+    from tests.harness import unpack
+
+    # ---- inputs (seeded, synthetic) ----
+    batches = [configs.sql_select_only(prefix_seed=5000 + k) for k in range(N_BATCHES)]
+    wl = batches[0]
+    cpu_base = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu_base = cpu_baseline_sample(wl)
+    B, V = wl["B"], len(wl["tokens"])
+    W = (V + 31) // 32
+    grammar = G.Grammar(wl["grammar"], wl["role"], wl["lexicons"])
+    vocab = G.Vocab(wl["tokens"], wl["eos"], wl["specials"])
+    spec = G.Spec(grammar, vocab)
+    stream = torch.cuda.current_stream()
+    cfgs, toks = [], []
+    status = torch.zeros(B, dtype=torch.int32, device=dev)
+    mask = torch.zeros((B, W), dtype=torch.int32, device=dev)
+    rng = np.random.default_rng(42)
+    for k, bw in enumerate(batches):
+        c = G.Configs(spec, B)
+        n = max(len(p) for p in bw["prefixes"])
+        tt = np.full((B, n), -1, dtype=np.int32)
+        for i, p in enumerate(bw["prefixes"]):
+            tt[i, :len(p)] = p
+        G.grid_advance(spec.h, c.h, c.h, torch.from_numpy(tt).to(dev), status)
+        torch.cuda.synchronize()
+        assert (status.cpu().numpy() == 0).all(), status
+        G.grid_masks(spec.h, c.h, mask, status)
+        torch.cuda.synchronize()
+        assert (status.cpu().numpy() == 0).all(), status
+        bits = unpack(mask.cpu().numpy().view(np.uint32), V)
+        pick = np.array([rng.choice(np.nonzero(bits[i])[0]) for i in range(B)], dtype=np.int32)
+        cfgs.append(c)
+        toks.append(torch.from_numpy(pick).to(dev))
+    scratch = G.Configs(spec, B)
+    logits = [torch.from_numpy(configs.logits(100 + k, B, V)).to(dev) for k in range(N_BATCHES)]
+
+    def step(k, ev=None):
+        i = k % N_BATCHES
+        if ev:
+            ev[0].record()
+        G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
+        if ev:
+            ev[1].record()
+        G.grid_masks(spec.h, scratch.h, mask, status, stream)
+        if ev:
+            ev[2].record()
+        G.grid_apply_mask(mask, logits[i], stream)
+        if ev:
+            ev[3].record()
+
+    for k in range(args.warmup):
+        step(k)
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    clk = ClockSampler(local if ws > 1 else int(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or 0)
+                       if False else 0)
+    clk.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record()
+    for k in range(args.steps):
+        step(args.warmup + k, evs[k])
+    t_end.record()
+    torch.cuda.synchronize()
+    clocks = clk.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    if ws > 1:
+        tt = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(tt.item())
+        torch.distributed.barrier()
+    per_step = [e[0].elapsed_time(e[3]) * 1e3 for e in evs]
+    adv_us = statistics.mean(e[0].elapsed_time(e[1]) * 1e3 for e in evs)
+    masks_us = statistics.mean(e[1].elapsed_time(e[2]) * 1e3 for e in evs)
+    apply_us = statistics.mean(e[2].elapsed_time(e[3]) * 1e3 for e in evs)
+    per_step.sort()
+    p50 = per_step[len(per_step) // 2]
+    p99 = per_step[min(len(per_step) - 1, int(math.ceil(0.99 * len(per_step))) - 1)]
+    value = ws * B * args.steps / (total_ms / 1e3)
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        h_logits = [torch.from_numpy(configs.logits(100 + k, B, V)).pin_memory() for k in range(4)]
+        h_toks = [t.cpu().pin_memory() for t in toks]
+        h_mask = torch.empty((B, W), dtype=torch.int32).pin_memory()
+        h_status = torch.empty(B, dtype=torch.int32).pin_memory()
+        d_tok = torch.empty(B, dtype=torch.int32, device=dev)
+        d_logits = torch.empty((B, V), dtype=torch.float32, device=dev)
+
+        def e2e_step(k):
+            i = k % N_BATCHES
+            d_tok.copy_(h_toks[i], non_blocking=True)
+            d_logits.copy_(h_logits[k % 4], non_blocking=True)
+            G.grid_advance(spec.h, cfgs[i].h, scratch.h, d_tok, status, stream)
+            G.grid_masks(spec.h, scratch.h, mask, status, stream)
+            G.grid_apply_mask(mask, d_logits, stream)
+            h_mask.copy_(mask, non_blocking=True)
+            h_status.copy_(status, non_blocking=True)
+
+        for k in range(args.warmup):
+            e2e_step(k)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for k in range(args.steps):
+            e2e_step(k)
+        b.record()
+        torch.cuda.synchronize()
+        e_ms = a.elapsed_time(b)
+        if ws > 1:
+            tt = torch.tensor([e_ms], device=dev)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+            e_ms = float(tt.item())
+        e2e = {"value": ws * B * args.steps / (e_ms / 1e3), "unit": "masks/s",
+               "h2d_bytes_per_step": B * 4 + B * V * 4, "d2h_bytes_per_step": B * W * 4 + B * 4}
+
+    # ---- roofline of the mask-apply kernel (HBM-bound, write-mostly) ----
+    peak, peak_kind = _peaks()
+    apply_bytes = B * W * 4 + B * V * 4
+    roof = {"kernel": "k_apply (grid_apply_mask)", "bound": "hbm", "achieved": apply_bytes / (apply_us * 1e-6) / 1e9,
+            "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "traffic": None}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "masks/s", "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+                "config": {"workload": "sql_select_only", "B": B, "V": V, "prefix_tokens": "U[50,2000]",
+                           "schema": "200 tables x 30 columns", "logits": "f32 N(0,3)",
+                           "batches": N_BATCHES, "l2": "rotating inputs: 16 logits batches = 311 MB > L2",
+                           "step": "grid_advance + grid_masks + grid_apply_mask"},
+                "p50_us": p50, "p99_us": p99,
+                "token_checks_per_s": value * V,
+                "kernel_us": {"grid_advance": adv_us, "grid_masks": masks_us, "grid_apply_mask": apply_us},
+                "roofline": roof, "cpu_baseline": cpu_base, "e2e": e2e,
+                "gpu_launches": args.steps * 5, "clocks": clocks}
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

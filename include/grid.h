@@ -1,0 +1,215 @@
+/*
+ * grid.h -- C ABI of libgrid: GRID's cold full-vocabulary next-token mask on
+ * NVIDIA GB300 (sm_103a).
+ *
+ * GRID ("Grammar-Railed Decoding", arXiv 2607.11951) masks an LLM's logits so
+ * that every sampled token keeps the detokenized output a viable prefix of a
+ * role- and schema-projected LALR(1) language.  This library implements the
+ * paper's data-parallel hot path for a batch of B parser configurations:
+ *
+ *   grid_compile       grammar text + role projection + schema lexicons
+ *                      -> LALR(1) ACTION/GOTO, union lexer DFA, identifier trie
+ *                      (Sec. 2 "Three grammar layers"; Fig. 1 offline band)
+ *   grid_load_vocab    token byte strings -> DFS-ordered byte trie with alias
+ *                      classes (Def. 3)
+ *   grid_specialize    upload + per-lexer-state context-independent (CI) token
+ *                      classes (Sec. 4.2 CI/CD split), once per schema
+ *   grid_configs_create / grid_advance
+ *                      configurations kappa = (sigma, rho) (Def. 1) and the
+ *                      batched per-token parser step (Sec. 6.1 step 7)
+ *   grid_masks         M(kappa) for B configurations as a packed B x ceil(V/32)
+ *                      uint32 bitmask (Def. 4, Sec. 4.1-4.2, Sec. 3.2 EOS gate)
+ *   grid_apply_mask    logits <- -inf where the mask bit is 0 (Sec. 2,
+ *                      "Masked decoding": masked_fill_(-inf))
+ *
+ * Conventions
+ *   - Every call returns 0 (GRID_OK) or a negative GRID_E_* code; the message of
+ *     the last failure on the calling thread is available from grid_last_error.
+ *   - Handles (grid_grammar, grid_vocab, grid_spec, grid_configs) are opaque and
+ *     owned by the library; release them with the matching *_free call.
+ *   - Pointers named d_* are CUDA device pointers owned by the caller.
+ *     `stream` is a cudaStream_t passed as void*; NULL means the legacy default
+ *     stream.  Calls that take a stream only enqueue work: they never
+ *     synchronize and never allocate.  grid_specialize and
+ *     grid_configs_create allocate device memory and synchronize.
+ *   - Data-dependent failures are reported per row in a caller-supplied device
+ *     int32 array d_status[B] with the GRID_ST_* codes below; they never trap
+ *     and every device loop has a static bound.
+ *   - Mask layout: bit t of row b is (d_mask[b*W + (t>>5)] >> (t&31)) & 1,
+ *     W = ceil(V/32), LSB first.  Bits >= V, special tokens and (unless the EOS
+ *     gate passes) EOS are 0.
+ *
+ * Grammar text format (one declaration per line, '#' comment lines):
+ *   %token NAME "literal"   |  %token NAME /regex/    terminal; line order is the
+ *                                                     priority of the contextual pick
+ *   %ignore NAME /regex/                              ignored terminal (the set I)
+ *   %category NAME                                    L3 lexicon category (<= 32)
+ *   %start SYMBOL
+ *   lhs -> X Y Z [@tag]                               production; %empty = epsilon
+ * Regex syntax: literal bytes, escapes \n \t \r \xHH \<punct>, classes [...] with
+ * ranges and leading ^, ( ), |, and postfix * + ?.  At most 127 terminals.
+ *
+ * Lexing semantics (readings of Sec. 2 and Sec. 4.1): maximal munch over the
+ * regex union automaton; when a byte kills it, the pending lexeme r is emitted
+ * and its candidates are the terminals accepting r (a category c also needs
+ * r in W_c); the first candidate in priority order that is ignored or whose
+ * simulated reduce chain reaches SHIFT is taken; otherwise the byte is rejected.
+ * The killing byte is then fed from the start state.  The output is viable iff
+ * the trailing lexeme is live for an ignored or allowed terminal (category
+ * terminals also need r in Prefix(W_c)).
+ */
+#ifndef GRID_H
+#define GRID_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes ---- */
+#define GRID_OK 0
+#define GRID_E_INVALID_ARG (-1)          /* NULL handle, bad size, bad dtype            */
+#define GRID_E_PARSE (-2)                /* grammar text or regex does not parse        */
+#define GRID_E_LALR_CONFLICT (-3)        /* projected grammar is not LALR(1)            */
+#define GRID_E_EMPTY_LANGUAGE (-4)       /* L(G_role) is empty (Sec. 2, L2 check)       */
+#define GRID_E_LEXICON_NOT_IN_REGEX (-5) /* some w in W_c is not in R_c (Prop. 8 (d))   */
+#define GRID_E_LEXER_PRECONDITION (-6)   /* lexer not accept-closed or not delimited    */
+#define GRID_E_CUDA (-7)                 /* a CUDA runtime call failed                  */
+#define GRID_E_TOO_LARGE (-8)            /* a table exceeds a documented limit          */
+#define GRID_E_VOCAB (-9)                /* empty spelling, bad id, bad offsets         */
+
+/* ---- per-row device status codes (d_status) ---- */
+#define GRID_ST_OK 0
+#define GRID_ST_NONVIABLE 1         /* the configuration is not a viable prefix      */
+#define GRID_ST_STACK_OVERFLOW 2    /* a push would exceed max_depth                 */
+#define GRID_ST_TOKEN_NOT_ALLOWED 3 /* grid_advance got a token outside the mask      */
+#define GRID_ST_EMPTY_MASK 4        /* viable row with an empty mask: a bug (Prop. 8) */
+#define GRID_ST_BOUND 5             /* a per-token overlay or reduce-chain bound hit  */
+#define GRID_ST_COMPLETE 6          /* the row accepted EOS; its mask is all zero     */
+
+/* ---- logits dtypes for grid_apply_mask ---- */
+#define GRID_DTYPE_F32 0
+#define GRID_DTYPE_BF16 1
+
+typedef struct grid_grammar grid_grammar;
+typedef struct grid_vocab grid_vocab;
+typedef struct grid_spec grid_spec;
+typedef struct grid_configs grid_configs;
+
+/* One L3 lexicon: the allowed words W_c of category terminal `category`
+ * (Sec. 2, L3).  Word i is words[offsets[i] .. offsets[i+1]); host memory,
+ * read during the call only. */
+typedef struct grid_lexicon {
+  const char* category;
+  const uint8_t* words;
+  const int64_t* offsets; /* n_words + 1 entries, non-decreasing, offsets[0] = 0 */
+  int32_t n_words;
+} grid_lexicon;
+
+typedef struct grid_options {
+  int32_t max_depth; /* stack capacity D per configuration (default 4096)          */
+  int32_t reserved[7];
+} grid_options;
+
+/* Thread-local message of the last failure on this thread; copies at most n-1
+ * bytes plus a NUL into buf and returns the full message length. */
+size_t grid_last_error(char* buf, size_t n);
+
+/* Sec. 2 (L1/L2/L3) and Fig. 1: parse `grammar_text`, keep the productions that
+ * are untagged or whose tag is in the comma-separated `role_keep` list
+ * (role_keep == NULL keeps every production), eliminate useless symbols, check
+ * L(G_role) is non-empty, build the LALR(1) tables, the minimised union lexer
+ * DFA and the identifier trie of the `n_lex` lexicons, and validate the
+ * preconditions: W_c subset of R_c, an accept-closed lexer (no live
+ * non-accepting state after an accepting one) and blank-delimited lexemes
+ * (0x20 kills every accepting state of a non-ignored terminal, and some ignored
+ * terminal accepts 0x20).  Host-only: touches no GPU.  `opt` may be NULL.
+ * On success *out owns the grammar; free with grid_grammar_free. */
+int grid_compile(const char* grammar_text, size_t len, const char* role_keep,
+                 const grid_lexicon* lex, int32_t n_lex, const grid_options* opt,
+                 grid_grammar** out);
+void grid_grammar_free(grid_grammar* g);
+
+/* Table sizes of a compiled grammar: out[0]=terminals incl. $end, out[1]=LALR
+ * states, out[2]=nonterminals, out[3]=productions, out[4]=DFA states,
+ * out[5]=byte classes, out[6]=lexicon-trie nodes, out[7]=categories. */
+int grid_grammar_info(const grid_grammar* g, int64_t out[8]);
+
+/* Def. 3: build the DFS-ordered byte trie of the vocabulary.  Token t has the
+ * spelling bytes[offsets[t] .. offsets[t+1]) (host memory, read during the call).
+ * `eos_id` and the `n_special` ids in `special_ids` are excluded from the trie
+ * and permanently masked (EOS is set only by the EOS gate).  Distinct ids with
+ * equal spellings form alias classes and always get equal bits.  An empty
+ * spelling of a non-special id is GRID_E_VOCAB.  Host-only.  *out owns the
+ * vocabulary; free with grid_vocab_free. */
+int grid_load_vocab(const uint8_t* bytes, const int64_t* offsets, int32_t V, int32_t eos_id,
+                    const int32_t* special_ids, int32_t n_special, grid_vocab** out);
+void grid_vocab_free(grid_vocab* v);
+
+/* Vocabulary facts: out[0]=V, out[1]=distinct spellings in the trie,
+ * out[2]=1 if all 256 single-byte spellings are present (byte-complete,
+ * Prop. 8 (a)), out[3]=total spelling bytes. */
+int grid_vocab_info(const grid_vocab* v, int64_t out[4]);
+
+/* Sec. 4.2 + Sec. 8 (cold-schema specialization): upload grammar and
+ * vocabulary tables to the current CUDA device and precompute, for every state
+ * of the lexer DFA, the context-independent class of every spelling (the
+ * spellings whose verdict is a function of the allowed-terminal set alone).
+ * The grammar and vocabulary must outlive the spec.  Allocates device memory,
+ * runs kernels on `stream` and synchronizes it.  *out owns the device tables;
+ * free with grid_spec_free. */
+int grid_specialize(const grid_grammar* g, const grid_vocab* v, void* stream, grid_spec** out);
+void grid_spec_free(grid_spec* s);
+
+/* Create B configurations, all at the start configuration (empty output),
+ * with the device scratch that grid_masks needs for B rows.  Allocates device
+ * memory and synchronizes.  Free with grid_configs_free. */
+int grid_configs_create(const grid_spec* s, int32_t B, grid_configs** out);
+void grid_configs_free(grid_configs* c);
+
+/* Reset every row of `c` to the start configuration (enqueued on `stream`). */
+int grid_configs_reset(const grid_spec* s, grid_configs* c, void* stream);
+
+/* Sec. 6.1 step 7: per row b, feed the tokens d_tokens[b*n_steps + k],
+ * k = 0..n_steps-1, in order (a negative id is a no-op).  Each token must be in
+ * the row's current mask: its bytes go through the lexer (maximal munch,
+ * parser-viable pick) and the emitted terminals are shifted/reduced on the
+ * row's stack; EOS (when the gate passes) completes the row.  `in` and `out`
+ * may be the same object (in place) or two configurations of the same B
+ * (out-of-place: `in` is not modified).  On a token outside the mask the row
+ * keeps its configuration as of the last accepted token and d_status[b] =
+ * GRID_ST_TOKEN_NOT_ALLOWED (also for out-of-range ids and special tokens);
+ * a full stack gives GRID_ST_STACK_OVERFLOW; a completed row gives
+ * GRID_ST_COMPLETE.  Enqueue only. */
+int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
+                 const int32_t* d_tokens, int32_t n_steps, int32_t* d_status, void* stream);
+
+/* Def. 4: write M(kappa_b) for every row of `c` into d_mask[B][W] (device,
+ * W = ceil(V/32), 4-byte aligned).  A viable row whose mask would be empty gets
+ * GRID_ST_EMPTY_MASK; a completed row gets an all-zero mask and
+ * GRID_ST_COMPLETE.  Uses the scratch held by `c`, so calls on the same
+ * configurations object must not overlap on the GPU.  Enqueue only. */
+int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
+               void* stream);
+
+/* Sec. 2 masked decoding: for b < B, t < V, set d_logits[b*row_stride + t] to
+ * -inf (fp32 0xFF800000 / bf16 0xFF80) where mask bit t of row b is 0; accepted
+ * values are left bit-identical.  d_logits is device memory of `dtype`
+ * (GRID_DTYPE_F32 or GRID_DTYPE_BF16); row_stride >= V elements.  In place,
+ * enqueue only. */
+int grid_apply_mask(const uint32_t* d_mask, void* d_logits, int32_t dtype, int32_t B, int32_t V,
+                    int64_t row_stride, void* stream);
+
+/* Debug/test view of row `row` (synchronous device-to-host copy): the stack
+ * (up to `cap` entries, bottom first), its depth, the lexer DFA state and
+ * lexicon-trie node of the pending lexeme, and flags (bit 0 = complete). */
+int grid_configs_export(const grid_configs* c, int32_t row, int32_t* stack, int32_t cap,
+                        int32_t* depth, int32_t* dfa_state, int32_t* lex_node, int32_t* flags);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GRID_H */

@@ -1,0 +1,285 @@
+"""Thin ctypes binding of libgrid (include/grid.h).
+
+Argument marshalling only: every step of the mask path runs in the CUDA
+library.  Functions keep the C names; the small classes own the opaque handles
+and free them.  Device buffers are torch CUDA tensors (masks are int32 tensors
+holding the uint32 words); streams default to torch's current stream.  If the
+shared library has not been built, every call raises ``GridLibraryMissing``:
+there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from .build import library_path
+
+GRID_OK = 0
+GRID_ST = {0: "OK", 1: "NONVIABLE", 2: "STACK_OVERFLOW", 3: "TOKEN_NOT_ALLOWED",
+           4: "EMPTY_MASK", 5: "BOUND", 6: "COMPLETE"}
+GRID_ST_OK, GRID_ST_NONVIABLE, GRID_ST_STACK_OVERFLOW, GRID_ST_TOKEN_NOT_ALLOWED = 0, 1, 2, 3
+GRID_ST_EMPTY_MASK, GRID_ST_BOUND, GRID_ST_COMPLETE = 4, 5, 6
+GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
+
+EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
+            "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
+            "grid_spec_free", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
+            "grid_advance", "grid_masks", "grid_apply_mask", "grid_configs_export"]
+
+
+class GridLibraryMissing(RuntimeError):
+    pass
+
+
+class GridError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__("libgrid error %d: %s" % (code, msg))
+        self.code = code
+
+
+class _Lexicon(ctypes.Structure):
+    _fields_ = [("category", ctypes.c_char_p), ("words", ctypes.c_void_p),
+                ("offsets", ctypes.c_void_p), ("n_words", ctypes.c_int32)]
+
+
+class _Options(ctypes.Structure):
+    _fields_ = [("max_depth", ctypes.c_int32), ("reserved", ctypes.c_int32 * 7)]
+
+
+_lib = None
+
+
+def lib():
+    """Load the in-tree libgrid.so (built by ``__graft_entry__.build()``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = library_path()
+    if not os.path.exists(path):
+        raise GridLibraryMissing("libgrid.so not built at %s: run __graft_entry__.build()" % path)
+    L = ctypes.CDLL(path)
+    P, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+    sig = {
+        "grid_last_error": (SZ, [ctypes.c_char_p, SZ]),
+        "grid_compile": (I32, [ctypes.c_char_p, SZ, ctypes.c_char_p, P, I32, P, ctypes.POINTER(P)]),
+        "grid_grammar_free": (None, [P]),
+        "grid_grammar_info": (I32, [P, ctypes.POINTER(I64)]),
+        "grid_load_vocab": (I32, [P, P, I32, I32, P, I32, ctypes.POINTER(P)]),
+        "grid_vocab_free": (None, [P]),
+        "grid_vocab_info": (I32, [P, ctypes.POINTER(I64)]),
+        "grid_specialize": (I32, [P, P, P, ctypes.POINTER(P)]),
+        "grid_spec_free": (None, [P]),
+        "grid_configs_create": (I32, [P, I32, ctypes.POINTER(P)]),
+        "grid_configs_free": (None, [P]),
+        "grid_configs_reset": (I32, [P, P, P]),
+        "grid_advance": (I32, [P, P, P, P, I32, P, P]),
+        "grid_masks": (I32, [P, P, P, P, P]),
+        "grid_apply_mask": (I32, [P, P, I32, I32, I32, I64, P]),
+        "grid_configs_export": (I32, [P, I32, P, I32, P, P, P, P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(L, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = L
+    return L
+
+
+def last_error() -> str:
+    buf = ctypes.create_string_buffer(4096)
+    lib().grid_last_error(buf, 4096)
+    return buf.value.decode(errors="replace")
+
+
+def _check(rc):
+    if rc != GRID_OK:
+        raise GridError(rc, last_error())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _pack(items):
+    """list of bytes -> (contiguous buffer, int64 offsets) kept alive by the caller."""
+    data = b"".join(items)
+    offs = [0]
+    for it in items:
+        offs.append(offs[-1] + len(it))
+    buf = ctypes.create_string_buffer(data, max(1, len(data)))
+    arr = (ctypes.c_int64 * len(offs))(*offs)
+    return buf, arr
+
+
+# ---------------------------------------------------------------------------
+def grid_compile(text: str, role_keep=None, lexicons=None, max_depth: int = 4096):
+    """Returns a grid_grammar handle (c_void_p).  ``role_keep`` is None (all
+    productions) or a list of kept production tags; ``lexicons`` maps a
+    category terminal name to its word list."""
+    L = lib()
+    raw = text.encode()
+    keep = None if role_keep is None else ",".join(role_keep).encode()
+    lex = lexicons or {}
+    arr = (_Lexicon * max(1, len(lex)))()
+    keep_alive = []
+    for i, (cat, words) in enumerate(lex.items()):
+        ws = [w if isinstance(w, bytes) else w.encode() for w in words]
+        buf, offs = _pack(ws)
+        c = cat.encode()
+        keep_alive += [buf, offs, c]
+        arr[i].category = c
+        arr[i].words = ctypes.cast(buf, ctypes.c_void_p)
+        arr[i].offsets = ctypes.cast(offs, ctypes.c_void_p)
+        arr[i].n_words = len(ws)
+    opt = _Options(max_depth, (ctypes.c_int32 * 7)())
+    out = ctypes.c_void_p()
+    _check(L.grid_compile(raw, len(raw), keep, ctypes.cast(arr, ctypes.c_void_p), len(lex),
+                          ctypes.byref(opt), ctypes.byref(out)))
+    return out
+
+
+def grid_grammar_info(g):
+    out = (ctypes.c_int64 * 8)()
+    _check(lib().grid_grammar_info(g, out))
+    keys = ["terminals", "lalr_states", "nonterminals", "productions", "dfa_states",
+            "byte_classes", "lexicon_nodes", "categories"]
+    return dict(zip(keys, list(out)))
+
+
+def grid_load_vocab(tokens, eos: int, specials=()):
+    L = lib()
+    buf, offs = _pack(tokens)
+    sp = (ctypes.c_int32 * max(1, len(specials)))(*specials)
+    out = ctypes.c_void_p()
+    _check(L.grid_load_vocab(ctypes.cast(buf, ctypes.c_void_p), ctypes.cast(offs, ctypes.c_void_p),
+                             len(tokens), eos, ctypes.cast(sp, ctypes.c_void_p), len(specials),
+                             ctypes.byref(out)))
+    return out
+
+
+def grid_vocab_info(v):
+    out = (ctypes.c_int64 * 4)()
+    _check(lib().grid_vocab_info(v, out))
+    return dict(zip(["V", "spellings", "byte_complete", "bytes"], list(out)))
+
+
+def grid_specialize(g, v, stream=None):
+    out = ctypes.c_void_p()
+    _check(lib().grid_specialize(g, v, _stream(stream), ctypes.byref(out)))
+    return out
+
+
+def grid_configs_create(spec, B: int):
+    out = ctypes.c_void_p()
+    _check(lib().grid_configs_create(spec, B, ctypes.byref(out)))
+    return out
+
+
+def grid_configs_reset(spec, cfg, stream=None):
+    _check(lib().grid_configs_reset(spec, cfg, _stream(stream)))
+
+
+def grid_advance(spec, cin, cout, tokens, status, stream=None):
+    """tokens: int32 CUDA tensor [B] or [B, n_steps]; status: int32 CUDA tensor [B]."""
+    n = 1 if tokens.dim() == 1 else tokens.shape[1]
+    assert tokens.is_contiguous() and status.is_contiguous()
+    _check(lib().grid_advance(spec, cin, cout, _ptr(tokens), n, _ptr(status), _stream(stream)))
+
+
+def grid_masks(spec, cfg, mask, status, stream=None):
+    """mask: int32 CUDA tensor [B, ceil(V/32)] (uint32 words); status: int32 [B]."""
+    assert mask.is_contiguous() and status.is_contiguous()
+    _check(lib().grid_masks(spec, cfg, _ptr(mask), _ptr(status), _stream(stream)))
+
+
+def grid_apply_mask(mask, logits, stream=None):
+    """In place on a float32 or bfloat16 CUDA tensor [B, >=V] (row stride = stride(0))."""
+    import torch
+    dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
+    B, V = logits.shape
+    assert logits.stride(1) == 1
+    _check(lib().grid_apply_mask(_ptr(mask), _ptr(logits), dt, B, V, logits.stride(0), _stream(stream)))
+
+
+def grid_apply_mask_raw(mask, logits_ptr: int, dtype: int, B: int, V: int, row_stride: int, stream=None):
+    _check(lib().grid_apply_mask(_ptr(mask), ctypes.c_void_p(logits_ptr), dtype, B, V, row_stride,
+                                 _stream(stream)))
+
+
+def grid_configs_export(cfg, row: int, cap: int = 1 << 16):
+    stack = (ctypes.c_int32 * cap)()
+    d, q, lx, fl = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    _check(lib().grid_configs_export(cfg, row, stack, cap, ctypes.byref(d), ctypes.byref(q),
+                                     ctypes.byref(lx), ctypes.byref(fl)))
+    return dict(stack=list(stack[:min(d.value, cap)]), depth=d.value, dfa_state=q.value,
+                lex_node=lx.value, flags=fl.value)
+
+
+# ---------------------------------------------------------------------------
+class Grammar:
+    def __init__(self, text, role_keep=None, lexicons=None, max_depth=4096):
+        self.h = grid_compile(text, role_keep, lexicons, max_depth)
+
+    def info(self):
+        return grid_grammar_info(self.h)
+
+    def __del__(self):
+        if getattr(self, "h", None) and _lib is not None:
+            _lib.grid_grammar_free(self.h)
+            self.h = None
+
+
+class Vocab:
+    def __init__(self, tokens, eos, specials=()):
+        self.V = len(tokens)
+        self.eos = eos
+        self.h = grid_load_vocab(tokens, eos, specials)
+
+    def info(self):
+        return grid_vocab_info(self.h)
+
+    def __del__(self):
+        if getattr(self, "h", None) and _lib is not None:
+            _lib.grid_vocab_free(self.h)
+            self.h = None
+
+
+class Spec:
+    """(grammar, vocabulary) tables on the device plus the CI classes."""
+
+    def __init__(self, grammar: Grammar, vocab: Vocab, stream=None):
+        self.grammar, self.vocab = grammar, vocab
+        self.V = vocab.V
+        self.W = (vocab.V + 31) // 32
+        self.h = grid_specialize(grammar.h, vocab.h, stream)
+
+    def __del__(self):
+        if getattr(self, "h", None) and _lib is not None:
+            _lib.grid_spec_free(self.h)
+            self.h = None
+
+
+class Configs:
+    def __init__(self, spec: Spec, B: int):
+        self.spec, self.B = spec, B
+        self.h = grid_configs_create(spec.h, B)
+
+    def reset(self, stream=None):
+        grid_configs_reset(self.spec.h, self.h, stream)
+
+    def export(self, row):
+        return grid_configs_export(self.h, row)
+
+    def __del__(self):
+        if getattr(self, "h", None) and _lib is not None:
+            _lib.grid_configs_free(self.h)
+            self.h = None

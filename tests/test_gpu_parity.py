@@ -1,0 +1,209 @@
+"""CUDA path vs oracle, bit-exact (Def. 4 masks, EOS gate, masked logits).
+
+Every test calls the library through the C ABI binding on the same seeded
+inputs as the oracle.  Masks are integer results: the bar is bit equality.
+"""
+import numpy as np
+import pytest
+
+from tests.harness import GpuRun, oracle_masks, oracle_masks_split, unpack
+from workloads import configs
+
+pytestmark = pytest.mark.gpu
+
+_runs = {}
+
+
+def _run(name, fn):
+    if name not in _runs:
+        wl = fn()
+        run = GpuRun(wl)
+        st = run.build_configs()
+        assert (st == 0).all(), ("grid_advance status", st)
+        _runs[name] = (wl, run)
+    return _runs[name]
+
+
+def _compare_full(wl, run, rows=None, split=False):
+    words, status = run.masks()
+    assert (status == 0).all(), ("grid_masks status", status)
+    bits = unpack(words, run.V)
+    rows = list(range(run.B)) if rows is None else rows
+    want = oracle_masks_split(wl, rows) if split else oracle_masks(wl, rows)
+    for k, r in enumerate(rows):
+        assert want[k] is not None, ("oracle rejects prefix", r)
+        w = np.asarray(want[k], dtype=np.uint8)
+        diff = np.nonzero(bits[r] != w)[0]
+        assert diff.size == 0, ("row", r, "ids", diff[:10].tolist(),
+                                [wl["tokens"][i] for i in diff[:5]], "gpu", bits[r][diff[:5]].tolist())
+    # padding bits beyond V are zero
+    W = words.shape[1]
+    if W * 32 > run.V:
+        pad = words[:, -1] >> np.uint32(run.V - (W - 1) * 32)
+        assert (pad == 0).all()
+    return bits
+
+
+def test_tiny_expr_full_parity():
+    wl, run = _run("tiny", configs.tiny_expr)
+    _compare_full(wl, run)
+
+
+def test_sql_admin_full_parity():
+    wl, run = _run("admin", configs.sql_admin)
+    _compare_full(wl, run, split=True)
+
+
+def test_sql_select_only_full_parity():
+    wl, run = _run("headline", configs.sql_select_only)
+    bits = _compare_full(wl, run, split=True)
+    # the headline batch is not degenerate: every row admits something, EOS never
+    assert bits.sum(axis=1).min() > 0
+
+
+@pytest.mark.parametrize("n,depth", [(100, 1), (100, 64), (1000, 8), (16000, 1), (16000, 64)])
+def test_sweep_cells_sampled(n, depth):
+    """Flatness sweep cells at full size: per row, 2,000 random ids plus up to
+    2,000 GPU-admitted ids are recomputed one by one by the oracle."""
+    wl = configs.sql_sweep_cell(n, depth)
+    run = GpuRun(wl)
+    st = run.build_configs()
+    assert (st == 0).all(), st
+    words, status = run.masks()
+    assert (status == 0).all(), status
+    bits = unpack(words, run.V)
+    rng = np.random.default_rng(n + depth)
+    rows = list(range(0, run.B, 4))
+    ids = []
+    for r in rows:
+        adm = np.nonzero(bits[r])[0]
+        pick = np.concatenate([rng.choice(run.V, 2000, replace=False),
+                               rng.choice(adm, min(2000, adm.size), replace=False) if adm.size else []])
+        ids.append(np.unique(pick.astype(np.int64)))
+    want = oracle_masks(wl, rows, ids)
+    for k, r in enumerate(rows):
+        assert want[k] is not None
+        got = bits[r][ids[k]]
+        w = np.asarray(want[k], dtype=np.uint8)
+        assert (got == w).all(), (n, depth, r, ids[k][np.nonzero(got != w)[0][:10]])
+
+
+def test_cold_schema_rows_full_parity():
+    """Cold-schema workload (B=256, 50k identifiers): full masks of 16 rows."""
+    wl, run = _run("cold", configs.sql_cold_schema)
+    words, status = run.masks()
+    assert (status == 0).all(), status
+    bits = unpack(words, run.V)
+    rows = list(range(0, 256, 16))
+    want = oracle_masks_split(wl, rows)
+    for k, r in enumerate(rows):
+        assert want[k] is not None
+        diff = np.nonzero(bits[r] != np.asarray(want[k], dtype=np.uint8))[0]
+        assert diff.size == 0, (r, diff[:10].tolist())
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_masked_logits_bit_exact(dtype):
+    """grid_apply_mask: rejected -> -inf, accepted values bit-identical (incl.
+    NaN payloads); strided rows."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl, run = _run("headline", configs.sql_select_only)
+    run.masks()
+    bits = torch.from_numpy(unpack(run.mask.cpu().numpy().view(np.uint32), run.V).astype(bool))
+    lg = torch.from_numpy(configs.logits(7, run.B, run.V))
+    lg[0, :7] = float("nan")
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    for stride in (run.V, run.V + 8):
+        buf = torch.zeros(run.B, stride, dtype=tdt)
+        buf[:, :run.V] = lg.to(tdt)
+        ref = buf.clone()
+        ref[:, :run.V] = torch.where(bits, buf[:, :run.V], torch.tensor(float("-inf"), dtype=tdt))
+        d = buf.cuda()
+        view = d[:, :run.V]
+        G.grid_apply_mask(run.mask, view)
+        torch.cuda.synchronize()
+        got = d.cpu()
+        iv = torch.int32 if dtype == "f32" else torch.int16
+        assert torch.equal(got.view(iv), ref.view(iv))
+
+
+def test_advance_semantics_and_status():
+    """Out-of-place advance leaves its input alone; a token outside the mask,
+    an out-of-range id and a special id give TOKEN_NOT_ALLOWED and keep the
+    row; EOS at a sentence completes the row (all-zero mask, COMPLETE)."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl, run = _run("admin", configs.sql_admin)
+    words0, _ = run.masks()
+    bits0 = unpack(words0, run.V)
+    out = G.Configs(run.spec, run.B)
+    B = run.B
+    rng = np.random.default_rng(3)
+    tok = np.zeros(B, dtype=np.int32)
+    kinds = []
+    for b in range(B):
+        adm = np.nonzero(bits0[b])[0]
+        rej = np.nonzero(bits0[b] == 0)[0]
+        k = b % 4
+        kinds.append(k)
+        if k == 0:
+            tok[b] = rng.choice(adm)
+        elif k == 1:
+            tok[b] = rng.choice(rej[rej != wl["eos"]])
+        elif k == 2:
+            tok[b] = run.V + 5
+        else:
+            tok[b] = wl["specials"][0]
+    st = torch.zeros(B, dtype=torch.int32, device="cuda")
+    G.grid_advance(run.spec.h, run.cfg.h, out.h, torch.from_numpy(tok).cuda(), st)
+    torch.cuda.synchronize()
+    st = st.cpu().numpy()
+    for b in range(B):
+        assert st[b] == (0 if kinds[b] == 0 else 3), (b, kinds[b], st[b])
+    # input unchanged
+    words1, _ = run.masks()
+    assert (words1 == words0).all()
+    # rejected rows of `out` equal their input; accepted rows match the oracle
+    words2, s2 = run.masks(out)
+    bits2 = unpack(words2, run.V)
+    from oracle import compile_grammar
+    og = compile_grammar(wl["grammar"], wl["role"], wl["lexicons"])
+    for b in range(0, B, 3):
+        if kinds[b] != 0:
+            assert (bits2[b] == bits0[b]).all()
+        else:
+            cfg = og.config_from_ids(list(wl["prefixes"][b]) + [int(tok[b])], wl["tokens"], wl["eos"], wl["specials"])
+            want = np.asarray(og.mask(cfg, wl["tokens"], wl["eos"], wl["specials"]), dtype=np.uint8)
+            assert (bits2[b] == want).all(), b
+
+
+def test_eos_completes_row_and_empty_prefix():
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    from workloads.gen import GreedyTokenizer
+    wl = configs.tiny_expr(B=4)
+    tk = GreedyTokenizer(wl["tokens"], [wl["eos"]])
+    wl["prefixes"] = [tk.encode(b"a+1"), [], tk.encode(b"(a"), tk.encode(b"1 ")]
+    run = GpuRun(wl)
+    assert (run.build_configs() == 0).all()
+    words, status = run.masks()
+    bits = unpack(words, run.V)
+    eos = wl["eos"]
+    assert bits[0][eos] == 1 and bits[1][eos] == 0 and bits[2][eos] == 0 and bits[3][eos] == 1
+    toks = torch.tensor([eos, eos, eos, -1], dtype=torch.int32, device="cuda")
+    st = torch.zeros(4, dtype=torch.int32, device="cuda")
+    G.grid_advance(run.spec.h, run.cfg.h, run.cfg.h, toks, st)
+    torch.cuda.synchronize()
+    assert st.cpu().tolist() == [0, 3, 3, 0]
+    words, status = run.masks()
+    assert status.tolist()[0] == G.GRID_ST_COMPLETE and (words[0] == 0).all()
+    assert status.tolist()[1:] == [0, 0, 0]
+
+
+def test_ragged_vocab_tail_and_single_row():
+    """V not a multiple of 32, B = 1, alias spellings."""
+    wl = configs.tiny_expr(B=1, V=517)
+    run = GpuRun(wl)
+    assert (run.build_configs() == 0).all()
+    _compare_full(wl, run)

@@ -1,0 +1,119 @@
+"""CPU-only checks of libgrid: the shared library loads, exports every symbol
+that include/grid.h declares, and its host-side compiler reports the
+documented errors (no GPU call is made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_11951_gb300 import grid as G
+from workloads import grammar_text
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not os.path.exists(G.library_path()):
+        import paper_2607_11951_gb300 as pkg
+        pkg.build()
+    G.lib()
+
+
+def _declared():
+    text = open(os.path.join(ROOT, "include", "grid.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:int|void|size_t)\s+(grid_[a-z_]+)\s*\(", text, re.M)))
+
+
+def test_exports_every_declared_symbol():
+    names = _declared()
+    assert len(names) >= 16
+    L = ctypes.CDLL(G.library_path())
+    for n in names:
+        assert hasattr(L, n), n
+    assert sorted(G.EXPORTED) == sorted(n for n in names if n in G.EXPORTED)
+
+
+def _err(text, role=None, lex=None):
+    with pytest.raises(G.GridError) as e:
+        G.Grammar(text, role, lex)
+    return e.value.code
+
+
+def test_compile_ok_and_sizes():
+    g = G.Grammar(grammar_text("sql"), [], {"TABLE_NAME": ["t1"], "COLUMN_NAME": ["c1"]})
+    info = g.info()
+    assert info["terminals"] == 60 and info["categories"] == 2 and info["lalr_states"] > 50
+    g2 = G.Grammar(grammar_text("sql"), ["dml"], {"TABLE_NAME": ["t1"], "COLUMN_NAME": ["c1"]})
+    assert g2.info()["lalr_states"] > info["lalr_states"]  # projection removed DML states
+
+
+def test_lalr_conflict_detected():
+    # LR(1) but not LALR(1): merging the two 'c' states gives a reduce/reduce conflict
+    text = """%token A "a"
+%token B "b"
+%token C "c"
+%token D "d"
+%token E "e"
+%ignore WS /[ ]+/
+%start s
+s -> A x D
+s -> B y D
+s -> A y E
+s -> B x E
+x -> C
+y -> C
+"""
+    assert _err(text) == -3
+    # the same grammar with one pair removed is LALR(1)
+    ok = text.replace("s -> B x E\n", "")
+    G.Grammar(ok)
+
+
+def test_empty_language_and_projection():
+    text = """%token A "a"
+%ignore WS /[ ]+/
+%start s
+s -> A @r
+"""
+    assert _err(text, role=[]) == -4
+    G.Grammar(text, role_keep=["r"])
+
+
+def test_lexicon_not_in_regex():
+    assert _err(grammar_text("sql"), [], {"TABLE_NAME": ["Official_ratings_(millions)"], "COLUMN_NAME": []}) == -5
+
+
+def test_lexer_preconditions():
+    # "ab" accepting, "abc" live but not accepting, "abcd" accepting: not accept-closed
+    text = """%token X "ab"
+%token Y "abcd"
+%ignore WS /[ ]+/
+%start s
+s -> X
+s -> Y
+"""
+    assert _err(text) == -6
+    # a blank extends a non-ignored lexeme: not blank-delimited
+    text2 = """%token X /a[ a]*/
+%ignore WS /[ ]+/
+%start s
+s -> X
+"""
+    assert _err(text2) == -6
+
+
+def test_parse_errors():
+    assert _err("%token A \"a\"\n%ignore WS /[ ]+/\n%start s\ns -> B\n") == -2
+    assert _err("%token A /(a/\n%ignore WS /[ ]+/\n%start s\ns -> A\n") == -2
+
+
+def test_vocab_errors_and_info():
+    v = G.Vocab([bytes([b]) for b in range(256)] + [b"ab", b"ab", b"<eos>"], 258)
+    info = v.info()
+    assert info["spellings"] == 257 and info["byte_complete"] == 1
+    with pytest.raises(G.GridError):
+        G.Vocab([b"a", b"", b"<eos>"], 2)
+    with pytest.raises(G.GridError):
+        G.Vocab([b"a", b"<eos>"], 5)

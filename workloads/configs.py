@@ -34,6 +34,13 @@ def _sql_vocab_cached(V: int, seed: int, multiword: float):
     return _cache[key]
 
 
+def _tokenizer_cached(V, toks, exclude):
+    key = ("tok", V, len(toks), toks[0], toks[-2])
+    if key not in _cache:
+        _cache[key] = GreedyTokenizer(toks, exclude)
+    return _cache[key]
+
+
 def tiny_expr(seed: int = 1001, B: int = 64, V: int = 512):
     """Expression grammar, V=512 vocab over [a-z0-9+*() ], 64 prefixes truncated
     at a uniformly random byte offset of a random derivation (nesting <= 8)."""
@@ -92,15 +99,15 @@ def sql_admin(seed: int = 1002, B: int = 32, V: int = SQL_V_ADMIN):
 
 
 def sql_select_only(seed: int = 1003, B: int = 32, V: int = SQL_V_HEADLINE,
-                    lo: int = 50, hi: int = 2000):
+                    lo: int = 50, hi: int = 2000, prefix_seed: int | None = None):
     """Headline workload: SQL grammar under the SELECT-only projection (DML
     productions removed), schema 200 x 30, V=151,936 with ~3% multi-word tokens,
     B=32 prefixes of U[50,2000] tokens, fp32 logits N(0,3)."""
     kws = grammar_keywords(grammar_text("sql"))
     tables, cols, words = make_schema(seed, 200, 30, kws, col_pool=3000)
     toks, eos, specials = _sql_vocab_cached(V, 1003, 0.03)
-    tk = GreedyTokenizer(toks, specials + [eos])
-    rng = np.random.default_rng(seed + 1)
+    tk = _tokenizer_cached(V, toks, specials + [eos])
+    rng = np.random.default_rng(seed + 1 if prefix_seed is None else prefix_seed)
     lens = [int(x) for x in rng.integers(lo, hi + 1, size=B)]
     prefixes, texts = _sql_prefixes(rng, SqlGen(rng, tables, cols, dml=False), tk, lens)
     return dict(name="sql_select_only", grammar=grammar_text("sql"), role=[],
