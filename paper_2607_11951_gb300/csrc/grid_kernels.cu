@@ -1,36 +1,44 @@
-// libgrid device side for sm_103a: table upload, configurations, and the
-// kernels of the cold full-vocabulary mask.
+// libgrid device side for sm_103a: table upload, CI precompute, configurations
+// and the kernels of the cold full-vocabulary mask.
 //
-//   k_reset    configurations <- start configuration (Def. 1)
-//   k_prep     per row: allowed terminals A(sigma) by reduce-chain simulation,
-//              the EOS gate (Sec. 3.2), and clearing of the row's scratch
-//   k_walk     per (row, spelling range): walk every token's bytes through the
-//              lexer DFA and the identifier trie; each emission picks the
-//              highest-priority parser-viable candidate and is shifted on a
-//              per-lane copy-on-write overlay over the row's read-only stack;
-//              rejected prefixes skip their whole trie subtree (Sec. 4.1)
-//   k_pack     spelling-order verdict bits -> id-order mask words with alias
-//              expansion, EOS bit, special tokens zero, empty-mask status
-//   k_advance  per row: feed sampled tokens, commit shifts/reduces (Sec. 6.1)
-//   k_apply    logits <- -inf where the mask bit is 0 (Sec. 2)
+// Specialization (grid_specialize, Sec. 4.2 / cold-schema specialization):
+//   k_classify  per (precomputed lexer state, spelling): CI class id, or
+//               always/never viable, or CD (context-dependent)
+//   k_compact   per lexer state: the ascending list of its CD spellings
+//   k_permute   class tables re-indexed by token id (coalesced in k_pack)
 //
-// Every loop is bounded; a bound that is hit writes GRID_ST_BOUND and the
-// token is counted as rejected.  No kernel traps.
+// Mask step (grid_masks, Def. 4):
+//   k_prep   one warp per row: A0 = A(sigma) by reduce-chain simulation; the
+//            forced emission of the pending lexeme (what every token whose first
+//            byte ends the lexeme must go through) -> sigma' and A1 = A(sigma');
+//            EOS gate (Sec. 3.2); class selections of both contexts; the
+//            first-byte ranges that continue the pending lexeme
+//   k_walk   CD spellings only: lanes walk token bytes through the DFA and the
+//            identifier trie, emissions pick the highest-priority parser-viable
+//            candidate on a copy-on-write overlay; a rejected prefix skips its
+//            whole trie subtree (Sec. 4.1)
+//   k_pack   per token id: CI class lookup | walked verdict | EOS gate, packed
+//            into the id-order mask (alias classes expand automatically)
+// Parser step (grid_advance):  k_advance.   Masked logits:  k_apply.
+//
+// Every loop is bounded; hitting a bound writes GRID_ST_BOUND.  No kernel traps.
 
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstring>
 #include <string>
 #include <vector>
 
-#include "grid_internal.h"
+#include "grid_device.cuh"
 
 namespace grid {
 namespace {
 
-constexpr int kMaxOvl = 64;       // per-token overlay / scratch entries per lane
-constexpr int kWalkWarps = 4;     // warps per k_walk block
-constexpr int kWalkSpan = 128;    // spellings per warp task
+constexpr int kWalkWarps = 8;    // warps per k_walk block
+constexpr int kSpan = 64;        // list entries / spellings per warp task
+constexpr int kPrepWarps = 4;    // rows per k_prep block
+constexpr int kMaxStage = 96 * 1024;
 
 #define GRID_CUDA(call)                                                                  \
   do {                                                                                   \
@@ -39,39 +47,25 @@ constexpr int kWalkSpan = 128;    // spellings per warp task
       return set_error(GRID_E_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
   } while (0)
 
-// All device tables of one (grammar, vocabulary) pair; passed by value.
-struct Tables {
-  int n_term, T1, S, NNT, P, Q, C, n_cat, LN;
-  int NS, V, eos, W, D;
-  uint32_t ignored[4];
-  uint32_t catmask[4];
-  int cat_term[32];
-  const uint8_t* byte_class;
-  const uint16_t* next;
-  const uint32_t* acc;
-  const uint32_t* live;
-  const int16_t* action;
-  const uint16_t* go;
-  const uint8_t* plen;
-  const uint16_t* plhs;
-  const int32_t* lx_cstart;
-  const uint8_t* lx_cbyte;
-  const int32_t* lx_cnode;
-  const uint32_t* lx_pcats;
-  const uint32_t* lx_wcats;
-  const int32_t* spell_off;
-  const uint8_t* spell_bytes;
-  const int32_t* skip;
-  const int32_t* spell_of_id;
+// Per-row scratch of one grid_masks call.
+struct RowCtx {
+  uint32_t A0[4];   // allowed terminals at sigma
+  uint32_t A1[4];   // allowed terminals at sigma' (after the forced emission)
+  int32_t q, lx, depth, tbl0;
+  int32_t emit_ok, eos_ok, status, complete;
+  uint32_t nonempty, done_blocks;
+  int32_t keep1, m1;
+  int32_t work0, total0;  // chunk counter / chunks of the row's walk queue
+  int32_t total1;         // leading chunks of the queue that belong to sigma' 
+  int32_t nrng;
+  uint16_t ovl1[kMaxOvl];
 };
 
-// Per-row scratch written by k_prep and read by k_walk / k_pack.
-struct RowCtx {
-  uint32_t A[4];      // allowed terminals at the row's stack
-  int32_t eos_ok;
-  int32_t status;
-  uint32_t nonempty;
-  uint32_t done_blocks;
+// Continuing first-byte ranges of a row without a CI table.
+struct RowRanges {
+  int32_t lo[256];
+  int32_t hi[256];
+  int32_t cpre[257];
 };
 
 struct DevConfigs {
@@ -81,216 +75,6 @@ struct DevConfigs {
   int32_t* lx;
   int32_t* flags;   // bit 0 = complete
 };
-
-__device__ __forceinline__ bool bit4(const uint32_t* m, int t) { return (m[t >> 5] >> (t & 31)) & 1u; }
-
-__device__ __forceinline__ int lex_step(const Tables& t, int lx, int b) {
-  if (lx < 0) return -1;
-  int lo = t.lx_cstart[lx], hi = t.lx_cstart[lx + 1];
-  const int end = hi;
-  while (lo < hi) {
-    int mid = (lo + hi) >> 1;
-    if ((int)t.lx_cbyte[mid] < b)
-      lo = mid + 1;
-    else
-      hi = mid;
-  }
-  return (lo < end && (int)t.lx_cbyte[lo] == b) ? t.lx_cnode[lo] : -1;
-}
-
-// Terminal set of state q filtered by the lexicon: non-category terminals pass,
-// category terminal c passes iff bit c of `cats` is set.
-__device__ __forceinline__ void lex_filter(const Tables& t, const uint32_t* __restrict__ src, int q,
-                                           uint32_t cats, uint32_t out[4]) {
-#pragma unroll
-  for (int w = 0; w < 4; ++w) out[w] = src[q * 4 + w] & ~t.catmask[w];
-  while (cats) {
-    int c = __ffs(cats) - 1;
-    cats &= cats - 1;
-    int term = t.cat_term[c];
-    out[term >> 5] |= src[q * 4 + (term >> 5)] & (1u << (term & 31));
-  }
-}
-
-__device__ __forceinline__ void live_prime(const Tables& t, int q, int lx, uint32_t out[4]) {
-  lex_filter(t, t.live, q, lx >= 0 ? t.lx_pcats[lx] : 0u, out);
-}
-
-__device__ __forceinline__ void cands(const Tables& t, int q, int lx, uint32_t out[4]) {
-  lex_filter(t, t.acc, q, lx >= 0 ? t.lx_wcats[lx] : 0u, out);
-}
-
-// Virtual stack = base[0:keep] ++ ovl[0:m] ++ scr[0:ns].  Runs the reduce
-// chain of terminal tau without modifying base or ovl.  Returns the ACTION
-// code that ends the chain (>0 shift target+1, kAccept) or 0 (error) or -1
-// (bound).  On a shift/accept, (keep_o, m_o, scr[0:ns]) is the stack below
-// the pushed state.
-__device__ int simulate(const Tables& t, const uint16_t* __restrict__ base, int keep,
-                        const uint16_t* ovl, int m, int tau, uint16_t* scr, int& keep_o, int& m_o,
-                        int& ns, int max_chain) {
-  int k = keep, mm = m;
-  ns = 0;
-  for (int it = 0; it < max_chain; ++it) {
-    int top = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
-    if (top >= t.S) return 0;
-    int a = t.action[top * t.T1 + tau];
-    if (a == 0) return 0;
-    if (a > 0) {
-      keep_o = k;
-      m_o = mm;
-      return a;
-    }
-    int p = -a - 1;
-    int n = t.plen[p];
-    int x = min(n, ns);
-    ns -= x;
-    n -= x;
-    x = min(n, mm);
-    mm -= x;
-    n -= x;
-    k -= n;
-    if (k < 1) return 0;
-    int top2 = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
-    if (top2 >= t.S) return 0;
-    if (ns >= kMaxOvl) return -1;
-    scr[ns++] = t.go[top2 * t.NNT + t.plhs[p]];
-  }
-  return -1;
-}
-
-// Per-token walk state over a row.
-struct Walker {
-  const uint16_t* base;
-  int keep, m;
-  int q, lx;
-  bool shifted;
-  uint16_t ovl[kMaxOvl];
-  uint16_t scr[kMaxOvl];
-};
-
-// Commit the result of a successful simulate(tau) + push of the shift target.
-__device__ __forceinline__ bool commit(Walker& w, int keep_o, int m_o, int ns, int target) {
-  if (m_o + ns + 1 > kMaxOvl) return false;
-  w.keep = keep_o;
-  w.m = m_o;
-  for (int i = 0; i < ns; ++i) w.ovl[w.m++] = w.scr[i];
-  w.ovl[w.m++] = (uint16_t)target;
-  return true;
-}
-
-// Emit the pending lexeme of (w.q, w.lx): pick the first candidate in priority
-// order that is ignored or reaches SHIFT; shift it.  `A` (may be NULL) is the
-// allowed set of the unmodified row stack, usable while nothing was shifted.
-// Returns 1 ok, 0 reject, -1 bound.
-__device__ int emit(const Tables& t, Walker& w, const uint32_t* A, int max_chain) {
-  uint32_t K[4];
-  cands(t, w.q, w.lx, K);
-  for (int wd = 0; wd < 4; ++wd) {
-    uint32_t bits = K[wd];
-    while (bits) {
-      int tau = wd * 32 + __ffs(bits) - 1;
-      bits &= bits - 1;
-      if (bit4(t.ignored, tau)) return 1;
-      if (A && !w.shifted && !bit4(A, tau)) continue;
-      int keep_o, m_o, ns;
-      int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, keep_o, m_o, ns, max_chain);
-      if (a < 0) return -1;
-      if (a > 0 && a != kAccept) {
-        if (!commit(w, keep_o, m_o, ns, a - 1)) return -1;
-        w.shifted = true;
-        return 1;
-      }
-    }
-  }
-  return 0;
-}
-
-// Trailing liveness (Def. 2): some terminal live at (q, lx) is ignored or
-// allowed at the current virtual stack.  1 / 0 / -1 (bound).
-__device__ int trailing_live(const Tables& t, Walker& w, const uint32_t* A, int max_chain) {
-  uint32_t L[4];
-  live_prime(t, w.q, w.lx, L);
-  if ((L[0] & t.ignored[0]) | (L[1] & t.ignored[1]) | (L[2] & t.ignored[2]) | (L[3] & t.ignored[3])) return 1;
-  if (A && !w.shifted) return ((L[0] & A[0]) | (L[1] & A[1]) | (L[2] & A[2]) | (L[3] & A[3])) ? 1 : 0;
-  for (int wd = 0; wd < 4; ++wd) {
-    uint32_t bits = L[wd];
-    while (bits) {
-      int tau = wd * 32 + __ffs(bits) - 1;
-      bits &= bits - 1;
-      int keep_o, m_o, ns;
-      int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, keep_o, m_o, ns, max_chain);
-      if (a < 0) return -1;
-      if (a > 0 && a != kAccept) return 1;
-    }
-  }
-  return 0;
-}
-
-// Walk the bytes of one token from the walker's state (Sec. 4.1).  Returns 1 if
-// the output stays a viable prefix, 0 if rejected (rej = index of the byte
-// from which on every extension is rejected), -1 on a bound.
-__device__ int walk_bytes(const Tables& t, Walker& w, const uint8_t* __restrict__ bytes, int len,
-                          const uint32_t* A, int max_chain, int& rej) {
-  uint32_t AI[4];
-  if (A) {
-#pragma unroll
-    for (int k = 0; k < 4; ++k) AI[k] = A[k] | t.ignored[k];
-  }
-  for (int i = 0; i < len; ++i) {
-    const int b = bytes[i];
-    const int c = t.byte_class[b];
-    int nq = t.next[w.q * t.C + c];
-    if (nq == kDead) {
-      if (w.q == kStart) {
-        rej = i;
-        return 0;
-      }
-      int e = emit(t, w, A, max_chain);
-      if (e <= 0) {
-        rej = i;
-        return e;
-      }
-      w.q = kStart;
-      w.lx = 0;
-      nq = t.next[kStart * t.C + c];
-      if (nq == kDead) {
-        rej = i;
-        return 0;
-      }
-    }
-    w.q = nq;
-    w.lx = lex_step(t, w.lx, b);
-    uint32_t L[4];
-    live_prime(t, w.q, w.lx, L);
-    bool any;
-    if (A && !w.shifted)
-      any = (L[0] & AI[0]) | (L[1] & AI[1]) | (L[2] & AI[2]) | (L[3] & AI[3]);
-    else
-      any = L[0] | L[1] | L[2] | L[3];
-    if (!any) {
-      rej = i;
-      return 0;
-    }
-  }
-  int r = trailing_live(t, w, A, max_chain);
-  if (r == 0) rej = len - 1;
-  return r;
-}
-
-// EOS gate (Sec. 3.2): the pending lexeme finalizes (same pick) and the reduce
-// chain of $end reaches ACCEPT on the resulting scratch stack.
-__device__ int eos_gate(const Tables& t, Walker& w, const uint32_t* A, int max_chain) {
-  if (w.q != kStart) {
-    int e = emit(t, w, A, max_chain);
-    if (e <= 0) return e;
-  }
-  int keep_o, m_o, ns;
-  int a = simulate(t, w.base, w.keep, w.ovl, w.m, t.n_term, w.scr, keep_o, m_o, ns, max_chain);
-  if (a < 0) return -1;
-  return a == kAccept ? 1 : 0;
-}
-
-__device__ __forceinline__ int max_chain_of(const Tables& t) { return 2 * t.D + 256; }
 
 // ---------------------------------------------------------------------------
 __global__ void k_reset(DevConfigs c, int B, int D) {
@@ -303,159 +87,499 @@ __global__ void k_reset(DevConfigs c, int B, int D) {
   c.flags[b] = 0;
 }
 
-// One warp per row: A(sigma) (lanes over terminals), EOS gate, scratch clear.
-__global__ void k_prep(Tables t, DevConfigs c, RowCtx* __restrict__ ctx, uint32_t* __restrict__ verd,
-                       int B, int words_ns) {
-  const int lane = threadIdx.x & 31;
-  const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+// ---------------- specialization ----------------
+__global__ void k_classify(Tables t, uint16_t* __restrict__ cls_sp, int32_t* __restrict__ cd_count) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ Tables ts;
+  stage_tables(t, ts, smem);
+  const int tbl = blockIdx.y;
+  const int q0 = t.tbl_q[tbl];
+  const int lx0 = q0 == kStart ? 0 : -1;
+  int cd = 0;
+  for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < t.NS; s += gridDim.x * blockDim.x) {
+    const int off = t.spell_off[s];
+    const int len = t.spell_off[s + 1] - off;
+    const uint8_t* by = t.spell_bytes + off;
+    uint16_t code;
+    if (!t.ci_on)
+      code = kClsCD;
+    else if (q0 != kStart && ts.next[q0 * ts.C + ts.byte_class[by[0]]] == kDead)
+      code = kClsNA;
+    else
+      code = classify(ts, q0, lx0, by, len);
+    cls_sp[(size_t)tbl * t.NS + s] = code;
+    cd += code == kClsCD;
+  }
+  cd = __reduce_add_sync(0xffffffffu, cd);
+  if ((threadIdx.x & 31) == 0 && cd) atomicAdd(&cd_count[tbl], cd);
+}
+
+// One block per table: ordered stream compaction of the CD spellings.
+__global__ void k_compact(const uint16_t* __restrict__ cls_sp, int NS, const int32_t* __restrict__ cd_off,
+                          int32_t* __restrict__ cd_list) {
+  __shared__ int32_t warp_tot[32];
+  __shared__ int32_t base;
+  const int tbl = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  if (threadIdx.x == 0) base = cd_off[tbl];
+  __syncthreads();
+  for (int s0 = 0; s0 < NS; s0 += blockDim.x) {
+    const int s = s0 + threadIdx.x;
+    const bool f = s < NS && cls_sp[(size_t)tbl * NS + s] == kClsCD;
+    const uint32_t bal = __ballot_sync(0xffffffffu, f);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    int before = 0;
+    for (int k = 0; k < warp; ++k) before += warp_tot[k];
+    if (f) cd_list[base + before + __popc(bal & ((1u << lane) - 1u))] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int tot = 0;
+      for (int k = 0; k < nw; ++k) tot += warp_tot[k];
+      base += tot;
+    }
+    __syncthreads();
+  }
+}
+
+__global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, uint16_t* __restrict__ cls_by_id,
+                          uint8_t* __restrict__ fb_by_id) {
+  const int id = blockIdx.x * blockDim.x + threadIdx.x;
+  if (id >= t.V) return;
+  const int s = t.spell_of_id[id];
+  fb_by_id[id] = s >= 0 ? t.spell_bytes[t.spell_off[s]] : 0;
+  for (int k = 0; k < t.n_tbl; ++k) cls_by_id[(size_t)k * t.V + id] = s >= 0 ? cls_sp[(size_t)k * t.NS + s] : kClsNA;
+}
+
+// ---------------- mask step ----------------
+__device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* out, int lane) {
+  uint32_t AI[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) AI[k] = A[k] | t.ignored[k];
+  for (int w0 = 0; w0 < t.nselw; ++w0) {
+    const int cls = w0 * 32 + lane;
+    bool v = false;
+    if (cls < t.ncls) {
+      uint32_t S[4];
+      class_set(t, cls, S);
+      v = (S[0] & AI[0]) | (S[1] & AI[1]) | (S[2] & AI[2]) | (S[3] & AI[3]);
+    }
+    const uint32_t word = __ballot_sync(0xffffffffu, v);
+    if (lane == 0) out[w0] = word;
+  }
+}
+
+__device__ void allowed_set(const Tables& t, const uint16_t* base, int keep, const uint16_t* ovl, int m,
+                            uint32_t A[4], int& status, int lane) {
+  const int mc = max_chain_of(t);
+  for (int wd = 0; wd < 4; ++wd) {
+    const int tau = wd * 32 + lane;
+    bool ok = false;
+    if (tau < t.n_term && !bit4(t.ignored, tau)) {
+      uint16_t scr[kMaxOvl];
+      int keep_o, m_o, ns;
+      int a = simulate(t, base, keep, ovl, m, tau, scr, keep_o, m_o, ns, mc);
+      ok = a > 0 && a != kAccept;
+      if (a < 0) status = GRID_ST_BOUND;
+    }
+    A[wd] = __ballot_sync(0xffffffffu, ok);
+  }
+}
+
+__global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
+                                                          RowRanges* __restrict__ rng, uint32_t* __restrict__ sel,
+                                                          uint32_t* __restrict__ verd0, uint32_t* __restrict__ verd1,
+                                                          int B, int words_ns) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ uint16_t s_ovl[kPrepWarps][kMaxOvl];
+  __shared__ int s_km[kPrepWarps][3];
+  const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
+  if ((int)blockIdx.x >= row_blocks) {
+    // clearing blocks: zero both verdict bitmaps of every row
+    const size_t n = (size_t)B * words_ns;
+    const size_t n4 = n >> 2;
+    const size_t stride = (size_t)(gridDim.x - row_blocks) * blockDim.x;
+    const size_t first = (size_t)(blockIdx.x - row_blocks) * blockDim.x + threadIdx.x;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    for (size_t i = first; i < n4; i += stride) {
+      reinterpret_cast<uint4*>(verd0)[i] = z;
+      reinterpret_cast<uint4*>(verd1)[i] = z;
+    }
+    for (size_t i = (n4 << 2) + first; i < n; i += stride) {
+      verd0[i] = 0u;
+      verd1[i] = 0u;
+    }
+    return;
+  }
+  __shared__ Tables ts;
+  stage_tables(t, ts, smem);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int b = blockIdx.x * kPrepWarps + warp;
   if (b >= B) return;
   RowCtx& r = ctx[b];
-  uint32_t* vb = verd + (size_t)b * words_ns;
-  for (int i = lane; i < words_ns; i += 32) vb[i] = 0u;
   const int complete = c.flags[b] & 1;
   const uint16_t* base = c.stack + (size_t)b * t.D;
-  const int depth = c.depth[b];
+  const int depth = c.depth[b], q = c.q[b], lx = c.lx[b];
   const int mc = max_chain_of(t);
   int status = complete ? GRID_ST_COMPLETE : GRID_ST_OK;
-  uint32_t A[4] = {0, 0, 0, 0};
-  if (!complete) {
-    for (int wd = 0; wd < 4; ++wd) {
-      int tau = wd * 32 + lane;
-      bool ok = false;
-      if (tau < t.n_term && !bit4(t.ignored, tau)) {
-        uint16_t scr[kMaxOvl];
-        int keep_o, m_o, ns;
-        int a = simulate(t, base, depth, nullptr, 0, tau, scr, keep_o, m_o, ns, mc);
-        ok = a > 0 && a != kAccept;
-        if (a < 0) status = GRID_ST_BOUND;
-      }
-      A[wd] = __ballot_sync(0xffffffffu, ok);
-    }
-    status = __reduce_max_sync(0xffffffffu, status);
-  }
+  uint32_t A0[4] = {0, 0, 0, 0}, A1[4] = {0, 0, 0, 0};
+  if (!complete) allowed_set(ts, base, depth, nullptr, 0, A0, status, lane);
+  // forced emission of the pending lexeme + EOS gate (lane 0)
   if (lane == 0) {
-    int eos = 0;
+    int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
     if (!complete) {
       Walker w;
       w.base = base;
       w.keep = depth;
       w.m = 0;
-      w.q = c.q[b];
-      w.lx = c.lx[b];
+      w.q = q;
+      w.lx = lx;
       w.shifted = false;
-      int e = eos_gate(t, w, A, mc);
-      if (e < 0) status = GRID_ST_BOUND;
-      eos = e > 0;
+      if (q == kStart) {
+        emit_ok = 1;
+      } else {
+        int e = emit(ts, w, A0, mc);
+        if (e < 0) status = GRID_ST_BOUND;
+        emit_ok = e > 0;
+        keep1 = w.keep;
+        m1 = w.m;
+        for (int i = 0; i < m1; ++i) s_ovl[warp][i] = w.ovl[i];
+      }
+      Walker w2;
+      w2.base = base;
+      w2.keep = depth;
+      w2.m = 0;
+      w2.q = q;
+      w2.lx = lx;
+      w2.shifted = false;
+      int g = eos_gate(ts, w2, A0, mc);
+      if (g < 0) status = GRID_ST_BOUND;
+      eos = g > 0;
     }
-    for (int k = 0; k < 4; ++k) r.A[k] = A[k];
+    s_km[warp][0] = emit_ok;
+    s_km[warp][1] = keep1;
+    s_km[warp][2] = m1;
     r.eos_ok = eos;
+  }
+  __syncwarp();
+  const int emit_ok = s_km[warp][0], keep1 = s_km[warp][1], m1 = s_km[warp][2];
+  if (!complete && emit_ok) {
+    if (keep1 == depth && m1 == 0) {
+      for (int k = 0; k < 4; ++k) A1[k] = A0[k];
+    } else {
+      allowed_set(ts, base, keep1, s_ovl[warp], m1, A1, status, lane);
+    }
+  }
+  status = __reduce_max_sync(0xffffffffu, status);
+  const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
+  uint32_t* sel0 = sel + (size_t)b * 2 * t.nselw;
+  uint32_t* sel1 = sel0 + t.nselw;
+  if (!complete && t.ci_on) {
+    if (tbl0 >= 0) select_classes(ts, A0, sel0, lane);
+    if (emit_ok) select_classes(ts, A1, sel1, lane);
+  }
+  // continuing first-byte ranges (rows without a CI table for q)
+  int total0 = 0, nrng = 0;
+  if (!complete && q != kStart) {
+    if (tbl0 >= 0) {
+      const int len = t.cd_off[tbl0 + 1] - t.cd_off[tbl0];
+      total0 = (len + kSpan - 1) / kSpan;
+    } else {
+      RowRanges& R = rng[b];
+      for (int b0 = 0; b0 < 256; b0 += 32) {
+        const int by = b0 + lane;
+        const int lo = t.first_of_byte[by], hi = t.first_of_byte[by + 1];
+        const bool cont = hi > lo && ts.next[q * ts.C + ts.byte_class[by]] != kDead;
+        const int chunks = cont ? (hi - lo + kSpan - 1) / kSpan : 0;
+        const uint32_t bal = __ballot_sync(0xffffffffu, cont);
+        int incl = chunks;
+        for (int d = 1; d < 32; d <<= 1) {
+          int v = __shfl_up_sync(0xffffffffu, incl, d);
+          if (lane >= d) incl += v;
+        }
+        if (cont) {
+          const int k = nrng + __popc(bal & ((1u << lane) - 1u));
+          R.lo[k] = lo;
+          R.hi[k] = hi;
+          R.cpre[k] = total0 + incl - chunks;
+        }
+        total0 += __shfl_sync(0xffffffffu, incl, 31);
+        nrng += __popc(bal);
+      }
+      if (lane == 0) R.cpre[nrng] = total0;
+    }
+  }
+  const int start_len = t.cd_off[1] - t.cd_off[0];
+  const int total1 = (!complete && emit_ok) ? (start_len + kSpan - 1) / kSpan : 0;
+  if (lane == 0) {
+    for (int k = 0; k < 4; ++k) {
+      r.A0[k] = A0[k];
+      r.A1[k] = A1[k];
+    }
+    r.q = q;
+    r.lx = lx;
+    r.depth = depth;
+    r.tbl0 = tbl0;
+    r.emit_ok = emit_ok;
     r.status = status;
+    r.complete = complete;
     r.nonempty = 0;
     r.done_blocks = 0;
+    r.keep1 = keep1;
+    r.m1 = m1;
+    r.work0 = 0;
+    r.total0 = total1 + total0;
+    r.total1 = total1;
+    r.nrng = nrng;
   }
+  for (int i = lane; i < m1; i += 32) r.ovl1[i] = s_ovl[warp][i];
 }
 
-// grid = (chunks, B); each warp walks kWalkSpan consecutive spellings.
-__global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
-                                                          uint32_t* __restrict__ verd, int words_ns) {
-  const int b = blockIdx.y;
-  if (c.flags[b] & 1) return;
+struct WalkCtx {
+  const uint16_t* base;
+  int keep, m;
+  const uint16_t* ovl;
+  int q, lx;
+  int kill_q;  // >= 0: spellings whose first byte continues this DFA state are skipped
+  uint32_t A[4];
+};
+
+// Walk list positions [p0, p1) (list == NULL: spelling indices).  Verdict bits
+// go to vb (spelling order).
+__device__ void walk_span(const Tables& t, const WalkCtx& wc, const int32_t* __restrict__ list, int p0, int p1,
+                          uint32_t* __restrict__ vb, int& bound) {
   const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
-  const int lo = (blockIdx.x * kWalkWarps + warp) * kWalkSpan;
-  __shared__ uint32_t sA[4];
-  if (threadIdx.x < 4) sA[threadIdx.x] = ctx[b].A[threadIdx.x];
-  __syncthreads();
-  if (lo >= t.NS) return;
-  const int hi = min(lo + kWalkSpan, t.NS);
-  uint32_t A[4] = {sA[0], sA[1], sA[2], sA[3]};
-  const uint16_t* base = c.stack + (size_t)b * t.D;
-  const int depth = c.depth[b], q0 = c.q[b], lx0 = c.lx[b];
   const int mc = max_chain_of(t);
-  uint32_t* vb = verd + (size_t)b * words_ns;
-  int bound = 0;
   Walker w;
-  for (int cursor = lo; cursor < hi;) {
-    const int s = cursor + lane;
-    int ok = 0, rej = -1;
-    if (s < hi) {
+  for (int pos = p0; pos < p1;) {
+    const int i = pos + lane;
+    int s = -1, ok = 0, rej = -1;
+    if (i < p1) {
+      s = list ? list[i] : i;
       const int off = t.spell_off[s];
       const int len = t.spell_off[s + 1] - off;
-      w.base = base;
-      w.keep = depth;
-      w.m = 0;
-      w.q = q0;
-      w.lx = lx0;
-      w.shifted = false;
-      int r = walk_bytes(t, w, t.spell_bytes + off, len, A, mc, rej);
-      if (r < 0) {
-        bound = 1;
-        rej = -1;
+      const uint8_t* by = t.spell_bytes + off;
+      if (wc.kill_q >= 0 && t.next[wc.kill_q * t.C + t.byte_class[by[0]]] != kDead) {
+        rej = 0;  // continues the pending lexeme: handled by the other context
+      } else {
+        w.base = wc.base;
+        w.keep = wc.keep;
+        w.m = wc.m;
+        for (int k = 0; k < wc.m; ++k) w.ovl[k] = wc.ovl[k];
+        w.q = wc.q;
+        w.lx = wc.lx;
+        w.shifted = false;
+        const int r = walk_bytes(t, w, by, len, wc.A, mc, rej);
+        if (r < 0) {
+          bound = 1;
+          rej = -1;
+        }
+        ok = r > 0;
       }
-      ok = r > 0;
     }
-    const uint32_t m = __ballot_sync(0xffffffffu, ok);
-    if (lane == 0 && m) {
-      const int sh = cursor & 31;
-      atomicOr(&vb[cursor >> 5], m << sh);
-      if (sh && (m >> (32 - sh))) atomicOr(&vb[(cursor >> 5) + 1], m >> (32 - sh));
+    if (list) {
+      if (ok) atomicOr(&vb[s >> 5], 1u << (s & 31));
+    } else {
+      const uint32_t m = __ballot_sync(0xffffffffu, ok);
+      if (lane == 0 && m) {
+        const int sh = pos & 31;
+        atomicOr(&vb[pos >> 5], m << sh);
+        if (sh && (m >> (32 - sh))) atomicOr(&vb[(pos >> 5) + 1], m >> (32 - sh));
+      }
     }
-    // skip the rejected subtree of the last lane's spelling
-    int nxt = cursor + 32;
-    const int last = min(31, hi - 1 - cursor);
+    int nxt = pos + 32;
+    const int last = min(31, p1 - 1 - pos);
     const int lrej = __shfl_sync(0xffffffffu, rej, last);
+    const int ls = __shfl_sync(0xffffffffu, s, last);
     if (lrej >= 0) {
-      const int sl = cursor + last;
-      const int sk = t.skip[t.spell_off[sl] + lrej];
-      nxt = max(nxt, sk);
+      const int sk = t.skip[t.spell_off[ls] + lrej];
+      if (list) {
+        int lo = nxt, hi = p1;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (list[mid] < sk)
+            lo = mid + 1;
+          else
+            hi = mid;
+        }
+        nxt = lo;
+      } else {
+        nxt = max(nxt, sk);
+      }
     }
-    cursor = nxt;
+    pos = nxt;
   }
-  if (__any_sync(0xffffffffu, bound) && lane == 0) atomicCAS(&ctx[b].status, GRID_ST_OK, GRID_ST_BOUND);
 }
 
-// grid = (ceil(W/8), B), 256 threads: one thread per token id.
-__global__ void k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ verd, int words_ns,
-                       uint32_t* __restrict__ mask, int32_t* __restrict__ d_status) {
-  const int b = blockIdx.y;
-  const int id = blockIdx.x * blockDim.x + threadIdx.x;
-  const int lane = threadIdx.x & 31;
-  RowCtx& r = ctx[b];
-  const bool complete = r.status == GRID_ST_COMPLETE;
-  bool bit = false;
-  if (id < t.V && !complete) {
-    if (id == t.eos) {
-      bit = r.eos_ok != 0;
-    } else {
-      int s = t.spell_of_id[id];
-      if (s >= 0) bit = (verd[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
+// Persistent walk.  Every row owns one work queue of chunks: chunks
+// [0, total1) cover the start state's CD list under sigma' (tokens whose first
+// byte ends the pending lexeme), chunks [total1, total) the spellings that
+// continue the pending lexeme (the CD list of its lexer state, or its
+// continuing first-byte ranges).  Warps start at different rows, drain a row's
+// queue chunk by chunk and move on; a warp stops after finding every queue
+// empty once in a row.
+__global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __restrict__ ctx,
+                                                          const RowRanges* __restrict__ rng, const uint16_t* stacks,
+                                                          uint32_t* __restrict__ verd0, uint32_t* __restrict__ verd1,
+                                                          int words_ns, int B) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
+  __shared__ Tables ts;
+  stage_tables(t, ts, smem);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kWalkWarps + warp;
+  const int start_len = t.cd_off[1] - t.cd_off[0];
+  const int32_t* start_list = t.cd_list + t.cd_off[0];
+  int row = gw % B;
+  int fails = 0;
+  int bound = 0, bound_row = -1;
+  while (fails < B) {
+    RowCtx& r = ctx[row];
+    const int total = r.total0;
+    int cidx = total;
+    if (lane == 0 && *((volatile int32_t*)&r.work0) < total) cidx = atomicAdd(&r.work0, 1);
+    cidx = __shfl_sync(0xffffffffu, cidx, 0);
+    if (cidx >= total) {
+      ++fails;
+      row = row + 1 == B ? 0 : row + 1;
+      continue;
     }
+    fails = 0;
+    const int total1 = r.total1;
+    WalkCtx wc;
+    wc.base = stacks + (size_t)row * t.D;
+    if (cidx < total1) {
+      const int m1 = r.m1;
+      __syncwarp();
+      for (int i = lane; i < m1; i += 32) s_ovl[warp][i] = r.ovl1[i];
+      __syncwarp();
+      wc.keep = r.keep1;
+      wc.m = m1;
+      wc.ovl = s_ovl[warp];
+      wc.q = kStart;
+      wc.lx = 0;
+      wc.kill_q = r.q == kStart ? -1 : r.q;
+      for (int k = 0; k < 4; ++k) wc.A[k] = r.A1[k];
+      const int p0 = cidx * kSpan;
+      walk_span(ts, wc, start_list, p0, min(start_len, p0 + kSpan), verd1 + (size_t)row * words_ns, bound);
+    } else {
+      const int c0 = cidx - total1;
+      wc.keep = r.depth;
+      wc.m = 0;
+      wc.ovl = s_ovl[warp];
+      wc.q = r.q;
+      wc.lx = r.lx;
+      wc.kill_q = -1;
+      for (int k = 0; k < 4; ++k) wc.A[k] = r.A0[k];
+      const int tbl0 = r.tbl0;
+      if (tbl0 >= 0) {
+        const int32_t* list = t.cd_list + t.cd_off[tbl0];
+        const int len = t.cd_off[tbl0 + 1] - t.cd_off[tbl0];
+        const int p0 = c0 * kSpan;
+        walk_span(ts, wc, list, p0, min(len, p0 + kSpan), verd0 + (size_t)row * words_ns, bound);
+      } else {
+        const RowRanges& R = rng[row];
+        int lo = 0, hi = r.nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
+        while (hi - lo > 1) {
+          const int mid = (lo + hi) >> 1;
+          if (R.cpre[mid] <= c0)
+            lo = mid;
+          else
+            hi = mid;
+        }
+        const int p0 = R.lo[lo] + (c0 - R.cpre[lo]) * kSpan;
+        walk_span(ts, wc, nullptr, p0, min(R.hi[lo], p0 + kSpan), verd0 + (size_t)row * words_ns, bound);
+      }
+    }
+    if (bound && bound_row < 0) bound_row = row;
   }
-  const uint32_t word = __ballot_sync(0xffffffffu, bit);
-  const int wi = id >> 5;
-  if (lane == 0 && wi < t.W) {
-    mask[(size_t)b * t.W + wi] = word;
-    if (word) atomicOr(&r.nonempty, 1u);
-    __threadfence();
+  if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
+}
+
+// grid = (ceil(V/1024), B), 256 threads x 4 token ids.
+__global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
+                                              const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
+                                              int words_ns, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status) {
+  extern __shared__ __align__(16) uint32_t s_sel[];  // 2 * nselw
+  __shared__ __align__(16) RowCtx s_r;
+  const int b = blockIdx.y;
+  {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(&ctx[b]);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(&s_r);
+    for (int i = threadIdx.x; i < (int)(sizeof(RowCtx) / 4); i += blockDim.x) dst[i] = src[i];
   }
+  for (int i = threadIdx.x; i < 2 * t.nselw; i += blockDim.x) s_sel[i] = sel[(size_t)b * 2 * t.nselw + i];
   __syncthreads();
+  const RowCtx& r = s_r;
+  const int lane = threadIdx.x & 31;
+  const uint32_t* v0 = verd0 + (size_t)b * words_ns;
+  const uint32_t* v1 = verd1 + (size_t)b * words_ns;
+  const uint16_t* cls0 = r.tbl0 >= 0 ? t.cls_by_id + (size_t)r.tbl0 * t.V : nullptr;
+  int any = 0;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int id = (blockIdx.x * 4 + k) * blockDim.x + threadIdx.x;
+    bool bit = false;
+    if (id < t.V && !r.complete) {
+      if (id == t.eos) {
+        bit = r.eos_ok != 0;
+      } else {
+        const int s = t.spell_of_id[id];
+        if (s >= 0) {
+          const int b0 = t.first_byte_by_id[id];
+          const bool kills = r.q == kStart || t.next[r.q * t.C + t.byte_class[b0]] == kDead;
+          if (kills) {
+            if (r.emit_ok) {
+              const uint16_t cl = t.cls_by_id[id];
+              if (cl < kClsNA)
+                bit = (s_sel[t.nselw + (cl >> 5)] >> (cl & 31)) & 1u;
+              else if (cl == kClsAcc)
+                bit = true;
+              else if (cl == kClsCD)
+                bit = (v1[s >> 5] >> (s & 31)) & 1u;
+            }
+          } else if (cls0) {
+            const uint16_t cl = cls0[id];
+            if (cl < kClsNA)
+              bit = (s_sel[cl >> 5] >> (cl & 31)) & 1u;
+            else if (cl == kClsAcc)
+              bit = true;
+            else if (cl == kClsCD)
+              bit = (v0[s >> 5] >> (s & 31)) & 1u;
+          } else {
+            bit = (v0[s >> 5] >> (s & 31)) & 1u;
+          }
+        }
+      }
+    }
+    const uint32_t word = __ballot_sync(0xffffffffu, bit);
+    const int wi = id >> 5;
+    if (lane == 0 && wi < t.W) mask[(size_t)b * t.W + wi] = word;
+    any |= word != 0u;
+  }
+  any = __syncthreads_or(any);
   if (threadIdx.x == 0) {
+    if (any) atomicOr(&ctx[b].nonempty, 1u);
     __threadfence();
-    unsigned prev = atomicAdd(&r.done_blocks, 1u);
+    const unsigned prev = atomicAdd(&ctx[b].done_blocks, 1u);
     if (prev == gridDim.x - 1) {
       __threadfence();
-      int st = atomicAdd(&r.status, 0);
-      if (st == GRID_ST_OK && atomicAdd(&r.nonempty, 0u) == 0u) st = GRID_ST_EMPTY_MASK;
+      int st = atomicAdd(&ctx[b].status, 0);
+      if (st == GRID_ST_OK && atomicAdd(&ctx[b].nonempty, 0u) == 0u) st = GRID_ST_EMPTY_MASK;
       d_status[b] = st;
     }
   }
 }
 
 // One warp per row; lane 0 feeds the tokens, all lanes copy for out-of-place.
-__global__ void k_advance(Tables t, DevConfigs cin, DevConfigs cout, const int32_t* __restrict__ tokens,
-                          int n_steps, int32_t* __restrict__ d_status, int B, int copy) {
+__global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfigs cin, DevConfigs cout,
+                                                             const int32_t* __restrict__ tokens, int n_steps,
+                                                             int32_t* __restrict__ d_status, int B, int copy) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ Tables ts;
+  stage_tables(t, ts, smem);
   const int lane = threadIdx.x & 31;
-  const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int b = blockIdx.x * kPrepWarps + (threadIdx.x >> 5);
   if (b >= B) return;
   if (copy) {
     const int d = cin.depth[b];
@@ -492,7 +616,7 @@ __global__ void k_advance(Tables t, DevConfigs cin, DevConfigs cout, const int32
     w.lx = lx;
     w.shifted = false;
     if (tok == t.eos) {
-      int e = eos_gate(t, w, nullptr, mc);
+      const int e = eos_gate(ts, w, nullptr, mc);
       if (e < 0) {
         status = GRID_ST_BOUND;
         break;
@@ -511,7 +635,7 @@ __global__ void k_advance(Tables t, DevConfigs cin, DevConfigs cout, const int32
     }
     const int off = t.spell_off[s];
     int rej;
-    int r = walk_bytes(t, w, t.spell_bytes + off, t.spell_off[s + 1] - off, nullptr, mc, rej);
+    const int r = walk_bytes(ts, w, t.spell_bytes + off, t.spell_off[s + 1] - off, nullptr, mc, rej);
     if (r < 0) {
       status = GRID_ST_BOUND;
       break;
@@ -536,10 +660,12 @@ __global__ void k_advance(Tables t, DevConfigs cin, DevConfigs cout, const int32
   d_status[b] = status;
 }
 
-// In-place -inf fill: one thread per 32-byte sector of logits.
+// In-place -inf fill: one thread per 32-byte sector of logits.  A sector whose
+// tokens are all rejected is written without being read; a mixed sector is
+// read, blended and written; a fully accepted sector is not touched.
 template <typename T>
-__global__ void k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logits, int B, int V, int W,
-                        long long stride, int vec_ok) {
+__global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logits, int B,
+                                               int V, int W, long long stride, int vec_ok) {
   constexpr int E = 32 / sizeof(T);  // elements per sector: 8 fp32 or 16 bf16
   const long long per_row = (V + E - 1) / E;
   const long long total = per_row * B;
@@ -548,20 +674,18 @@ __global__ void k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logit
     const int b = (int)(g / per_row);
     const int e0 = (int)(g - (long long)b * per_row) * E;
     const uint32_t word = mask[(size_t)b * W + (e0 >> 5)];
-    const uint32_t bits = (word >> (e0 & 31)) & ((E == 32) ? 0xffffffffu : ((1u << E) - 1u));
+    const uint32_t full = (1u << E) - 1u;
+    const uint32_t bits = (word >> (e0 & 31)) & full;
     T* p = logits + (size_t)b * stride + e0;
     const int n = min(E, V - e0);
     if (vec_ok && n == E) {
       uint4* p4 = reinterpret_cast<uint4*>(p);
       if (bits == 0u) {
-        uint4 v;
-        if (sizeof(T) == 4)
-          v = make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
-        else
-          v = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+        const uint4 v = sizeof(T) == 4 ? make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u)
+                                       : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
         p4[0] = v;
         p4[1] = v;
-      } else if (bits != ((1u << E) - 1u)) {
+      } else if (bits != full) {
         uint4 v[2] = {p4[0], p4[1]};
         if (sizeof(T) == 4) {
           uint32_t* u = reinterpret_cast<uint32_t*>(v);
@@ -590,16 +714,31 @@ __global__ void k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logit
   }
 }
 
-template <typename T>
-int upload(std::vector<void*>& owned, const std::vector<T>& v, const T** out) {
-  void* p = nullptr;
-  size_t n = std::max<size_t>(v.size(), 1) * sizeof(T);
-  GRID_CUDA(cudaMalloc(&p, n));
-  owned.push_back(p);
-  if (!v.empty()) GRID_CUDA(cudaMemcpy(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice));
-  *out = static_cast<const T*>(p);
-  return GRID_OK;
-}
+// ---------------------------------------------------------------------------
+struct Arena {
+  std::vector<void*> owned;
+  template <typename T>
+  int upload(const std::vector<T>& v, const T** out) {
+    void* p = nullptr;
+    size_t n = std::max<size_t>(v.size(), 1) * sizeof(T);
+    GRID_CUDA(cudaMalloc(&p, n));
+    owned.push_back(p);
+    if (!v.empty()) GRID_CUDA(cudaMemcpy(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice));
+    *out = static_cast<const T*>(p);
+    return GRID_OK;
+  }
+  int alloc(size_t n, void** out) {
+    GRID_CUDA(cudaMalloc(out, std::max<size_t>(n, 16)));
+    owned.push_back(*out);
+    return GRID_OK;
+  }
+  void release() {
+    for (void* p : owned) cudaFree(p);
+    owned.clear();
+  }
+};
+
+size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 }  // namespace
 }  // namespace grid
@@ -610,23 +749,42 @@ struct grid_spec {
   const grid_grammar* g = nullptr;
   const grid_vocab* v = nullptr;
   Tables t;
-  std::vector<void*> owned;
+  Arena mem;
   int device = 0;
+  int sms = 152;
+  int n1 = 0;  // walk chunks of the start state's CD list
+  int walk_blocks = 0;  // persistent k_walk grid: resident blocks per SM x SMs
 };
 
 struct grid_configs {
   int B = 0, D = 0, words_ns = 0;
   DevConfigs c;
   RowCtx* ctx = nullptr;
-  uint32_t* verd = nullptr;
-  std::vector<void*> owned;
+  RowRanges* rng = nullptr;
+  uint32_t* sel = nullptr;
+  uint32_t* verd0 = nullptr;
+  uint32_t* verd1 = nullptr;
+  Arena mem;
 };
+
+// The dynamic shared-memory cap is a per-function attribute shared by every
+// spec in the process, so it is raised once to the largest staged block
+// allowed instead of to this spec's size.
+static int set_smem_limits() {
+  const int dyn = kMaxStage;
+  GRID_CUDA(cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  return GRID_OK;
+}
 
 extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void* stream, grid_spec** out) {
   if (!g || !v || !out) return set_error(GRID_E_INVALID_ARG, "grid_specialize: bad arguments");
   *out = nullptr;
   const HostGrammar& h = g->h;
   const HostVocab& hv = v->h;
+  cudaStream_t st = (cudaStream_t)stream;
   auto* s = new grid_spec();
   s->g = g;
   s->v = v;
@@ -651,34 +809,128 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     t.catmask[k] = h.catmask[k];
   }
   for (int c = 0; c < h.n_cat; ++c) t.cat_term[c] = h.cat_term[c];
-  std::vector<uint8_t> bc(h.byte_class, h.byte_class + 256);
-  int rc = GRID_OK;
-  auto& o = s->owned;
-  if ((rc = upload(o, bc, &t.byte_class)) || (rc = upload(o, h.next, &t.next)) ||
-      (rc = upload(o, h.acc, &t.acc)) || (rc = upload(o, h.live, &t.live)) ||
-      (rc = upload(o, h.action, &t.action)) || (rc = upload(o, h.go, &t.go)) ||
-      (rc = upload(o, h.plen, &t.plen)) || (rc = upload(o, h.plhs, &t.plhs)) ||
-      (rc = upload(o, h.lx_cstart, &t.lx_cstart)) || (rc = upload(o, h.lx_cbyte, &t.lx_cbyte)) ||
-      (rc = upload(o, h.lx_cnode, &t.lx_cnode)) || (rc = upload(o, h.lx_pcats, &t.lx_pcats)) ||
-      (rc = upload(o, h.lx_wcats, &t.lx_wcats)) || (rc = upload(o, hv.spell_off, &t.spell_off)) ||
-      (rc = upload(o, hv.spell_bytes, &t.spell_bytes)) || (rc = upload(o, hv.skip, &t.skip)) ||
-      (rc = upload(o, hv.spell_of_id, &t.spell_of_id))) {
-    grid_spec_free(s);
+  auto fail = [&](int rc) {
+    s->mem.release();
+    delete s;
     return rc;
+  };
+  // staged block: byte classes, DFA, acc/live, ACTION, GOTO, production tables
+  std::vector<size_t> off(9, 0);
+  const size_t sizes[8] = {256, h.next.size() * 2, h.acc.size() * 4, h.live.size() * 4, h.action.size() * 2,
+                           h.go.size() * 2, h.plen.size(), h.plhs.size() * 2};
+  for (int k = 0; k < 8; ++k) off[k + 1] = align16(off[k] + sizes[k]);
+  std::vector<uint8_t> blob(off[8], 0);
+  std::memcpy(blob.data() + off[0], h.byte_class, 256);
+  std::memcpy(blob.data() + off[1], h.next.data(), sizes[1]);
+  std::memcpy(blob.data() + off[2], h.acc.data(), sizes[2]);
+  std::memcpy(blob.data() + off[3], h.live.data(), sizes[3]);
+  std::memcpy(blob.data() + off[4], h.action.data(), sizes[4]);
+  std::memcpy(blob.data() + off[5], h.go.data(), sizes[5]);
+  std::memcpy(blob.data() + off[6], h.plen.data(), sizes[6]);
+  std::memcpy(blob.data() + off[7], h.plhs.data(), sizes[7]);
+  const uint8_t* dblob = nullptr;
+  int rc = s->mem.upload(blob, &dblob);
+  if (rc) return fail(rc);
+  t.blob = dblob;
+  t.blob_bytes = off[8] <= (size_t)kMaxStage ? (int)off[8] : 0;
+  t.byte_class = dblob + off[0];
+  t.next = reinterpret_cast<const uint16_t*>(dblob + off[1]);
+  t.acc = reinterpret_cast<const uint32_t*>(dblob + off[2]);
+  t.live = reinterpret_cast<const uint32_t*>(dblob + off[3]);
+  t.action = reinterpret_cast<const int16_t*>(dblob + off[4]);
+  t.go = reinterpret_cast<const uint16_t*>(dblob + off[5]);
+  t.plen = dblob + off[6];
+  t.plhs = reinterpret_cast<const uint16_t*>(dblob + off[7]);
+  Arena& a = s->mem;
+  if ((rc = a.upload(h.lx_cstart, &t.lx_cstart)) || (rc = a.upload(h.lx_cbyte, &t.lx_cbyte)) ||
+      (rc = a.upload(h.lx_cnode, &t.lx_cnode)) || (rc = a.upload(h.lx_pcats, &t.lx_pcats)) ||
+      (rc = a.upload(h.lx_wcats, &t.lx_wcats)) || (rc = a.upload(hv.spell_off, &t.spell_off)) ||
+      (rc = a.upload(hv.spell_bytes, &t.spell_bytes)) || (rc = a.upload(hv.skip, &t.skip)) ||
+      (rc = a.upload(hv.spell_of_id, &t.spell_of_id)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
+    return fail(rc);
+  // precomputed lexer states: the start state and every state at which no
+  // lexicon category is live (there the lexicon node cannot matter)
+  std::vector<int32_t> tq{kStart};
+  std::vector<int16_t> tbl_of_q(h.Q, -1);
+  tbl_of_q[kStart] = 0;
+  const long ncls = (long)(2 * h.Q) << h.n_cat;
+  t.ci_on = ncls < (long)kClsNA ? 1 : 0;
+  if (t.ci_on) {
+    for (int q = 2; q < h.Q; ++q) {
+      bool catlive = false;
+      for (int w = 0; w < 4; ++w)
+        if (h.live[q * 4 + w] & h.catmask[w]) catlive = true;
+      if (!catlive && tq.size() < 4096) {
+        tbl_of_q[q] = (int16_t)tq.size();
+        tq.push_back(q);
+      }
+    }
   }
-  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
-  if (e != cudaSuccess) {
-    grid_spec_free(s);
-    return set_error(GRID_E_CUDA, std::string("grid_specialize: ") + cudaGetErrorString(e));
+  t.n_tbl = (int)tq.size();
+  t.ncls = t.ci_on ? (int)ncls : 0;
+  t.nselw = (t.ncls + 31) / 32;
+  if ((rc = a.upload(tq, &t.tbl_q)) || (rc = a.upload(tbl_of_q, &t.tbl_of_q))) return fail(rc);
+  if ((rc = set_smem_limits())) return fail(rc);
+  int dev = 0;
+  cudaGetDevice(&dev);
+  s->device = dev;
+  cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
+  // CI classification on the device
+  uint16_t* cls_sp = nullptr;
+  int32_t* cd_count = nullptr;
+  uint16_t* cls_by_id = nullptr;
+  uint8_t* fb = nullptr;
+  if ((rc = a.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&cls_sp)) ||
+      (rc = a.alloc((size_t)t.n_tbl * 4, (void**)&cd_count)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.V * 2, (void**)&cls_by_id)) || (rc = a.alloc((size_t)t.V, (void**)&fb)))
+    return fail(rc);
+  t.cls_by_id = cls_by_id;
+  t.first_byte_by_id = fb;
+  GRID_CUDA(cudaMemsetAsync(cd_count, 0, (size_t)t.n_tbl * 4, st));
+  {
+    dim3 grid(std::max(1, std::min((t.NS + 255) / 256, 4 * s->sms)), t.n_tbl);
+    k_classify<<<grid, 256, t.blob_bytes, st>>>(t, cls_sp, cd_count);
   }
-  cudaGetDevice(&s->device);
+  std::vector<int32_t> counts(t.n_tbl);
+  GRID_CUDA(cudaMemcpyAsync(counts.data(), cd_count, t.n_tbl * 4, cudaMemcpyDeviceToHost, st));
+  GRID_CUDA(cudaStreamSynchronize(st));
+  std::vector<int32_t> cdoff(t.n_tbl + 1, 0);
+  for (int k = 0; k < t.n_tbl; ++k) cdoff[k + 1] = cdoff[k] + counts[k];
+  int32_t* cd_list = nullptr;
+  if ((rc = a.upload(cdoff, &t.cd_off)) || (rc = a.alloc((size_t)cdoff.back() * 4, (void**)&cd_list)))
+    return fail(rc);
+  t.cd_list = cd_list;
+  k_compact<<<t.n_tbl, 1024, 0, st>>>(cls_sp, t.NS, t.cd_off, cd_list);
+  k_permute<<<(t.V + 255) / 256, 256, 0, st>>>(t, cls_sp, cls_by_id, fb);
+  GRID_CUDA(cudaGetLastError());
+  GRID_CUDA(cudaStreamSynchronize(st));
+  s->n1 = (counts[0] + kSpan - 1) / kSpan;
+  int per_sm = 0;
+  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, t.blob_bytes));
+  s->walk_blocks = std::max(1, per_sm) * s->sms;
   *out = s;
+  return GRID_OK;
+}
+
+extern "C" int grid_spec_info(const grid_spec* s, int64_t out[8]) {
+  if (!s || !out) return set_error(GRID_E_INVALID_ARG, "grid_spec_info: bad arguments");
+  const Tables& t = s->t;
+  std::vector<int32_t> off(t.n_tbl + 1);
+  GRID_CUDA(cudaMemcpy(off.data(), t.cd_off, (t.n_tbl + 1) * 4, cudaMemcpyDeviceToHost));
+  out[0] = t.n_tbl;
+  out[1] = t.ncls;
+  out[2] = off[1] - off[0];
+  out[3] = off[t.n_tbl];
+  out[4] = t.blob_bytes;
+  out[5] = s->n1;
+  out[6] = t.ci_on;
+  out[7] = t.NS;
   return GRID_OK;
 }
 
 extern "C" void grid_spec_free(grid_spec* s) {
   if (!s) return;
-  for (void* p : s->owned) cudaFree(p);
+  s->mem.release();
   delete s;
 }
 
@@ -689,18 +941,16 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
   c->B = B;
   c->D = s->t.D;
   c->words_ns = (s->t.NS + 31) / 32 + 1;
-  auto alloc = [&](void** p, size_t n) -> int {
-    GRID_CUDA(cudaMalloc(p, n));
-    c->owned.push_back(*p);
-    return GRID_OK;
-  };
+  Arena& a = c->mem;
   int rc;
-  if ((rc = alloc((void**)&c->c.stack, (size_t)B * c->D * sizeof(uint16_t))) ||
-      (rc = alloc((void**)&c->c.depth, B * sizeof(int32_t))) || (rc = alloc((void**)&c->c.q, B * sizeof(int32_t))) ||
-      (rc = alloc((void**)&c->c.lx, B * sizeof(int32_t))) ||
-      (rc = alloc((void**)&c->c.flags, B * sizeof(int32_t))) ||
-      (rc = alloc((void**)&c->ctx, B * sizeof(RowCtx))) ||
-      (rc = alloc((void**)&c->verd, (size_t)B * c->words_ns * sizeof(uint32_t)))) {
+  if ((rc = a.alloc((size_t)B * c->D * sizeof(uint16_t), (void**)&c->c.stack)) ||
+      (rc = a.alloc(B * 4, (void**)&c->c.depth)) || (rc = a.alloc(B * 4, (void**)&c->c.q)) ||
+      (rc = a.alloc(B * 4, (void**)&c->c.lx)) || (rc = a.alloc(B * 4, (void**)&c->c.flags)) ||
+      (rc = a.alloc(B * sizeof(RowCtx), (void**)&c->ctx)) ||
+      (rc = a.alloc(B * sizeof(RowRanges), (void**)&c->rng)) ||
+      (rc = a.alloc((size_t)B * 2 * std::max(1, s->t.nselw) * 4, (void**)&c->sel)) ||
+      (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd0)) ||
+      (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd1))) {
     grid_configs_free(c);
     return rc;
   }
@@ -716,7 +966,7 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
 
 extern "C" void grid_configs_free(grid_configs* c) {
   if (!c) return;
-  for (void* p : c->owned) cudaFree(p);
+  c->mem.release();
   delete c;
 }
 
@@ -732,8 +982,8 @@ extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_con
   if (!s || !in || !out || !d_tokens || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
     return set_error(GRID_E_INVALID_ARG, "grid_advance: bad arguments");
   const int B = in->B;
-  k_advance<<<(B + 3) / 4, 128, 0, (cudaStream_t)stream>>>(s->t, in->c, out->c, d_tokens, n_steps, d_status, B,
-                                                          in != out ? 1 : 0);
+  k_advance<<<(B + kPrepWarps - 1) / kPrepWarps, kPrepWarps * 32, s->t.blob_bytes, (cudaStream_t)stream>>>(
+      s->t, in->c, out->c, d_tokens, n_steps, d_status, B, in != out ? 1 : 0);
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
@@ -744,12 +994,14 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
   cudaStream_t st = (cudaStream_t)stream;
   const Tables& t = s->t;
   const int B = c->B;
-  k_prep<<<(B + 3) / 4, 128, 0, st>>>(t, c->c, c->ctx, c->verd, B, c->words_ns);
-  const int per_block = kWalkWarps * kWalkSpan;
-  dim3 gw((t.NS + per_block - 1) / per_block, B);
-  if (t.NS > 0) k_walk<<<gw, kWalkWarps * 32, 0, st>>>(t, c->c, c->ctx, c->verd, c->words_ns);
-  dim3 gp((t.W + 7) / 8, B);
-  k_pack<<<gp, 256, 0, st>>>(t, c->ctx, c->verd, c->words_ns, d_mask, d_status);
+  const int zero_blocks = std::min(128, (int)(((size_t)B * c->words_ns / 4 + 1023) / 1024) + 1);
+  k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(
+      t, c->c, c->ctx, c->rng, c->sel, c->verd0, c->verd1, B, c->words_ns);
+  k_walk<<<s->walk_blocks, kWalkWarps * 32, t.blob_bytes, st>>>(t, c->ctx, c->rng, c->c.stack, c->verd0,
+                                                                          c->verd1, c->words_ns, B);
+  dim3 gp((t.V + 1023) / 1024, B);
+  k_pack<<<gp, 256, 2 * std::max(1, t.nselw) * 4, st>>>(t, c->ctx, c->sel, c->verd0, c->verd1, c->words_ns, d_mask,
+                                                        d_status);
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }

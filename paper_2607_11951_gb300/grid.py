@@ -23,7 +23,7 @@ GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 
 EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
-            "grid_spec_free", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
+            "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
             "grid_advance", "grid_masks", "grid_apply_mask", "grid_configs_export"]
 
 
@@ -69,6 +69,7 @@ def lib():
         "grid_vocab_info": (I32, [P, ctypes.POINTER(I64)]),
         "grid_specialize": (I32, [P, P, P, ctypes.POINTER(P)]),
         "grid_spec_free": (None, [P]),
+        "grid_spec_info": (I32, [P, ctypes.POINTER(I64)]),
         "grid_configs_create": (I32, [P, I32, ctypes.POINTER(P)]),
         "grid_configs_free": (None, [P]),
         "grid_configs_reset": (I32, [P, P, P]),
@@ -178,6 +179,14 @@ def grid_specialize(g, v, stream=None):
     return out
 
 
+def grid_spec_info(spec):
+    out = (ctypes.c_int64 * 8)()
+    _check(lib().grid_spec_info(spec, out))
+    keys = ["ci_tables", "ci_classes", "cd_start", "cd_total", "staged_bytes", "walk_blocks_start",
+            "ci_on", "spellings"]
+    return dict(zip(keys, list(out)))
+
+
 def grid_configs_create(spec, B: int):
     out = ctypes.c_void_p()
     _check(lib().grid_configs_create(spec, B, ctypes.byref(out)))
@@ -261,6 +270,9 @@ class Spec:
         self.V = vocab.V
         self.W = (vocab.V + 31) // 32
         self.h = grid_specialize(grammar.h, vocab.h, stream)
+
+    def info(self):
+        return grid_spec_info(self.h)
 
     def __del__(self):
         if getattr(self, "h", None) and _lib is not None:
