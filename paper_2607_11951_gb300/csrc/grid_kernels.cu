@@ -13,6 +13,8 @@
 //            byte ends the lexeme must go through) -> sigma' and A1 = A(sigma');
 //            EOS gate (Sec. 3.2); class selections of both contexts; the
 //            first-byte ranges that continue the pending lexeme
+//   k_succ   per row, context and allowed terminal tau: the allowed set after
+//            shifting tau, so walks simulate nothing before their second shift
 //   k_walk   CD spellings only: lanes walk token bytes through the DFA and the
 //            identifier trie, emissions pick the highest-priority parser-viable
 //            candidate on a copy-on-write overlay; a rejected prefix skips its
@@ -36,8 +38,15 @@ namespace grid {
 namespace {
 
 constexpr int kWalkWarps = 8;    // warps per k_walk block
-constexpr int kSpan = 64;        // list entries / spellings per warp task
+constexpr int kSpan = 32;        // CD list entries per walk item (one warp batch)
 constexpr int kPrepWarps = 4;    // rows per k_prep block
+constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_prep/k_advance
+constexpr int kPackRows = 32;    // rows staged at a time by k_pack
+constexpr int kRangeSpan = 64;   // continuing first-byte ranges are walked in items of this many spellings
+constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
+constexpr int kSuccWarps = 8;    // warps per k_succ block
+constexpr int kSuccSlots = 4;    // k_succ blocks per (row, context)
+constexpr int kLaneOvl = 32;     // overlay / scratch entries per walk lane (shared memory)
 constexpr int kMaxStage = 96 * 1024;
 
 #define GRID_CUDA(call)                                                                  \
@@ -52,6 +61,7 @@ struct RowCtx {
   uint32_t A0[4];   // allowed terminals at sigma
   uint32_t A1[4];   // allowed terminals at sigma' (after the forced emission)
   int32_t q, lx, depth, tbl0;
+  uint32_t pc0, wc0;  // category bits of the pending lexeme's trie node
   int32_t emit_ok, eos_ok, status, complete;
   uint32_t nonempty, done_blocks;
   int32_t keep1, m1;
@@ -88,7 +98,8 @@ __global__ void k_reset(DevConfigs c, int B, int D) {
 }
 
 // ---------------- specialization ----------------
-__global__ void k_classify(Tables t, uint16_t* __restrict__ cls_sp, int32_t* __restrict__ cd_count) {
+__global__ void k_classify(Tables t, uint16_t* __restrict__ cls_sp, uint16_t* __restrict__ key_sp,
+                           uint32_t* __restrict__ pair_sp, int32_t* __restrict__ cd_count) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
@@ -100,14 +111,17 @@ __global__ void k_classify(Tables t, uint16_t* __restrict__ cls_sp, int32_t* __r
     const int off = t.spell_off[s];
     const int len = t.spell_off[s + 1] - off;
     const uint8_t* by = t.spell_bytes + off;
-    uint16_t code;
+    uint16_t code, key = 0xFFFF;
+    uint32_t pair = 0u;
     if (!t.ci_on)
       code = kClsCD;
     else if (q0 != kStart && ts.next[q0 * ts.C + ts.byte_class[by[0]]] == kDead)
       code = kClsNA;
     else
-      code = classify(ts, q0, lx0, by, len);
+      code = classify(ts, q0, lx0, by, len, key, pair);
     cls_sp[(size_t)tbl * t.NS + s] = code;
+    key_sp[(size_t)tbl * t.NS + s] = key;
+    pair_sp[(size_t)tbl * t.NS + s] = pair;
     cd += code == kClsCD;
   }
   cd = __reduce_add_sync(0xffffffffu, cd);
@@ -115,8 +129,9 @@ __global__ void k_classify(Tables t, uint16_t* __restrict__ cls_sp, int32_t* __r
 }
 
 // One block per table: ordered stream compaction of the CD spellings.
-__global__ void k_compact(const uint16_t* __restrict__ cls_sp, int NS, const int32_t* __restrict__ cd_off,
-                          int32_t* __restrict__ cd_list) {
+__global__ void k_compact(const uint16_t* __restrict__ cls_sp, const uint16_t* __restrict__ key_sp, int NS,
+                          const int32_t* __restrict__ cd_off, int32_t* __restrict__ cd_list,
+                          uint16_t* __restrict__ cd_key) {
   __shared__ int32_t warp_tot[32];
   __shared__ int32_t base;
   const int tbl = blockIdx.x;
@@ -131,7 +146,11 @@ __global__ void k_compact(const uint16_t* __restrict__ cls_sp, int NS, const int
     __syncthreads();
     int before = 0;
     for (int k = 0; k < warp; ++k) before += warp_tot[k];
-    if (f) cd_list[base + before + __popc(bal & ((1u << lane) - 1u))] = s;
+    if (f) {
+      const int at = base + before + __popc(bal & ((1u << lane) - 1u));
+      cd_list[at] = s;
+      cd_key[at] = key_sp[(size_t)tbl * NS + s];
+    }
     __syncthreads();
     if (threadIdx.x == 0) {
       int tot = 0;
@@ -142,17 +161,24 @@ __global__ void k_compact(const uint16_t* __restrict__ cls_sp, int NS, const int
   }
 }
 
-__global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, uint16_t* __restrict__ cls_by_id,
+__global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const uint32_t* __restrict__ pair_sp,
+                          uint16_t* __restrict__ cls_by_id, uint32_t* __restrict__ pair_by_id,
                           uint8_t* __restrict__ fb_by_id) {
   const int id = blockIdx.x * blockDim.x + threadIdx.x;
   if (id >= t.V) return;
   const int s = t.spell_of_id[id];
   fb_by_id[id] = s >= 0 ? t.spell_bytes[t.spell_off[s]] : 0;
-  for (int k = 0; k < t.n_tbl; ++k) cls_by_id[(size_t)k * t.V + id] = s >= 0 ? cls_sp[(size_t)k * t.NS + s] : kClsNA;
+  for (int k = 0; k < t.n_tbl; ++k) {
+    cls_by_id[(size_t)k * t.V + id] = s >= 0 ? cls_sp[(size_t)k * t.NS + s] : kClsNA;
+    pair_by_id[(size_t)k * t.V + id] = s >= 0 ? pair_sp[(size_t)k * t.NS + s] : 0u;
+  }
 }
 
 // ---------------- mask step ----------------
-__device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* out, int lane) {
+// Class selection for allowed set A: bit c = set(c) meets A u I.  With `pick`,
+// also the first terminal of set(c) & A (0xFF if none), i.e. the terminal a
+// first stack-dependent emission of class c shifts.
+__device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* out, uint8_t* pick, int lane) {
   uint32_t AI[4];
 #pragma unroll
   for (int k = 0; k < 4; ++k) AI[k] = A[k] | t.ignored[k];
@@ -163,6 +189,11 @@ __device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* o
       uint32_t S[4];
       class_set(t, cls, S);
       v = (S[0] & AI[0]) | (S[1] & AI[1]) | (S[2] & AI[2]) | (S[3] & AI[3]);
+      if (pick) {
+        const uint32_t SA[4] = {S[0] & A[0], S[1] & A[1], S[2] & A[2], S[3] & A[3]};
+        const int f = lowest4(SA);
+        pick[cls] = f < 0 ? 0xFF : (uint8_t)f;
+      }
     }
     const uint32_t word = __ballot_sync(0xffffffffu, v);
     if (lane == 0) out[w0] = word;
@@ -178,7 +209,7 @@ __device__ void allowed_set(const Tables& t, const uint16_t* base, int keep, con
     if (tau < t.n_term && !bit4(t.ignored, tau)) {
       uint16_t scr[kMaxOvl];
       int keep_o, m_o, ns;
-      int a = simulate(t, base, keep, ovl, m, tau, scr, keep_o, m_o, ns, mc);
+      int a = simulate(t, base, keep, ovl, m, tau, LArr{scr, 1}, kMaxOvl, keep_o, m_o, ns, mc);
       ok = a > 0 && a != kAccept;
       if (a < 0) status = GRID_ST_BOUND;
     }
@@ -187,11 +218,11 @@ __device__ void allowed_set(const Tables& t, const uint16_t* base, int keep, con
 }
 
 __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
-                                                          RowRanges* __restrict__ rng, uint32_t* __restrict__ sel,
-                                                          uint32_t* __restrict__ verd0, uint32_t* __restrict__ verd1,
-                                                          int B, int words_ns) {
+                                                          RowRanges* __restrict__ rng, uint32_t* __restrict__ verd0,
+                                                          uint32_t* __restrict__ verd1, int B, int words_ns) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kPrepWarps][kMaxOvl];
+  __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
   __shared__ int s_km[kPrepWarps][3];
   const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
   if ((int)blockIdx.x >= row_blocks) {
@@ -218,8 +249,15 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   if (b >= B) return;
   RowCtx& r = ctx[b];
   const int complete = c.flags[b] & 1;
-  const uint16_t* base = c.stack + (size_t)b * t.D;
+  const uint16_t* gbase = c.stack + (size_t)b * t.D;
   const int depth = c.depth[b], q = c.q[b], lx = c.lx[b];
+  const uint32_t pc0 = lx >= 0 ? t.lx_pcats[lx] : 0u, wc0 = lx >= 0 ? t.lx_wcats[lx] : 0u;
+  const uint16_t* base = gbase;
+  if (depth <= kStackWin) {  // the reduce chains below read the stack top repeatedly
+    for (int i = lane; i < depth; i += 32) s_stk[warp][i] = gbase[i];
+    __syncwarp();
+    base = s_stk[warp];
+  }
   const int mc = max_chain_of(t);
   int status = complete ? GRID_ST_COMPLETE : GRID_ST_OK;
   uint32_t A0[4] = {0, 0, 0, 0}, A1[4] = {0, 0, 0, 0};
@@ -229,16 +267,12 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
     if (!complete) {
       Walker w;
-      w.base = base;
-      w.keep = depth;
-      w.m = 0;
-      w.q = q;
-      w.lx = lx;
-      w.shifted = false;
+      uint16_t lo[kMaxOvl], ls[kMaxOvl];
+      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, A0, nullptr);
       if (q == kStart) {
         emit_ok = 1;
       } else {
-        int e = emit(ts, w, A0, mc);
+        int e = emit(ts, w, mc);
         if (e < 0) status = GRID_ST_BOUND;
         emit_ok = e > 0;
         keep1 = w.keep;
@@ -246,13 +280,8 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
         for (int i = 0; i < m1; ++i) s_ovl[warp][i] = w.ovl[i];
       }
       Walker w2;
-      w2.base = base;
-      w2.keep = depth;
-      w2.m = 0;
-      w2.q = q;
-      w2.lx = lx;
-      w2.shifted = false;
-      int g = eos_gate(ts, w2, A0, mc);
+      walker_init(w2, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, A0, nullptr);
+      int g = eos_gate(ts, w2, mc);
       if (g < 0) status = GRID_ST_BOUND;
       eos = g > 0;
     }
@@ -272,12 +301,6 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   }
   status = __reduce_max_sync(0xffffffffu, status);
   const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
-  uint32_t* sel0 = sel + (size_t)b * 2 * t.nselw;
-  uint32_t* sel1 = sel0 + t.nselw;
-  if (!complete && t.ci_on) {
-    if (tbl0 >= 0) select_classes(ts, A0, sel0, lane);
-    if (emit_ok) select_classes(ts, A1, sel1, lane);
-  }
   // continuing first-byte ranges (rows without a CI table for q)
   int total0 = 0, nrng = 0;
   if (!complete && q != kStart) {
@@ -290,7 +313,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
         const int by = b0 + lane;
         const int lo = t.first_of_byte[by], hi = t.first_of_byte[by + 1];
         const bool cont = hi > lo && ts.next[q * ts.C + ts.byte_class[by]] != kDead;
-        const int chunks = cont ? (hi - lo + kSpan - 1) / kSpan : 0;
+        const int chunks = cont ? (hi - lo + kRangeSpan - 1) / kRangeSpan : 0;
         const uint32_t bal = __ballot_sync(0xffffffffu, cont);
         int incl = chunks;
         for (int d = 1; d < 32; d <<= 1) {
@@ -318,6 +341,8 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     }
     r.q = q;
     r.lx = lx;
+    r.pc0 = pc0;
+    r.wc0 = wc0;
     r.depth = depth;
     r.tbl0 = tbl0;
     r.emit_ok = emit_ok;
@@ -340,146 +365,290 @@ struct WalkCtx {
   int keep, m;
   const uint16_t* ovl;
   int q, lx;
+  uint32_t pc, wc;
   int kill_q;  // >= 0: spellings whose first byte continues this DFA state are skipped
   uint32_t A[4];
+  const uint32_t* A2;  // allowed sets after the first shift, per terminal (4 words each)
 };
 
-// Walk list positions [p0, p1) (list == NULL: spelling indices).  Verdict bits
-// go to vb (spelling order).
-__device__ void walk_span(const Tables& t, const WalkCtx& wc, const int32_t* __restrict__ list, int p0, int p1,
-                          uint32_t* __restrict__ vb, int& bound) {
+// grid = (B, 2, kSuccSlots): row b, context cx (0: sigma, 1: sigma' after the
+// forced emission).  Jobs j = 0..n_term of a (row, context) are spread over
+// its kSuccSlots * kSuccWarps warps.  Job tau < n_term, for tau allowed in the
+// context: the allowed set after tau's reduce chain and shift (A2) and its
+// class selection (sel2), so that walks simulate nothing before their second
+// shift and two-event spellings need no walk.  Job n_term: the context's own
+// class selection and, per emission class, the terminal it would shift (pick).
+__global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c, const RowCtx* __restrict__ ctx,
+                                                          uint32_t* __restrict__ A2, uint32_t* __restrict__ sel2,
+                                                          uint32_t* __restrict__ sel, uint8_t* __restrict__ pick) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ Tables ts;
+  __shared__ uint16_t s_win[kWalkWin];
+  __shared__ uint16_t s_ovl1[kMaxOvl];
+  __shared__ uint16_t s_ovl2[kSuccWarps][kMaxOvl];
+  __shared__ int s_keep2[kSuccWarps], s_m2[kSuccWarps];
+  const int b = blockIdx.x, cx = blockIdx.y;
+  const RowCtx& r = ctx[b];
+  if (r.complete || (cx == 1 && !r.emit_ok) || (cx == 0 && r.q == kStart)) return;
+  stage_tables(t, ts, smem);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int depth = r.depth;
+  const uint16_t* base = c.stack + (size_t)b * t.D;
+  const int m = cx ? r.m1 : 0;
+  for (int i = threadIdx.x; i < m; i += blockDim.x) s_ovl1[i] = r.ovl1[i];
+  if (depth <= kWalkWin) {
+    for (int i = threadIdx.x; i < depth; i += blockDim.x) s_win[i] = base[i];
+    base = s_win;
+  }
+  __syncthreads();
+  const int keep = cx ? r.keep1 : depth;
+  uint32_t A[4];
+  for (int k = 0; k < 4; ++k) A[k] = cx ? r.A1[k] : r.A0[k];
+  const int mc = max_chain_of(t);
+  uint32_t* out = A2 + ((size_t)b * 2 + cx) * t.T1 * 4;
+  int status = GRID_ST_OK;
+  const int nw = kSuccSlots * kSuccWarps;
+  for (int j = blockIdx.z * kSuccWarps + warp; j <= t.n_term; j += nw) {
+    if (j == t.n_term) {
+      if (t.ci_on && (cx == 1 || r.tbl0 >= 0))
+        select_classes(ts, A, sel + ((size_t)b * 2 + cx) * t.nselw, pick + ((size_t)b * 2 + cx) * t.ncls, lane);
+      continue;
+    }
+    const int tau = j;
+    if (!bit4(A, tau)) continue;
+    if (lane == 0) {
+      uint16_t scr[kMaxOvl];
+      int keep_o, m_o, ns;
+      const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, LArr{scr, 1}, kMaxOvl, keep_o, m_o, ns, mc);
+      int m2 = -1;
+      if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
+        for (int i = 0; i < m_o; ++i) s_ovl2[warp][i] = s_ovl1[i];
+        for (int i = 0; i < ns; ++i) s_ovl2[warp][m_o + i] = scr[i];
+        s_ovl2[warp][m_o + ns] = (uint16_t)(a - 1);
+        m2 = m_o + ns + 1;
+      }
+      s_keep2[warp] = keep_o;
+      s_m2[warp] = m2;
+    }
+    __syncwarp();
+    const int m2 = s_m2[warp];
+    uint32_t An[4] = {0, 0, 0, 0};
+    if (m2 > 0)
+      allowed_set(ts, base, s_keep2[warp], s_ovl2[warp], m2, An, status, lane);
+    else
+      status = GRID_ST_BOUND;
+    if (lane == 0)
+      for (int k = 0; k < 4; ++k) out[tau * 4 + k] = An[k];
+    if (t.ci_on) select_classes(ts, An, sel2 + (((size_t)b * 2 + cx) * t.T1 + tau) * t.nselw, nullptr, lane);
+    __syncwarp();
+  }
+  status = __reduce_max_sync(0xffffffffu, status);
+  if (lane == 0 && status != GRID_ST_OK) atomicCAS(const_cast<int32_t*>(&ctx[b].status), GRID_ST_OK, status);
+}
+
+// Walk the spellings [p0, p1) of a continuing first-byte range.  Verdict bits
+// go to vb (spelling order).  When the last lane's spelling is rejected, every
+// spelling sharing its rejected prefix is skipped (a trie subtree, contiguous
+// in DFS order).
+__device__ void walk_span(const Tables& t, const WalkCtx& wc, int p0, int p1, uint32_t* __restrict__ vb, int& bound,
+                          uint16_t* lane_store) {
   const int lane = threadIdx.x & 31;
   const int mc = max_chain_of(t);
+  const LArr lo{lane_store + lane, 32}, ls{lane_store + kLaneOvl * 32 + lane, 32};
   Walker w;
   for (int pos = p0; pos < p1;) {
-    const int i = pos + lane;
-    int s = -1, ok = 0, rej = -1;
-    if (i < p1) {
-      s = list ? list[i] : i;
-      const int off = t.spell_off[s];
-      const int len = t.spell_off[s + 1] - off;
-      const uint8_t* by = t.spell_bytes + off;
-      if (wc.kill_q >= 0 && t.next[wc.kill_q * t.C + t.byte_class[by[0]]] != kDead) {
-        rej = 0;  // continues the pending lexeme: handled by the other context
-      } else {
-        w.base = wc.base;
-        w.keep = wc.keep;
-        w.m = wc.m;
-        for (int k = 0; k < wc.m; ++k) w.ovl[k] = wc.ovl[k];
-        w.q = wc.q;
-        w.lx = wc.lx;
-        w.shifted = false;
-        const int r = walk_bytes(t, w, by, len, wc.A, mc, rej);
-        if (r < 0) {
-          bound = 1;
-          rej = -1;
-        }
-        ok = r > 0;
+    const int s = pos + lane;
+    int ok = 0, rej = -1;
+    if (s < p1) {
+      const Spell sp = load_spell(t, s);
+      walker_init(w, lo, ls, kLaneOvl, wc.base, wc.keep, wc.ovl, wc.m, wc.q, wc.lx, wc.pc, wc.wc, wc.A, wc.A2);
+      const int r = walk_bytes(t, w, sp, mc, rej);
+      if (r < 0) {
+        bound = 1;
+        rej = -1;
       }
+      ok = r > 0;
     }
-    if (list) {
-      if (ok) atomicOr(&vb[s >> 5], 1u << (s & 31));
-    } else {
-      const uint32_t m = __ballot_sync(0xffffffffu, ok);
-      if (lane == 0 && m) {
-        const int sh = pos & 31;
-        atomicOr(&vb[pos >> 5], m << sh);
-        if (sh && (m >> (32 - sh))) atomicOr(&vb[(pos >> 5) + 1], m >> (32 - sh));
-      }
+    const uint32_t m = __ballot_sync(0xffffffffu, ok);
+    if (lane == 0 && m) {
+      const int sh = pos & 31;
+      atomicOr(&vb[pos >> 5], m << sh);
+      if (sh && (m >> (32 - sh))) atomicOr(&vb[(pos >> 5) + 1], m >> (32 - sh));
     }
     int nxt = pos + 32;
     const int last = min(31, p1 - 1 - pos);
     const int lrej = __shfl_sync(0xffffffffu, rej, last);
-    const int ls = __shfl_sync(0xffffffffu, s, last);
-    if (lrej >= 0) {
-      const int sk = t.skip[t.spell_off[ls] + lrej];
-      if (list) {
-        int lo = nxt, hi = p1;
-        while (lo < hi) {
-          const int mid = (lo + hi) >> 1;
-          if (list[mid] < sk)
-            lo = mid + 1;
-          else
-            hi = mid;
-        }
-        nxt = lo;
-      } else {
-        nxt = max(nxt, sk);
-      }
-    }
+    if (lrej >= 0) nxt = max(nxt, t.skip[t.spell_off[pos + last] + lrej]);
     pos = nxt;
   }
 }
 
-// Persistent walk.  Every row owns one work queue of chunks: chunks
+// Walk the CD spellings list[p0:p1) of one row (p1 - p0 <= 32).  A spelling
+// is walked only if the class of its first stack-dependent emission is
+// selected for the context's allowed set (`sel`; otherwise that emission, and
+// so the spelling, fails) and, for the sigma' context, if its first byte ends
+// the pending lexeme.  Survivors are compacted so that lanes stay busy.
+__device__ void walk_list(const Tables& t, const WalkCtx& wc, const int32_t* __restrict__ list,
+                          const uint16_t* __restrict__ keys, int p0, int p1, const uint32_t* __restrict__ sel,
+                          uint32_t* __restrict__ vb, int& bound, uint16_t* lane_store) {
+  const int lane = threadIdx.x & 31;
+  const int mc = max_chain_of(t);
+  const LArr lo{lane_store + lane, 32}, ls{lane_store + kLaneOvl * 32 + lane, 32};
+  const int i = p0 + lane;
+  bool pass = false;
+  int s = -1;
+  Spell sp;
+  if (i < p1) {
+    s = list[i];
+    const uint16_t k = keys[i];
+    pass = k == 0xFFFF || ((sel[k >> 5] >> (k & 31)) & 1u);
+    if (pass) {
+      sp = load_spell(t, s);
+      if (wc.kill_q >= 0) pass = t.next[wc.kill_q * t.C + t.byte_class[sp.at(0)]] == kDead;
+    }
+  }
+  const uint32_t bal = __ballot_sync(0xffffffffu, pass);
+  if (!bal) return;
+  // compact the survivors onto the low lanes
+  const int dst = __popc(bal & ((1u << lane) - 1u));
+  const int n = __popc(bal);
+  int src_lane = 0;
+  {
+    // lane d takes the d-th set bit of bal
+    uint32_t rest = bal;
+    for (int d = 0; d < lane && rest; ++d) rest &= rest - 1;
+    src_lane = rest ? __ffs(rest) - 1 : 0;
+  }
+  (void)dst;
+  const int s2 = __shfl_sync(0xffffffffu, s, src_lane);
+  const uint4 h2 = make_uint4(__shfl_sync(0xffffffffu, sp.head.x, src_lane), __shfl_sync(0xffffffffu, sp.head.y, src_lane),
+                              __shfl_sync(0xffffffffu, sp.head.z, src_lane), __shfl_sync(0xffffffffu, sp.head.w, src_lane));
+  const int len2 = __shfl_sync(0xffffffffu, sp.len, src_lane);
+  if (lane < n) {
+    Spell sp2;
+    sp2.head = h2;
+    sp2.len = len2;
+    sp2.all = t.spell_bytes + t.spell_off[s2];
+    Walker w;
+    walker_init(w, lo, ls, kLaneOvl, wc.base, wc.keep, wc.ovl, wc.m, wc.q, wc.lx, wc.pc, wc.wc, wc.A, wc.A2);
+    int rej;
+    const int r = walk_bytes(t, w, sp2, mc, rej);
+    if (r < 0) bound = 1;
+    if (r > 0) atomicOr(&vb[s2 >> 5], 1u << (s2 & 31));
+  }
+}
+
+// Persistent walk.  Every row owns one work queue of items: items
 // [0, total1) cover the start state's CD list under sigma' (tokens whose first
-// byte ends the pending lexeme), chunks [total1, total) the spellings that
+// byte ends the pending lexeme), items [total1, total) the spellings that
 // continue the pending lexeme (the CD list of its lexer state, or its
 // continuing first-byte ranges).  Warps start at different rows, drain a row's
-// queue chunk by chunk and move on; a warp stops after finding every queue
-// empty once in a row.
+// queue item by item and move on; a warp stops after finding every queue
+// empty once in a row.  A warp keeps the current row's context (allowed sets,
+// sigma' overlay, stack mirror) until it moves to another row.
 __global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __restrict__ ctx,
                                                           const RowRanges* __restrict__ rng, const uint16_t* stacks,
-                                                          uint32_t* __restrict__ verd0, uint32_t* __restrict__ verd1,
-                                                          int words_ns, int B) {
+                                                          const uint32_t* __restrict__ sel,
+                                                          const uint32_t* __restrict__ A2, uint32_t* __restrict__ verd0,
+                                                          uint32_t* __restrict__ verd1, int words_ns, int B) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
+  __shared__ uint16_t s_win[kWalkWarps][kWalkWin];
+  __shared__ uint16_t s_lane[kWalkWarps][2 * kLaneOvl * 32];
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWalkWarps + warp;
   const int start_len = t.cd_off[1] - t.cd_off[0];
   const int32_t* start_list = t.cd_list + t.cd_off[0];
+  const uint16_t* start_keys = t.cd_key + t.cd_off[0];
   int row = gw % B;
   int fails = 0;
   int bound = 0, bound_row = -1;
+  int cur = -1;  // row whose context is cached below
+  int total1 = 0, tbl0 = -1, depth = 0, q = 0, lx = 0, keep1 = 0, m1 = 0, nrng = 0;
+  uint32_t pc0 = 0, wc0 = 0, A0[4] = {0, 0, 0, 0}, A1[4] = {0, 0, 0, 0};
+  const uint16_t* base = stacks;
   while (fails < B) {
     RowCtx& r = ctx[row];
-    const int total = r.total0;
-    int cidx = total;
-    if (lane == 0 && *((volatile int32_t*)&r.work0) < total) cidx = atomicAdd(&r.work0, 1);
+    int cidx = 0, total = 0;
+    if (lane == 0) {
+      total = r.total0;
+      cidx = *((volatile int32_t*)&r.work0) < total ? atomicAdd(&r.work0, 1) : total;
+    }
     cidx = __shfl_sync(0xffffffffu, cidx, 0);
+    total = __shfl_sync(0xffffffffu, total, 0);
     if (cidx >= total) {
       ++fails;
       row = row + 1 == B ? 0 : row + 1;
       continue;
     }
     fails = 0;
-    const int total1 = r.total1;
+    if (cur != row) {
+      cur = row;
+      total1 = r.total1;
+      tbl0 = r.tbl0;
+      depth = r.depth;
+      q = r.q;
+      lx = r.lx;
+      pc0 = r.pc0;
+      wc0 = r.wc0;
+      keep1 = r.keep1;
+      m1 = r.m1;
+      nrng = r.nrng;
+      for (int k = 0; k < 4; ++k) {
+        A0[k] = r.A0[k];
+        A1[k] = r.A1[k];
+      }
+      __syncwarp();
+      for (int i = lane; i < m1 && i < kMaxOvl; i += 32) s_ovl[warp][i] = r.ovl1[i];
+      base = stacks + (size_t)row * t.D;
+      if (depth <= kWalkWin) {  // mirror the row's stack: reduce chains read its top repeatedly
+        for (int i = lane; i < depth; i += 32) s_win[warp][i] = base[i];
+        base = s_win[warp];
+      }
+      __syncwarp();
+    }
+    const bool c1 = cidx < total1;
     WalkCtx wc;
-    wc.base = stacks + (size_t)row * t.D;
-    if (cidx < total1) {
-      const int m1 = r.m1;
-      __syncwarp();
-      for (int i = lane; i < m1; i += 32) s_ovl[warp][i] = r.ovl1[i];
-      __syncwarp();
-      wc.keep = r.keep1;
-      wc.m = m1;
-      wc.ovl = s_ovl[warp];
-      wc.q = kStart;
-      wc.lx = 0;
-      wc.kill_q = r.q == kStart ? -1 : r.q;
-      for (int k = 0; k < 4; ++k) wc.A[k] = r.A1[k];
-      const int p0 = cidx * kSpan;
-      walk_span(ts, wc, start_list, p0, min(start_len, p0 + kSpan), verd1 + (size_t)row * words_ns, bound);
+    wc.base = base;
+    wc.A2 = A2 + ((size_t)row * 2 + (c1 ? 1 : 0)) * t.T1 * 4;
+    if (c1) {
+      if (m1 > kLaneOvl) {
+        bound = 1;  // sigma' overlay larger than a walk lane holds: flag the row
+      } else {
+        wc.keep = keep1;
+        wc.m = m1;
+        wc.ovl = s_ovl[warp];
+        wc.q = kStart;
+        wc.lx = 0;
+        wc.pc = t.root_pc;
+        wc.wc = t.root_wc;
+        wc.kill_q = q == kStart ? -1 : q;
+        for (int k = 0; k < 4; ++k) wc.A[k] = A1[k];
+        const int p0 = cidx * kSpan;
+        walk_list(ts, wc, start_list, start_keys, p0, min(start_len, p0 + kSpan),
+                  sel + ((size_t)row * 2 + 1) * t.nselw, verd1 + (size_t)row * words_ns, bound, s_lane[warp]);
+      }
     } else {
       const int c0 = cidx - total1;
-      wc.keep = r.depth;
+      wc.keep = depth;
       wc.m = 0;
       wc.ovl = s_ovl[warp];
-      wc.q = r.q;
-      wc.lx = r.lx;
+      wc.q = q;
+      wc.lx = lx;
+      wc.pc = pc0;
+      wc.wc = wc0;
       wc.kill_q = -1;
-      for (int k = 0; k < 4; ++k) wc.A[k] = r.A0[k];
-      const int tbl0 = r.tbl0;
+      for (int k = 0; k < 4; ++k) wc.A[k] = A0[k];
       if (tbl0 >= 0) {
-        const int32_t* list = t.cd_list + t.cd_off[tbl0];
         const int len = t.cd_off[tbl0 + 1] - t.cd_off[tbl0];
         const int p0 = c0 * kSpan;
-        walk_span(ts, wc, list, p0, min(len, p0 + kSpan), verd0 + (size_t)row * words_ns, bound);
+        walk_list(ts, wc, t.cd_list + t.cd_off[tbl0], t.cd_key + t.cd_off[tbl0], p0, min(len, p0 + kSpan),
+                  sel + (size_t)row * 2 * t.nselw, verd0 + (size_t)row * words_ns, bound, s_lane[warp]);
       } else {
         const RowRanges& R = rng[row];
-        int lo = 0, hi = r.nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
+        int lo = 0, hi = nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
         while (hi - lo > 1) {
           const int mid = (lo + hi) >> 1;
           if (R.cpre[mid] <= c0)
@@ -487,8 +656,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __re
           else
             hi = mid;
         }
-        const int p0 = R.lo[lo] + (c0 - R.cpre[lo]) * kSpan;
-        walk_span(ts, wc, nullptr, p0, min(R.hi[lo], p0 + kSpan), verd0 + (size_t)row * words_ns, bound);
+        const int p0 = R.lo[lo] + (c0 - R.cpre[lo]) * kRangeSpan;
+        walk_span(ts, wc, p0, min(R.hi[lo], p0 + kRangeSpan), verd0 + (size_t)row * words_ns, bound, s_lane[warp]);
       }
     }
     if (bound && bound_row < 0) bound_row = row;
@@ -496,74 +665,110 @@ __global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __re
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
 }
 
-// grid = (ceil(V/1024), B), 256 threads x 4 token ids.
+// Verdict of a kClsCD2 spelling in context cx of row b: its first emission
+// shifts pick[key1] (none: rejected); the second event is decided by the class
+// selection after that shift.
+__device__ __forceinline__ bool cd2_bit(const Tables& t, const uint8_t* __restrict__ pick,
+                                        const uint32_t* __restrict__ sel2, int b, int cx, uint32_t pair) {
+  const uint32_t key1 = pair >> 16, key2 = pair & 0xFFFFu;
+  const int tau = pick[((size_t)b * 2 + cx) * t.ncls + key1];
+  if (tau == 0xFF) return false;
+  return (sel2[(((size_t)b * 2 + cx) * t.T1 + tau) * t.nselw + (key2 >> 5)] >> (key2 & 31)) & 1u;
+}
+
 __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
+                                              const uint8_t* __restrict__ pick, const uint32_t* __restrict__ sel2,
                                               const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
-                                              int words_ns, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status) {
-  extern __shared__ __align__(16) uint32_t s_sel[];  // 2 * nselw
-  __shared__ __align__(16) RowCtx s_r;
-  const int b = blockIdx.y;
-  {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(&ctx[b]);
-    uint32_t* dst = reinterpret_cast<uint32_t*>(&s_r);
-    for (int i = threadIdx.x; i < (int)(sizeof(RowCtx) / 4); i += blockDim.x) dst[i] = src[i];
-  }
-  for (int i = threadIdx.x; i < 2 * t.nselw; i += blockDim.x) s_sel[i] = sel[(size_t)b * 2 * t.nselw + i];
-  __syncthreads();
-  const RowCtx& r = s_r;
+                                              int words_ns, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
+                                              int B) {
+  extern __shared__ __align__(16) uint32_t s_sel[];  // kPackRows * 2 * nselw
+  __shared__ int s_q[kPackRows], s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
+  __shared__ int s_last;
+  const int id = blockIdx.x * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31;
-  const uint32_t* v0 = verd0 + (size_t)b * words_ns;
-  const uint32_t* v1 = verd1 + (size_t)b * words_ns;
-  const uint16_t* cls0 = r.tbl0 >= 0 ? t.cls_by_id + (size_t)r.tbl0 * t.V : nullptr;
-  int any = 0;
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int id = (blockIdx.x * 4 + k) * blockDim.x + threadIdx.x;
-    bool bit = false;
-    if (id < t.V && !r.complete) {
-      if (id == t.eos) {
-        bit = r.eos_ok != 0;
-      } else {
-        const int s = t.spell_of_id[id];
-        if (s >= 0) {
-          const int b0 = t.first_byte_by_id[id];
-          const bool kills = r.q == kStart || t.next[r.q * t.C + t.byte_class[b0]] == kDead;
+  const int wi = id >> 5;
+  int s = -1, b0 = 0;
+  uint16_t cl_start = kClsNA;
+  if (id < t.V && id != t.eos) {
+    s = t.spell_of_id[id];
+    if (s >= 0) {
+      b0 = t.first_byte_by_id[id];
+      cl_start = t.cls_by_id[id];
+    }
+  }
+  const int bc = t.byte_class[b0];
+  const int nw = t.nselw;
+  for (int r0 = 0; r0 < B; r0 += kPackRows) {
+    const int nr = min(kPackRows, B - r0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nr; i += blockDim.x) {
+      const RowCtx& rc = ctx[r0 + i];
+      s_q[i] = rc.q;
+      s_tbl[i] = rc.tbl0;
+      s_fl[i] = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
+      s_any[i] = 0;
+    }
+    for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) s_sel[i] = sel[(size_t)r0 * 2 * nw + i];
+    __syncthreads();
+    for (int k = 0; k < nr; ++k) {
+      const int b = r0 + k;
+      const int fl = s_fl[k];
+      bool bit = false;
+      if (id < t.V && !(fl & 4)) {
+        if (id == t.eos) {
+          bit = fl & 2;
+        } else if (s >= 0) {
+          const int q = s_q[k];
+          const bool kills = q == kStart || t.next[q * t.C + bc] == kDead;
           if (kills) {
-            if (r.emit_ok) {
-              const uint16_t cl = t.cls_by_id[id];
-              if (cl < kClsNA)
-                bit = (s_sel[t.nselw + (cl >> 5)] >> (cl & 31)) & 1u;
+            if (fl & 1) {
+              const uint16_t cl = cl_start;
+              if (cl < kClsFirstCode)
+                bit = (s_sel[(2 * k + 1) * nw + (cl >> 5)] >> (cl & 31)) & 1u;
               else if (cl == kClsAcc)
                 bit = true;
               else if (cl == kClsCD)
-                bit = (v1[s >> 5] >> (s & 31)) & 1u;
+                bit = (verd1[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
+              else if (cl == kClsCD2)
+                bit = cd2_bit(t, pick, sel2, b, 1, t.pair_by_id[id]);
             }
-          } else if (cls0) {
-            const uint16_t cl = cls0[id];
-            if (cl < kClsNA)
-              bit = (s_sel[cl >> 5] >> (cl & 31)) & 1u;
-            else if (cl == kClsAcc)
-              bit = true;
-            else if (cl == kClsCD)
-              bit = (v0[s >> 5] >> (s & 31)) & 1u;
           } else {
-            bit = (v0[s >> 5] >> (s & 31)) & 1u;
+            const int tbl0 = s_tbl[k];
+            if (tbl0 >= 0) {
+              const uint16_t cl = t.cls_by_id[(size_t)tbl0 * t.V + id];
+              if (cl < kClsFirstCode)
+                bit = (s_sel[2 * k * nw + (cl >> 5)] >> (cl & 31)) & 1u;
+              else if (cl == kClsAcc)
+                bit = true;
+              else if (cl == kClsCD)
+                bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
+              else if (cl == kClsCD2)
+                bit = cd2_bit(t, pick, sel2, b, 0, t.pair_by_id[(size_t)tbl0 * t.V + id]);
+            } else {
+              bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
+            }
           }
         }
       }
+      const uint32_t word = __ballot_sync(0xffffffffu, bit);
+      if (lane == 0 && wi < t.W) {
+        mask[(size_t)b * t.W + wi] = word;
+        if (word) s_any[k] = 1;
+      }
     }
-    const uint32_t word = __ballot_sync(0xffffffffu, bit);
-    const int wi = id >> 5;
-    if (lane == 0 && wi < t.W) mask[(size_t)b * t.W + wi] = word;
-    any |= word != 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < nr; i += blockDim.x)
+      if (s_any[i]) atomicOr(&ctx[r0 + i].nonempty, 1u);
   }
-  any = __syncthreads_or(any);
+  __syncthreads();
   if (threadIdx.x == 0) {
-    if (any) atomicOr(&ctx[b].nonempty, 1u);
     __threadfence();
-    const unsigned prev = atomicAdd(&ctx[b].done_blocks, 1u);
-    if (prev == gridDim.x - 1) {
-      __threadfence();
+    s_last = atomicAdd(&ctx[0].done_blocks, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    for (int b = threadIdx.x; b < B; b += blockDim.x) {
       int st = atomicAdd(&ctx[b].status, 0);
       if (st == GRID_ST_OK && atomicAdd(&ctx[b].nonempty, 0u) == 0u) st = GRID_ST_EMPTY_MASK;
       d_status[b] = st;
@@ -577,9 +782,10 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
                                                              int32_t* __restrict__ d_status, int B, int copy) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
+  __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
   stage_tables(t, ts, smem);
-  const int lane = threadIdx.x & 31;
-  const int b = blockIdx.x * kPrepWarps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int b = blockIdx.x * kPrepWarps + warp;
   if (b >= B) return;
   if (copy) {
     const int d = cin.depth[b];
@@ -592,12 +798,22 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
     }
     __syncwarp();
   }
-  if (lane != 0) return;
   uint16_t* stack = cout.stack + (size_t)b * t.D;
-  int depth = cout.depth[b], q = cout.q[b], lx = cout.lx[b], flags = cout.flags[b];
+  // the row's stack is mirrored in shared memory while it fits; the global
+  // copy is always written and stays authoritative
+  const int depth0 = copy ? cin.depth[b] : cout.depth[b];
+  const uint16_t* src = copy ? cin.stack + (size_t)b * t.D : stack;
+  bool use_win = depth0 <= kStackWin;
+  if (use_win)
+    for (int i = lane; i < depth0; i += 32) s_stk[warp][i] = src[i];
+  __syncwarp();
+  if (lane != 0) return;
+  int depth = depth0, q = cout.q[b], lx = cout.lx[b], flags = cout.flags[b];
+  uint32_t pc = lx >= 0 ? t.lx_pcats[lx] : 0u, wcat = lx >= 0 ? t.lx_wcats[lx] : 0u;
   int status = GRID_ST_OK;
   const int mc = max_chain_of(t);
   Walker w;
+  uint16_t lo[kMaxOvl], ls[kMaxOvl];
   for (int k = 0; k < n_steps; ++k) {
     const int tok = tokens[(size_t)b * n_steps + k];
     if (tok < 0) continue;
@@ -609,14 +825,10 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
       status = GRID_ST_TOKEN_NOT_ALLOWED;
       break;
     }
-    w.base = stack;
-    w.keep = depth;
-    w.m = 0;
-    w.q = q;
-    w.lx = lx;
-    w.shifted = false;
+    walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, use_win ? s_stk[warp] : stack, depth, nullptr, 0, q, lx, pc,
+                wcat, nullptr, nullptr);
     if (tok == t.eos) {
-      const int e = eos_gate(ts, w, nullptr, mc);
+      const int e = eos_gate(ts, w, mc);
       if (e < 0) {
         status = GRID_ST_BOUND;
         break;
@@ -633,9 +845,8 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
       status = GRID_ST_TOKEN_NOT_ALLOWED;
       break;
     }
-    const int off = t.spell_off[s];
     int rej;
-    const int r = walk_bytes(ts, w, t.spell_bytes + off, t.spell_off[s + 1] - off, nullptr, mc, rej);
+    const int r = walk_bytes(ts, w, load_spell(t, s), mc, rej);
     if (r < 0) {
       status = GRID_ST_BOUND;
       break;
@@ -649,9 +860,16 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
       break;
     }
     for (int i = 0; i < w.m; ++i) stack[w.keep + i] = w.ovl[i];
+    if (use_win && w.keep + w.m <= kStackWin) {
+      for (int i = 0; i < w.m; ++i) s_stk[warp][w.keep + i] = w.ovl[i];
+    } else {
+      use_win = false;
+    }
     depth = w.keep + w.m;
     q = w.q;
     lx = w.lx;
+    pc = w.pc;
+    wcat = w.wc;
   }
   cout.depth[b] = depth;
   cout.q[b] = q;
@@ -764,6 +982,9 @@ struct grid_configs {
   uint32_t* sel = nullptr;
   uint32_t* verd0 = nullptr;
   uint32_t* verd1 = nullptr;
+  uint32_t* A2 = nullptr;
+  uint8_t* pick = nullptr;
+  uint32_t* sel2 = nullptr;
   Arena mem;
 };
 
@@ -775,6 +996,7 @@ static int set_smem_limits() {
   GRID_CUDA(cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_succ, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   return GRID_OK;
 }
@@ -842,19 +1064,56 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   t.plen = dblob + off[6];
   t.plhs = reinterpret_cast<const uint16_t*>(dblob + off[7]);
   Arena& a = s->mem;
+  {
+    // identifier-trie edges -> open-addressing hash (load factor <= 1/2)
+    const size_t edges = h.lx_cbyte.size();
+    int bits = 4;
+    while ((size_t(1) << bits) < 2 * edges + 2) ++bits;
+    std::vector<uint32_t> hv4((size_t(4) << bits), 0u);
+    for (size_t i = 0; i < (size_t(1) << bits); ++i) hv4[4 * i] = kHashEmpty;
+    const uint32_t mask = (1u << bits) - 1u;
+    for (int n = 0; n < h.LN; ++n)
+      for (int e = h.lx_cstart[n]; e < h.lx_cstart[n + 1]; ++e) {
+        const uint32_t key = (uint32_t)n * 256u + h.lx_cbyte[e];
+        uint32_t hh = (key * 0x9E3779B1u) >> (32 - bits);
+        while (hv4[4 * hh] != kHashEmpty) hh = (hh + 1u) & mask;
+        const int child = h.lx_cnode[e];
+        hv4[4 * hh] = key;
+        hv4[4 * hh + 1] = (uint32_t)child;
+        hv4[4 * hh + 2] = h.lx_pcats[child];
+        hv4[4 * hh + 3] = h.lx_wcats[child];
+      }
+    const uint32_t* dh = nullptr;
+    if ((rc = a.upload(hv4, &dh))) return fail(rc);
+    t.lx_hash = reinterpret_cast<const uint4*>(dh);
+    t.lx_hmask = mask;
+    t.lx_hshift = 32 - bits;
+    t.root_pc = h.LN > 0 ? h.lx_pcats[0] : 0u;
+    t.root_wc = h.LN > 0 ? h.lx_wcats[0] : 0u;
+  }
   if ((rc = a.upload(h.lx_cstart, &t.lx_cstart)) || (rc = a.upload(h.lx_cbyte, &t.lx_cbyte)) ||
       (rc = a.upload(h.lx_cnode, &t.lx_cnode)) || (rc = a.upload(h.lx_pcats, &t.lx_pcats)) ||
       (rc = a.upload(h.lx_wcats, &t.lx_wcats)) || (rc = a.upload(hv.spell_off, &t.spell_off)) ||
       (rc = a.upload(hv.spell_bytes, &t.spell_bytes)) || (rc = a.upload(hv.skip, &t.skip)) ||
       (rc = a.upload(hv.spell_of_id, &t.spell_of_id)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
     return fail(rc);
+  {
+    std::vector<uint32_t> s16((size_t)hv.NS * 4, 0u);
+    for (int sp = 0; sp < hv.NS; ++sp) {
+      const int off = hv.spell_off[sp], len = std::min(16, hv.spell_off[sp + 1] - off);
+      std::memcpy(reinterpret_cast<uint8_t*>(s16.data() + (size_t)sp * 4), hv.spell_bytes.data() + off, len);
+    }
+    const uint32_t* d16 = nullptr;
+    if ((rc = a.upload(s16, &d16))) return fail(rc);
+    t.spell16 = reinterpret_cast<const uint4*>(d16);
+  }
   // precomputed lexer states: the start state and every state at which no
   // lexicon category is live (there the lexicon node cannot matter)
   std::vector<int32_t> tq{kStart};
   std::vector<int16_t> tbl_of_q(h.Q, -1);
   tbl_of_q[kStart] = 0;
   const long ncls = (long)(2 * h.Q) << h.n_cat;
-  t.ci_on = ncls < (long)kClsNA ? 1 : 0;
+  t.ci_on = ncls < (long)kClsFirstCode ? 1 : 0;
   if (t.ci_on) {
     for (int q = 2; q < h.Q; ++q) {
       bool catlive = false;
@@ -877,19 +1136,26 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
   // CI classification on the device
   uint16_t* cls_sp = nullptr;
+  uint16_t* key_sp = nullptr;
+  uint32_t* pair_sp = nullptr;
+  uint32_t* pair_by_id = nullptr;
   int32_t* cd_count = nullptr;
   uint16_t* cls_by_id = nullptr;
   uint8_t* fb = nullptr;
   if ((rc = a.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&cls_sp)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&key_sp)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.NS * 4, (void**)&pair_sp)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.V * 4, (void**)&pair_by_id)) ||
       (rc = a.alloc((size_t)t.n_tbl * 4, (void**)&cd_count)) ||
       (rc = a.alloc((size_t)t.n_tbl * t.V * 2, (void**)&cls_by_id)) || (rc = a.alloc((size_t)t.V, (void**)&fb)))
     return fail(rc);
   t.cls_by_id = cls_by_id;
+  t.pair_by_id = pair_by_id;
   t.first_byte_by_id = fb;
   GRID_CUDA(cudaMemsetAsync(cd_count, 0, (size_t)t.n_tbl * 4, st));
   {
     dim3 grid(std::max(1, std::min((t.NS + 255) / 256, 4 * s->sms)), t.n_tbl);
-    k_classify<<<grid, 256, t.blob_bytes, st>>>(t, cls_sp, cd_count);
+    k_classify<<<grid, 256, t.blob_bytes, st>>>(t, cls_sp, key_sp, pair_sp, cd_count);
   }
   std::vector<int32_t> counts(t.n_tbl);
   GRID_CUDA(cudaMemcpyAsync(counts.data(), cd_count, t.n_tbl * 4, cudaMemcpyDeviceToHost, st));
@@ -897,16 +1163,19 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   std::vector<int32_t> cdoff(t.n_tbl + 1, 0);
   for (int k = 0; k < t.n_tbl; ++k) cdoff[k + 1] = cdoff[k] + counts[k];
   int32_t* cd_list = nullptr;
-  if ((rc = a.upload(cdoff, &t.cd_off)) || (rc = a.alloc((size_t)cdoff.back() * 4, (void**)&cd_list)))
+  uint16_t* cd_key = nullptr;
+  if ((rc = a.upload(cdoff, &t.cd_off)) || (rc = a.alloc((size_t)cdoff.back() * 4, (void**)&cd_list)) ||
+      (rc = a.alloc((size_t)cdoff.back() * 2, (void**)&cd_key)))
     return fail(rc);
   t.cd_list = cd_list;
-  k_compact<<<t.n_tbl, 1024, 0, st>>>(cls_sp, t.NS, t.cd_off, cd_list);
-  k_permute<<<(t.V + 255) / 256, 256, 0, st>>>(t, cls_sp, cls_by_id, fb);
+  t.cd_key = cd_key;
+  k_compact<<<t.n_tbl, 1024, 0, st>>>(cls_sp, key_sp, t.NS, t.cd_off, cd_list, cd_key);
+  k_permute<<<(t.V + 255) / 256, 256, 0, st>>>(t, cls_sp, pair_sp, cls_by_id, pair_by_id, fb);
   GRID_CUDA(cudaGetLastError());
   GRID_CUDA(cudaStreamSynchronize(st));
   s->n1 = (counts[0] + kSpan - 1) / kSpan;
   int per_sm = 0;
-  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, t.blob_bytes));
+  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, 0));
   s->walk_blocks = std::max(1, per_sm) * s->sms;
   *out = s;
   return GRID_OK;
@@ -950,7 +1219,10 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
       (rc = a.alloc(B * sizeof(RowRanges), (void**)&c->rng)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->t.nselw) * 4, (void**)&c->sel)) ||
       (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd0)) ||
-      (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd1))) {
+      (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd1)) ||
+      (rc = a.alloc((size_t)B * 2 * s->t.T1 * 16, (void**)&c->A2)) ||
+      (rc = a.alloc((size_t)B * 2 * std::max(1, s->t.ncls), (void**)&c->pick)) ||
+      (rc = a.alloc((size_t)B * 2 * s->t.T1 * std::max(1, s->t.nselw) * 4, (void**)&c->sel2))) {
     grid_configs_free(c);
     return rc;
   }
@@ -996,12 +1268,15 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
   const int B = c->B;
   const int zero_blocks = std::min(128, (int)(((size_t)B * c->words_ns / 4 + 1023) / 1024) + 1);
   k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(
-      t, c->c, c->ctx, c->rng, c->sel, c->verd0, c->verd1, B, c->words_ns);
-  k_walk<<<s->walk_blocks, kWalkWarps * 32, t.blob_bytes, st>>>(t, c->ctx, c->rng, c->c.stack, c->verd0,
-                                                                          c->verd1, c->words_ns, B);
-  dim3 gp((t.V + 1023) / 1024, B);
-  k_pack<<<gp, 256, 2 * std::max(1, t.nselw) * 4, st>>>(t, c->ctx, c->sel, c->verd0, c->verd1, c->words_ns, d_mask,
-                                                        d_status);
+      t, c->c, c->ctx, c->rng, c->verd0, c->verd1, B, c->words_ns);
+  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c->c, c->ctx, c->A2, c->sel2, c->sel,
+                                                                        c->pick);
+  Tables tw = t;  // the walk reads the small tables through L1; its shared memory holds lane overlays
+  tw.blob_bytes = 0;
+  k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, c->ctx, c->rng, c->c.stack, c->sel, c->A2, c->verd0,
+                                                     c->verd1, c->words_ns, B);
+  k_pack<<<(t.V + 255) / 256, 256, kPackRows * 2 * std::max(1, t.nselw) * 4, st>>>(
+      t, c->ctx, c->sel, c->pick, c->sel2, c->verd0, c->verd1, c->words_ns, d_mask, d_status, B);
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
