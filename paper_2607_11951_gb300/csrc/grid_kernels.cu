@@ -41,7 +41,7 @@ constexpr int kWalkWarps = 8;    // warps per k_walk block
 constexpr int kSpan = 32;        // CD list entries per walk item (one warp batch)
 constexpr int kPrepWarps = 4;    // rows per k_prep block
 constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_prep/k_advance
-constexpr int kPackRows = 32;    // rows staged at a time by k_pack
+constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 64;   // continuing first-byte ranges are walked in items of this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
 constexpr int kSuccWarps = 8;    // warps per k_succ block
@@ -68,6 +68,7 @@ struct RowCtx {
   int32_t work0, total0;  // chunk counter / chunks of the row's walk queue
   int32_t total1;         // leading chunks of the queue that belong to sigma' 
   int32_t nrng;
+  uint32_t kill[8];  // bit b: first byte b ends the pending lexeme
   uint16_t ovl1[kMaxOvl];
 };
 
@@ -200,16 +201,17 @@ __device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* o
   }
 }
 
+// A(sigma) for the virtual stack base[0:keep] ++ ovl[0:m]: lane l simulates
+// terminals l, l+32, ...; `scr` is the lane's scratch (kMaxOvl entries).
 __device__ void allowed_set(const Tables& t, const uint16_t* base, int keep, const uint16_t* ovl, int m,
-                            uint32_t A[4], int& status, int lane) {
+                            uint32_t A[4], int& status, int lane, LArr scr) {
   const int mc = max_chain_of(t);
   for (int wd = 0; wd < 4; ++wd) {
     const int tau = wd * 32 + lane;
     bool ok = false;
     if (tau < t.n_term && !bit4(t.ignored, tau)) {
-      uint16_t scr[kMaxOvl];
       int keep_o, m_o, ns;
-      int a = simulate(t, base, keep, ovl, m, tau, LArr{scr, 1}, kMaxOvl, keep_o, m_o, ns, mc);
+      int a = simulate(t, base, keep, ovl, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
       ok = a > 0 && a != kAccept;
       if (a < 0) status = GRID_ST_BOUND;
     }
@@ -223,6 +225,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kPrepWarps][kMaxOvl];
   __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
+  __shared__ uint16_t s_scr[kPrepWarps][kMaxOvl * 32];
   __shared__ int s_km[kPrepWarps][3];
   const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
   if ((int)blockIdx.x >= row_blocks) {
@@ -261,7 +264,8 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   const int mc = max_chain_of(t);
   int status = complete ? GRID_ST_COMPLETE : GRID_ST_OK;
   uint32_t A0[4] = {0, 0, 0, 0}, A1[4] = {0, 0, 0, 0};
-  if (!complete) allowed_set(ts, base, depth, nullptr, 0, A0, status, lane);
+  const LArr scr{s_scr[warp] + lane, 32};
+  if (!complete) allowed_set(ts, base, depth, nullptr, 0, A0, status, lane, scr);
   // forced emission of the pending lexeme + EOS gate (lane 0)
   if (lane == 0) {
     int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
@@ -296,7 +300,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     if (keep1 == depth && m1 == 0) {
       for (int k = 0; k < 4; ++k) A1[k] = A0[k];
     } else {
-      allowed_set(ts, base, keep1, s_ovl[warp], m1, A1, status, lane);
+      allowed_set(ts, base, keep1, s_ovl[warp], m1, A1, status, lane, scr);
     }
   }
   status = __reduce_max_sync(0xffffffffu, status);
@@ -332,6 +336,13 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
       if (lane == 0) R.cpre[nrng] = total0;
     }
   }
+  // first bytes that end the pending lexeme (every byte when it is empty)
+  for (int b0 = 0; b0 < 256; b0 += 32) {
+    const int by = b0 + lane;
+    const bool kill = q == kStart || ts.next[q * ts.C + ts.byte_class[by]] == kDead;
+    const uint32_t word = __ballot_sync(0xffffffffu, kill);
+    if (lane == 0) r.kill[b0 >> 5] = word;
+  }
   const int start_len = t.cd_off[1] - t.cd_off[0];
   const int total1 = (!complete && emit_ok) ? (start_len + kSpan - 1) / kSpan : 0;
   if (lane == 0) {
@@ -360,16 +371,6 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   for (int i = lane; i < m1; i += 32) r.ovl1[i] = s_ovl[warp][i];
 }
 
-struct WalkCtx {
-  const uint16_t* base;
-  int keep, m;
-  const uint16_t* ovl;
-  int q, lx;
-  uint32_t pc, wc;
-  int kill_q;  // >= 0: spellings whose first byte continues this DFA state are skipped
-  uint32_t A[4];
-  const uint32_t* A2;  // allowed sets after the first shift, per terminal (4 words each)
-};
 
 // grid = (B, 2, kSuccSlots): row b, context cx (0: sigma, 1: sigma' after the
 // forced emission).  Jobs j = 0..n_term of a (row, context) are spread over
@@ -386,6 +387,7 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   __shared__ uint16_t s_win[kWalkWin];
   __shared__ uint16_t s_ovl1[kMaxOvl];
   __shared__ uint16_t s_ovl2[kSuccWarps][kMaxOvl];
+  __shared__ uint16_t s_scr[kSuccWarps][kMaxOvl * 32];
   __shared__ int s_keep2[kSuccWarps], s_m2[kSuccWarps];
   const int b = blockIdx.x, cx = blockIdx.y;
   const RowCtx& r = ctx[b];
@@ -416,10 +418,10 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
     }
     const int tau = j;
     if (!bit4(A, tau)) continue;
+    const LArr scr{s_scr[warp] + lane, 32};
     if (lane == 0) {
-      uint16_t scr[kMaxOvl];
       int keep_o, m_o, ns;
-      const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, LArr{scr, 1}, kMaxOvl, keep_o, m_o, ns, mc);
+      const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
       int m2 = -1;
       if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
         for (int i = 0; i < m_o; ++i) s_ovl2[warp][i] = s_ovl1[i];
@@ -434,7 +436,7 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
     const int m2 = s_m2[warp];
     uint32_t An[4] = {0, 0, 0, 0};
     if (m2 > 0)
-      allowed_set(ts, base, s_keep2[warp], s_ovl2[warp], m2, An, status, lane);
+      allowed_set(ts, base, s_keep2[warp], s_ovl2[warp], m2, An, status, lane, scr);
     else
       status = GRID_ST_BOUND;
     if (lane == 0)
@@ -446,98 +448,6 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   if (lane == 0 && status != GRID_ST_OK) atomicCAS(const_cast<int32_t*>(&ctx[b].status), GRID_ST_OK, status);
 }
 
-// Walk the spellings [p0, p1) of a continuing first-byte range.  Verdict bits
-// go to vb (spelling order).  When the last lane's spelling is rejected, every
-// spelling sharing its rejected prefix is skipped (a trie subtree, contiguous
-// in DFS order).
-__device__ void walk_span(const Tables& t, const WalkCtx& wc, int p0, int p1, uint32_t* __restrict__ vb, int& bound,
-                          uint16_t* lane_store) {
-  const int lane = threadIdx.x & 31;
-  const int mc = max_chain_of(t);
-  const LArr lo{lane_store + lane, 32}, ls{lane_store + kLaneOvl * 32 + lane, 32};
-  Walker w;
-  for (int pos = p0; pos < p1;) {
-    const int s = pos + lane;
-    int ok = 0, rej = -1;
-    if (s < p1) {
-      const Spell sp = load_spell(t, s);
-      walker_init(w, lo, ls, kLaneOvl, wc.base, wc.keep, wc.ovl, wc.m, wc.q, wc.lx, wc.pc, wc.wc, wc.A, wc.A2);
-      const int r = walk_bytes(t, w, sp, mc, rej);
-      if (r < 0) {
-        bound = 1;
-        rej = -1;
-      }
-      ok = r > 0;
-    }
-    const uint32_t m = __ballot_sync(0xffffffffu, ok);
-    if (lane == 0 && m) {
-      const int sh = pos & 31;
-      atomicOr(&vb[pos >> 5], m << sh);
-      if (sh && (m >> (32 - sh))) atomicOr(&vb[(pos >> 5) + 1], m >> (32 - sh));
-    }
-    int nxt = pos + 32;
-    const int last = min(31, p1 - 1 - pos);
-    const int lrej = __shfl_sync(0xffffffffu, rej, last);
-    if (lrej >= 0) nxt = max(nxt, t.skip[t.spell_off[pos + last] + lrej]);
-    pos = nxt;
-  }
-}
-
-// Walk the CD spellings list[p0:p1) of one row (p1 - p0 <= 32).  A spelling
-// is walked only if the class of its first stack-dependent emission is
-// selected for the context's allowed set (`sel`; otherwise that emission, and
-// so the spelling, fails) and, for the sigma' context, if its first byte ends
-// the pending lexeme.  Survivors are compacted so that lanes stay busy.
-__device__ void walk_list(const Tables& t, const WalkCtx& wc, const int32_t* __restrict__ list,
-                          const uint16_t* __restrict__ keys, int p0, int p1, const uint32_t* __restrict__ sel,
-                          uint32_t* __restrict__ vb, int& bound, uint16_t* lane_store) {
-  const int lane = threadIdx.x & 31;
-  const int mc = max_chain_of(t);
-  const LArr lo{lane_store + lane, 32}, ls{lane_store + kLaneOvl * 32 + lane, 32};
-  const int i = p0 + lane;
-  bool pass = false;
-  int s = -1;
-  Spell sp;
-  if (i < p1) {
-    s = list[i];
-    const uint16_t k = keys[i];
-    pass = k == 0xFFFF || ((sel[k >> 5] >> (k & 31)) & 1u);
-    if (pass) {
-      sp = load_spell(t, s);
-      if (wc.kill_q >= 0) pass = t.next[wc.kill_q * t.C + t.byte_class[sp.at(0)]] == kDead;
-    }
-  }
-  const uint32_t bal = __ballot_sync(0xffffffffu, pass);
-  if (!bal) return;
-  // compact the survivors onto the low lanes
-  const int dst = __popc(bal & ((1u << lane) - 1u));
-  const int n = __popc(bal);
-  int src_lane = 0;
-  {
-    // lane d takes the d-th set bit of bal
-    uint32_t rest = bal;
-    for (int d = 0; d < lane && rest; ++d) rest &= rest - 1;
-    src_lane = rest ? __ffs(rest) - 1 : 0;
-  }
-  (void)dst;
-  const int s2 = __shfl_sync(0xffffffffu, s, src_lane);
-  const uint4 h2 = make_uint4(__shfl_sync(0xffffffffu, sp.head.x, src_lane), __shfl_sync(0xffffffffu, sp.head.y, src_lane),
-                              __shfl_sync(0xffffffffu, sp.head.z, src_lane), __shfl_sync(0xffffffffu, sp.head.w, src_lane));
-  const int len2 = __shfl_sync(0xffffffffu, sp.len, src_lane);
-  if (lane < n) {
-    Spell sp2;
-    sp2.head = h2;
-    sp2.len = len2;
-    sp2.all = t.spell_bytes + t.spell_off[s2];
-    Walker w;
-    walker_init(w, lo, ls, kLaneOvl, wc.base, wc.keep, wc.ovl, wc.m, wc.q, wc.lx, wc.pc, wc.wc, wc.A, wc.A2);
-    int rej;
-    const int r = walk_bytes(t, w, sp2, mc, rej);
-    if (r < 0) bound = 1;
-    if (r > 0) atomicOr(&vb[s2 >> 5], 1u << (s2 & 31));
-  }
-}
-
 // Persistent walk.  Every row owns one work queue of items: items
 // [0, total1) cover the start state's CD list under sigma' (tokens whose first
 // byte ends the pending lexeme), items [total1, total) the spellings that
@@ -546,15 +456,26 @@ __device__ void walk_list(const Tables& t, const WalkCtx& wc, const int32_t* __r
 // queue item by item and move on; a warp stops after finding every queue
 // empty once in a row.  A warp keeps the current row's context (allowed sets,
 // sigma' overlay, stack mirror) until it moves to another row.
-__global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __restrict__ ctx,
-                                                          const RowRanges* __restrict__ rng, const uint16_t* stacks,
-                                                          const uint32_t* __restrict__ sel,
-                                                          const uint32_t* __restrict__ A2, uint32_t* __restrict__ verd0,
-                                                          uint32_t* __restrict__ verd1, int words_ns, int B) {
+//
+// List items (kSpan CD spellings): a spelling is walked only if the class of
+// its first stack-dependent emission is selected for the context's allowed
+// set (otherwise that emission, and so the spelling, fails) and, for sigma',
+// if its first byte ends the pending lexeme; survivors are compacted onto the
+// low lanes.  Range items (kRangeSpan spellings of one first-byte range):
+// lanes walk consecutive spellings; when the last lane's spelling is rejected,
+// every spelling sharing its rejected prefix is skipped (a trie subtree,
+// contiguous in DFS order).  Both kinds share one call of walk_bytes.
+__global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* __restrict__ ctx,
+                                                             const RowRanges* __restrict__ rng, const uint16_t* stacks,
+                                                             const uint32_t* __restrict__ sel,
+                                                             const uint32_t* __restrict__ A2,
+                                                             uint32_t* __restrict__ verd0,
+                                                             uint32_t* __restrict__ verd1, int words_ns, int B) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
   __shared__ uint16_t s_win[kWalkWarps][kWalkWin];
   __shared__ uint16_t s_lane[kWalkWarps][2 * kLaneOvl * 32];
+  __shared__ uint32_t s_A[kWalkWarps][2][4];  // the cached row's A0 and A1
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -562,12 +483,14 @@ __global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __re
   const int start_len = t.cd_off[1] - t.cd_off[0];
   const int32_t* start_list = t.cd_list + t.cd_off[0];
   const uint16_t* start_keys = t.cd_key + t.cd_off[0];
+  const int mc = max_chain_of(t);
+  const LArr lo{s_lane[warp] + lane, 32}, ls{s_lane[warp] + kLaneOvl * 32 + lane, 32};
   int row = gw % B;
   int fails = 0;
   int bound = 0, bound_row = -1;
   int cur = -1;  // row whose context is cached below
   int total1 = 0, tbl0 = -1, depth = 0, q = 0, lx = 0, keep1 = 0, m1 = 0, nrng = 0;
-  uint32_t pc0 = 0, wc0 = 0, A0[4] = {0, 0, 0, 0}, A1[4] = {0, 0, 0, 0};
+  uint32_t pc0 = 0, wc0 = 0;
   const uint16_t* base = stacks;
   while (fails < B) {
     RowCtx& r = ctx[row];
@@ -596,11 +519,11 @@ __global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __re
       keep1 = r.keep1;
       m1 = r.m1;
       nrng = r.nrng;
-      for (int k = 0; k < 4; ++k) {
-        A0[k] = r.A0[k];
-        A1[k] = r.A1[k];
-      }
       __syncwarp();
+      if (lane < 4) {
+        s_A[warp][0][lane] = r.A0[lane];
+        s_A[warp][1][lane] = r.A1[lane];
+      }
       for (int i = lane; i < m1 && i < kMaxOvl; i += 32) s_ovl[warp][i] = r.ovl1[i];
       base = stacks + (size_t)row * t.D;
       if (depth <= kWalkWin) {  // mirror the row's stack: reduce chains read its top repeatedly
@@ -609,58 +532,114 @@ __global__ void __launch_bounds__(kWalkWarps * 32) k_walk(Tables t, RowCtx* __re
       }
       __syncwarp();
     }
+    // ---- the item: context and source
     const bool c1 = cidx < total1;
-    WalkCtx wc;
-    wc.base = base;
-    wc.A2 = A2 + ((size_t)row * 2 + (c1 ? 1 : 0)) * t.T1 * 4;
+    if (c1 && m1 > kLaneOvl) {  // sigma' overlay larger than a walk lane holds: flag the row
+      bound = 1;
+      bound_row = bound_row < 0 ? row : bound_row;
+      continue;
+    }
+    const uint32_t* Ac = s_A[warp][c1 ? 1 : 0];
+    const uint32_t* A2row = A2 + ((size_t)row * 2 + (c1 ? 1 : 0)) * t.T1 * 4;
+    const int ckeep = c1 ? keep1 : depth, cm = c1 ? m1 : 0;
+    const int cq = c1 ? kStart : q, clx = c1 ? 0 : lx;
+    const uint32_t cpc = c1 ? t.root_pc : pc0, cwc = c1 ? t.root_wc : wc0;
+    const int kill_q = (c1 && q != kStart) ? q : -1;
+    uint32_t* vb = (c1 ? verd1 : verd0) + (size_t)row * words_ns;
+    const int32_t* list = nullptr;
+    const uint16_t* keys = nullptr;
+    const uint32_t* csel = sel + ((size_t)row * 2 + (c1 ? 1 : 0)) * t.nselw;
+    int p0, p1;
     if (c1) {
-      if (m1 > kLaneOvl) {
-        bound = 1;  // sigma' overlay larger than a walk lane holds: flag the row
-      } else {
-        wc.keep = keep1;
-        wc.m = m1;
-        wc.ovl = s_ovl[warp];
-        wc.q = kStart;
-        wc.lx = 0;
-        wc.pc = t.root_pc;
-        wc.wc = t.root_wc;
-        wc.kill_q = q == kStart ? -1 : q;
-        for (int k = 0; k < 4; ++k) wc.A[k] = A1[k];
-        const int p0 = cidx * kSpan;
-        walk_list(ts, wc, start_list, start_keys, p0, min(start_len, p0 + kSpan),
-                  sel + ((size_t)row * 2 + 1) * t.nselw, verd1 + (size_t)row * words_ns, bound, s_lane[warp]);
-      }
+      list = start_list;
+      keys = start_keys;
+      p0 = cidx * kSpan;
+      p1 = min(start_len, p0 + kSpan);
+    } else if (tbl0 >= 0) {
+      const int c0 = cidx - total1;
+      list = t.cd_list + t.cd_off[tbl0];
+      keys = t.cd_key + t.cd_off[tbl0];
+      p0 = c0 * kSpan;
+      p1 = min(t.cd_off[tbl0 + 1] - t.cd_off[tbl0], p0 + kSpan);
     } else {
       const int c0 = cidx - total1;
-      wc.keep = depth;
-      wc.m = 0;
-      wc.ovl = s_ovl[warp];
-      wc.q = q;
-      wc.lx = lx;
-      wc.pc = pc0;
-      wc.wc = wc0;
-      wc.kill_q = -1;
-      for (int k = 0; k < 4; ++k) wc.A[k] = A0[k];
-      if (tbl0 >= 0) {
-        const int len = t.cd_off[tbl0 + 1] - t.cd_off[tbl0];
-        const int p0 = c0 * kSpan;
-        walk_list(ts, wc, t.cd_list + t.cd_off[tbl0], t.cd_key + t.cd_off[tbl0], p0, min(len, p0 + kSpan),
-                  sel + (size_t)row * 2 * t.nselw, verd0 + (size_t)row * words_ns, bound, s_lane[warp]);
-      } else {
-        const RowRanges& R = rng[row];
-        int lo = 0, hi = nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
-        while (hi - lo > 1) {
-          const int mid = (lo + hi) >> 1;
-          if (R.cpre[mid] <= c0)
-            lo = mid;
-          else
-            hi = mid;
+      const RowRanges& R = rng[row];
+      int a = 0, z = nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
+      while (z - a > 1) {
+        const int mid = (a + z) >> 1;
+        if (R.cpre[mid] <= c0)
+          a = mid;
+        else
+          z = mid;
+      }
+      p0 = R.lo[a] + (c0 - R.cpre[a]) * kRangeSpan;
+      p1 = min(R.hi[a], p0 + kRangeSpan);
+    }
+    // ---- one or more warp batches, one walk call site
+    int pos = p0;
+    for (bool first = true;; first = false) {
+      int s = -1;
+      bool go = false;
+      Spell sp;
+      if (list) {
+        if (!first) break;
+        const int i = p0 + lane;
+        bool pass = false;
+        if (i < p1) {
+          s = list[i];
+          const uint16_t k = keys[i];
+          pass = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
+          if (pass) {
+            sp = load_spell(ts, s);
+            if (kill_q >= 0) pass = ts.next[kill_q * ts.C + ts.byte_class[sp.at(0)]] == kDead;
+          }
         }
-        const int p0 = R.lo[lo] + (c0 - R.cpre[lo]) * kRangeSpan;
-        walk_span(ts, wc, p0, min(R.hi[lo], p0 + kRangeSpan), verd0 + (size_t)row * words_ns, bound, s_lane[warp]);
+        const uint32_t bal = __ballot_sync(0xffffffffu, pass);
+        if (!bal) break;
+        uint32_t rest = bal;  // lane d takes the d-th survivor
+        for (int d = 0; d < lane && rest; ++d) rest &= rest - 1;
+        const int src = rest ? __ffs(rest) - 1 : 0;
+        s = __shfl_sync(0xffffffffu, s, src);
+        sp.head.x = __shfl_sync(0xffffffffu, sp.head.x, src);
+        sp.head.y = __shfl_sync(0xffffffffu, sp.head.y, src);
+        sp.head.z = __shfl_sync(0xffffffffu, sp.head.z, src);
+        sp.head.w = __shfl_sync(0xffffffffu, sp.head.w, src);
+        sp.len = __shfl_sync(0xffffffffu, sp.len, src);
+        go = lane < __popc(bal);
+        if (go) sp.all = ts.spell_bytes + ts.spell_off[s];
+      } else {
+        if (pos >= p1) break;
+        s = pos + lane;
+        go = s < p1;
+        if (go) sp = load_spell(ts, s);
+      }
+      int res = 0, rej = -1;
+      if (go) {
+        Walker w;
+        walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
+        res = walk_bytes(ts, w, sp, mc, rej);
+        if (res < 0) {
+          bound = 1;
+          rej = -1;
+          if (bound_row < 0) bound_row = row;
+        }
+      }
+      if (list) {
+        if (res > 0) atomicOr(&vb[s >> 5], 1u << (s & 31));
+      } else {
+        const uint32_t m = __ballot_sync(0xffffffffu, res > 0);
+        if (lane == 0 && m) {
+          const int sh = pos & 31;
+          atomicOr(&vb[pos >> 5], m << sh);
+          if (sh && (m >> (32 - sh))) atomicOr(&vb[(pos >> 5) + 1], m >> (32 - sh));
+        }
+        int nxt = pos + 32;
+        const int last = min(31, p1 - 1 - pos);
+        const int lrej = __shfl_sync(0xffffffffu, rej, last);
+        if (lrej >= 0) nxt = max(nxt, ts.skip[ts.spell_off[pos + last] + lrej]);
+        pos = nxt;
       }
     }
-    if (bound && bound_row < 0) bound_row = row;
   }
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
 }
@@ -676,94 +655,97 @@ __device__ __forceinline__ bool cd2_bit(const Tables& t, const uint8_t* __restri
   return (sel2[(((size_t)b * 2 + cx) * t.T1 + tau) * t.nselw + (key2 >> 5)] >> (key2 & 31)) & 1u;
 }
 
+// grid = (ceil(V/256), ceil(B/kPackRows)), 256 threads: one token id per
+// thread and kPackRows rows per block.  The per-id data (spelling, first byte,
+// start-state class) is loaded once; each warp writes one mask word per row.
+// The last block to finish writes every row's status (EMPTY_MASK for a viable
+// row with no bit set).
 __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
                                               const uint8_t* __restrict__ pick, const uint32_t* __restrict__ sel2,
                                               const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
                                               int words_ns, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
                                               int B) {
   extern __shared__ __align__(16) uint32_t s_sel[];  // kPackRows * 2 * nselw
-  __shared__ int s_q[kPackRows], s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
+  __shared__ int s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
+  __shared__ uint32_t s_kill[kPackRows][8];
   __shared__ int s_last;
   const int id = blockIdx.x * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31;
   const int wi = id >> 5;
+  const int r0 = blockIdx.y * kPackRows;
+  const int nr = min(kPackRows, B - r0);
+  const int nw = t.nselw;
+  for (int i = threadIdx.x; i < nr; i += blockDim.x) {
+    const RowCtx& rc = ctx[r0 + i];
+    s_tbl[i] = rc.tbl0;
+    s_fl[i] = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
+    s_any[i] = 0;
+  }
+  for (int i = threadIdx.x; i < nr * 8; i += blockDim.x) s_kill[i >> 3][i & 7] = ctx[r0 + (i >> 3)].kill[i & 7];
+  for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) s_sel[i] = sel[(size_t)r0 * 2 * nw + i];
   int s = -1, b0 = 0;
   uint16_t cl_start = kClsNA;
+  uint32_t pair_start = 0u;
   if (id < t.V && id != t.eos) {
     s = t.spell_of_id[id];
     if (s >= 0) {
       b0 = t.first_byte_by_id[id];
       cl_start = t.cls_by_id[id];
+      if (cl_start == kClsCD2) pair_start = t.pair_by_id[id];
     }
   }
-  const int bc = t.byte_class[b0];
-  const int nw = t.nselw;
-  for (int r0 = 0; r0 < B; r0 += kPackRows) {
-    const int nr = min(kPackRows, B - r0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < nr; i += blockDim.x) {
-      const RowCtx& rc = ctx[r0 + i];
-      s_q[i] = rc.q;
-      s_tbl[i] = rc.tbl0;
-      s_fl[i] = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
-      s_any[i] = 0;
-    }
-    for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) s_sel[i] = sel[(size_t)r0 * 2 * nw + i];
-    __syncthreads();
-    for (int k = 0; k < nr; ++k) {
-      const int b = r0 + k;
-      const int fl = s_fl[k];
-      bool bit = false;
-      if (id < t.V && !(fl & 4)) {
-        if (id == t.eos) {
-          bit = fl & 2;
-        } else if (s >= 0) {
-          const int q = s_q[k];
-          const bool kills = q == kStart || t.next[q * t.C + bc] == kDead;
-          if (kills) {
-            if (fl & 1) {
-              const uint16_t cl = cl_start;
-              if (cl < kClsFirstCode)
-                bit = (s_sel[(2 * k + 1) * nw + (cl >> 5)] >> (cl & 31)) & 1u;
-              else if (cl == kClsAcc)
-                bit = true;
-              else if (cl == kClsCD)
-                bit = (verd1[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-              else if (cl == kClsCD2)
-                bit = cd2_bit(t, pick, sel2, b, 1, t.pair_by_id[id]);
-            }
-          } else {
-            const int tbl0 = s_tbl[k];
-            if (tbl0 >= 0) {
-              const uint16_t cl = t.cls_by_id[(size_t)tbl0 * t.V + id];
-              if (cl < kClsFirstCode)
-                bit = (s_sel[2 * k * nw + (cl >> 5)] >> (cl & 31)) & 1u;
-              else if (cl == kClsAcc)
-                bit = true;
-              else if (cl == kClsCD)
-                bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-              else if (cl == kClsCD2)
-                bit = cd2_bit(t, pick, sel2, b, 0, t.pair_by_id[(size_t)tbl0 * t.V + id]);
-            } else {
+  __syncthreads();
+  for (int k = 0; k < nr; ++k) {
+    const int b = r0 + k;
+    const int fl = s_fl[k];
+    bool bit = false;
+    if (id < t.V && !(fl & 4)) {
+      if (id == t.eos) {
+        bit = fl & 2;
+      } else if (s >= 0) {
+        if ((s_kill[k][b0 >> 5] >> (b0 & 31)) & 1u) {
+          if (fl & 1) {
+            const uint16_t cl = cl_start;
+            if (cl < kClsFirstCode)
+              bit = (s_sel[(2 * k + 1) * nw + (cl >> 5)] >> (cl & 31)) & 1u;
+            else if (cl == kClsAcc)
+              bit = true;
+            else if (cl == kClsCD)
+              bit = (verd1[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
+            else if (cl == kClsCD2)
+              bit = cd2_bit(t, pick, sel2, b, 1, pair_start);
+          }
+        } else {
+          const int tbl0 = s_tbl[k];
+          if (tbl0 >= 0) {
+            const uint16_t cl = t.cls_by_id[(size_t)tbl0 * t.V + id];
+            if (cl < kClsFirstCode)
+              bit = (s_sel[2 * k * nw + (cl >> 5)] >> (cl & 31)) & 1u;
+            else if (cl == kClsAcc)
+              bit = true;
+            else if (cl == kClsCD)
               bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-            }
+            else if (cl == kClsCD2)
+              bit = cd2_bit(t, pick, sel2, b, 0, t.pair_by_id[(size_t)tbl0 * t.V + id]);
+          } else {
+            bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
           }
         }
       }
-      const uint32_t word = __ballot_sync(0xffffffffu, bit);
-      if (lane == 0 && wi < t.W) {
-        mask[(size_t)b * t.W + wi] = word;
-        if (word) s_any[k] = 1;
-      }
     }
-    __syncthreads();
-    for (int i = threadIdx.x; i < nr; i += blockDim.x)
-      if (s_any[i]) atomicOr(&ctx[r0 + i].nonempty, 1u);
+    const uint32_t word = __ballot_sync(0xffffffffu, bit);
+    if (lane == 0 && wi < t.W) {
+      mask[(size_t)b * t.W + wi] = word;
+      if (word) s_any[k] = 1;
+    }
   }
+  __syncthreads();
+  for (int i = threadIdx.x; i < nr; i += blockDim.x)
+    if (s_any[i]) atomicOr(&ctx[r0 + i].nonempty, 1u);
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
-    s_last = atomicAdd(&ctx[0].done_blocks, 1u) == gridDim.x - 1;
+    s_last = atomicAdd(&ctx[0].done_blocks, 1u) == gridDim.x * gridDim.y - 1;
   }
   __syncthreads();
   if (s_last) {
@@ -1275,7 +1257,8 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
   tw.blob_bytes = 0;
   k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, c->ctx, c->rng, c->c.stack, c->sel, c->A2, c->verd0,
                                                      c->verd1, c->words_ns, B);
-  k_pack<<<(t.V + 255) / 256, 256, kPackRows * 2 * std::max(1, t.nselw) * 4, st>>>(
+  k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
+           st>>>(
       t, c->ctx, c->sel, c->pick, c->sel2, c->verd0, c->verd1, c->words_ns, d_mask, d_status, B);
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
