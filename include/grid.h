@@ -164,11 +164,12 @@ int grid_specialize(const grid_grammar* g, const grid_vocab* v, void* stream, gr
 void grid_spec_free(grid_spec* s);
 
 /* Facts about a spec (synchronous): out[0]=precomputed lexer states (CI
- * tables), out[1]=CI class ids, out[2]=CD spellings of the start state,
- * out[3]=CD entries over all tables, out[4]=bytes of the tables staged in
- * shared memory (0 = not staged), out[5]=walk blocks per row for the start
- * state's CD list, out[6]=1 if CI classes are enabled, out[7]=distinct
- * spellings. */
+ * tables), out[1]=CI class ids, out[2]=spellings of the start state walked
+ * byte by byte at mask time (more stack-dependent events than one record
+ * holds), out[3]=such entries over all tables, out[4]=bytes of the tables
+ * staged in shared memory (0 = not staged), out[5]=verdict classes (distinct
+ * event records of stack-dependent spellings) over all tables, out[6]=1 if CI
+ * classes are enabled, out[7]=distinct spellings. */
 int grid_spec_info(const grid_spec* s, int64_t out[8]);
 
 /* Create B configurations, all at the start configuration (empty output),

@@ -24,17 +24,64 @@ constexpr int kMaxOvl = 48;  // per-token overlay / scratch entries per lane
 // (q, cats) meets A u I" (token ends inside one lexeme), kind 1 = "the
 // candidate set of (q, cats) meets A u I" (one boundary, then ignored bytes).
 constexpr uint16_t kClsFirstCode = 0xFFFB;  // class ids are below this value
-constexpr uint16_t kClsCD2 = 0xFFFB;  // two stack-dependent events: resolved by (key1, key2) lookups
+constexpr uint16_t kClsVC = 0xFFFB;   // context-dependent, decided by its verdict class (event record)
 constexpr uint16_t kClsNA = 0xFFFC;   // spelling does not continue this lexer state
 constexpr uint16_t kClsAcc = 0xFFFD;  // viable for every allowed set
 constexpr uint16_t kClsRej = 0xFFFE;  // viable for no allowed set
-constexpr uint16_t kClsCD = 0xFFFF;   // context-dependent: walked against the live stack
+constexpr uint16_t kClsCD = 0xFFFF;   // context-dependent, too many events: walked byte by byte
+
+// Event record of a context-dependent spelling (GRID Sec. 4.2, verdict-
+// equivalence grouping): rec[0] = number of stack-dependent emissions n,
+// rec[1] = the final test (a live class id, or kClsAcc when the trailing
+// lexeme is live for an ignored terminal), rec[2 .. 2+n) = the candidate
+// classes of the emissions in order.  Spellings with equal records have equal
+// verdicts at every stack; each distinct record is a verdict class.
+constexpr int kRecLen = 16;
+constexpr int kMaxEv = kRecLen - 2;
+
+// A set of at most 128 terminals held in four registers.  Word access goes
+// through selects, never through a runtime-indexed array (which would live
+// in local memory).
+struct Bits4 {
+  uint32_t x, y, z, w;
+  __host__ __device__ __forceinline__ static Bits4 zero() { return Bits4{0u, 0u, 0u, 0u}; }
+  __device__ __forceinline__ static Bits4 load(const uint32_t* p) { return Bits4{p[0], p[1], p[2], p[3]}; }
+  __device__ __forceinline__ uint32_t word(int i) const { return i == 0 ? x : (i == 1 ? y : (i == 2 ? z : w)); }
+  __device__ __forceinline__ bool has(int t) const { return (word(t >> 5) >> (t & 31)) & 1u; }
+  __device__ __forceinline__ void set(int t) {
+    const uint32_t b = 1u << (t & 31);
+    const int i = t >> 5;
+    x |= i == 0 ? b : 0u;
+    y |= i == 1 ? b : 0u;
+    z |= i == 2 ? b : 0u;
+    w |= i == 3 ? b : 0u;
+  }
+  __device__ __forceinline__ bool any() const { return (x | y | z | w) != 0u; }
+  __device__ __forceinline__ Bits4 operator&(const Bits4& o) const { return Bits4{x & o.x, y & o.y, z & o.z, w & o.w}; }
+  __device__ __forceinline__ Bits4 operator|(const Bits4& o) const { return Bits4{x | o.x, y | o.y, z | o.z, w | o.w}; }
+  __device__ __forceinline__ Bits4 andnot(const Bits4& o) const {
+    return Bits4{x & ~o.x, y & ~o.y, z & ~o.z, w & ~o.w};
+  }
+  __device__ __forceinline__ int lowest() const {
+    return x ? __ffs(x) - 1 : (y ? 31 + __ffs(y) : (z ? 63 + __ffs(z) : (w ? 95 + __ffs(w) : -1)));
+  }
+  __device__ __forceinline__ void clear_lowest() {
+    if (x)
+      x &= x - 1u;
+    else if (y)
+      y &= y - 1u;
+    else if (z)
+      z &= z - 1u;
+    else
+      w &= w - 1u;
+  }
+};
 
 struct Tables {
   int n_term, T1, S, NNT, P, Q, C, n_cat, LN;
   int NS, V, eos, W, D;
-  uint32_t ignored[4];
-  uint32_t catmask[4];
+  Bits4 ign;  // ignored terminals (the set I)
+  Bits4 cm;   // category terminals
   int cat_term[32];
   // staged block: these eight arrays live contiguously in `blob`
   const uint8_t* blob;
@@ -78,17 +125,14 @@ struct Tables {
   const int32_t* cd_off;      // n_tbl + 1
   const int32_t* cd_list;     // ascending spelling indices per table
   const uint16_t* cd_key;     // per cd_list entry: class of its first stack-dependent emission
-  const uint32_t* pair_by_id; // n_tbl * V: (key1 << 16 | key2) of kClsCD2 spellings
+  // verdict classes: table k owns records vc_off[k] .. vc_off[k+1] of vc_rec
+  const int32_t* vc_off;
+  const uint16_t* vc_rec;     // kRecLen per verdict class
+  const uint32_t* vc_by_id;   // n_tbl * V: verdict class (within its table) of kClsVC spellings
 };
 
+// Membership test in a 4-word set stored in memory.
 __device__ __forceinline__ bool bit4(const uint32_t* m, int t) { return (m[t >> 5] >> (t & 31)) & 1u; }
-
-__device__ __forceinline__ int lowest4(const uint32_t m[4]) {
-#pragma unroll
-  for (int w = 0; w < 4; ++w)
-    if (m[w]) return w * 32 + __ffs(m[w]) - 1;
-  return -1;
-}
 
 // Copy the staged block into shared memory and publish one block-wide copy of
 // the table descriptor, rebased onto it, in shared memory (`ts`).  Every thread
@@ -142,29 +186,25 @@ __device__ __forceinline__ int lex_step(const Tables& t, int lx, int b, uint32_t
 
 // Terminal set of DFA state q filtered by the lexicon: non-category terminals
 // pass, category terminal c passes iff bit c of `cats` is set.
-__device__ __forceinline__ void lex_filter(const Tables& t, const uint32_t* src, int q, uint32_t cats,
-                                           uint32_t out[4]) {
-#pragma unroll
-  for (int w = 0; w < 4; ++w) out[w] = src[q * 4 + w] & ~t.catmask[w];
+__device__ __forceinline__ Bits4 lex_filter(const Tables& t, const uint32_t* src, int q, uint32_t cats) {
+  const Bits4 v = Bits4::load(src + q * 4);
+  Bits4 out = v.andnot(t.cm);
   while (cats) {
-    int c = __ffs(cats) - 1;
+    const int c = __ffs(cats) - 1;
     cats &= cats - 1;
-    int term = t.cat_term[c];
-    out[term >> 5] |= src[q * 4 + (term >> 5)] & (1u << (term & 31));
+    const int term = t.cat_term[c];
+    if (v.has(term)) out.set(term);
   }
+  return out;
 }
 
 // live'(q, r): terminals live at q, category terminals only while r is a
 // prefix of one of their words (pc = prefix category bits of r's trie node).
-__device__ __forceinline__ void live_prime(const Tables& t, int q, uint32_t pc, uint32_t out[4]) {
-  lex_filter(t, t.live, q, pc, out);
-}
+__device__ __forceinline__ Bits4 live_prime(const Tables& t, int q, uint32_t pc) { return lex_filter(t, t.live, q, pc); }
 
 // Emission candidates of r: terminals accepting at q, category terminals only
 // if r is one of their words (wc = word category bits of r's trie node).
-__device__ __forceinline__ void cands(const Tables& t, int q, uint32_t wc, uint32_t out[4]) {
-  lex_filter(t, t.acc, q, wc, out);
-}
+__device__ __forceinline__ Bits4 cands(const Tables& t, int q, uint32_t wc) { return lex_filter(t, t.acc, q, wc); }
 
 __device__ __forceinline__ int max_chain_of(const Tables& t) { return 2 * t.D + 256; }
 
@@ -265,49 +305,47 @@ __device__ __forceinline__ bool commit(Walker& w, int keep_o, int m_o, int ns, i
 // candidate in priority order that is ignored or reaches SHIFT wins and is
 // shifted.  `A` (may be NULL) = allowed set of the walker's starting stack,
 // valid while nothing has been shifted.  Returns 1 ok, 0 reject, -1 bound.
-__device__ __forceinline__ int emit(const Tables& t, Walker& w, int max_chain) {
-  uint32_t K[4];
-  cands(t, w.q, w.wc, K);
-  for (int wd = 0; wd < 4; ++wd) {
-    uint32_t bits = K[wd];
-    while (bits) {
-      int tau = wd * 32 + __ffs(bits) - 1;
-      bits &= bits - 1;
-      if (bit4(t.ignored, tau)) return 1;
-      if (w.Acur && !bit4(w.Acur, tau)) continue;
-      int keep_o, m_o, ns;
-      int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
-      if (a < 0) return -1;
-      if (a > 0 && a != kAccept) {
-        if (!commit(w, keep_o, m_o, ns, a - 1)) return -1;
-        w.shifted = true;
-        w.Acur = (w.nshift == 0 && w.A2) ? w.A2 + tau * 4 : nullptr;
-        ++w.nshift;
-        return 1;
-      }
+__device__ __forceinline__ int emit_set(const Tables& t, Walker& w, Bits4 K, int max_chain) {
+  while (K.any()) {
+    const int tau = K.lowest();
+    K.clear_lowest();
+    if (t.ign.has(tau)) return 1;
+    if (w.Acur && !bit4(w.Acur, tau)) continue;
+    int keep_o, m_o, ns;
+    int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+    if (a < 0) return -1;
+    if (a > 0 && a != kAccept) {
+      if (!commit(w, keep_o, m_o, ns, a - 1)) return -1;
+      w.shifted = true;
+      w.Acur = (w.nshift == 0 && w.A2) ? w.A2 + tau * 4 : nullptr;
+      ++w.nshift;
+      return 1;
     }
   }
   return 0;
 }
 
-// Def. 2 trailing liveness.  1 / 0 / -1.
-__device__ __forceinline__ int trailing_live(const Tables& t, Walker& w, int max_chain) {
-  uint32_t L[4];
-  live_prime(t, w.q, w.pc, L);
-  if ((L[0] & t.ignored[0]) | (L[1] & t.ignored[1]) | (L[2] & t.ignored[2]) | (L[3] & t.ignored[3])) return 1;
-  if (const uint32_t* A = w.Acur) return ((L[0] & A[0]) | (L[1] & A[1]) | (L[2] & A[2]) | (L[3] & A[3])) ? 1 : 0;
-  for (int wd = 0; wd < 4; ++wd) {
-    uint32_t bits = L[wd];
-    while (bits) {
-      int tau = wd * 32 + __ffs(bits) - 1;
-      bits &= bits - 1;
-      int keep_o, m_o, ns;
-      int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
-      if (a < 0) return -1;
-      if (a > 0 && a != kAccept) return 1;
-    }
+__device__ __forceinline__ int emit(const Tables& t, Walker& w, int max_chain) {
+  return emit_set(t, w, cands(t, w.q, w.wc), max_chain);
+}
+
+// Def. 2 trailing liveness for live set L.  1 / 0 / -1.
+__device__ __forceinline__ int trailing_set(const Tables& t, Walker& w, Bits4 L, int max_chain) {
+  if ((L & t.ign).any()) return 1;
+  if (const uint32_t* A = w.Acur) return (L & Bits4::load(A)).any() ? 1 : 0;
+  while (L.any()) {
+    const int tau = L.lowest();
+    L.clear_lowest();
+    int keep_o, m_o, ns;
+    int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+    if (a < 0) return -1;
+    if (a > 0 && a != kAccept) return 1;
   }
   return 0;
+}
+
+__device__ __forceinline__ int trailing_live(const Tables& t, Walker& w, int max_chain) {
+  return trailing_set(t, w, live_prime(t, w.q, w.pc), max_chain);
 }
 
 // A spelling's bytes: the first 16 come from one 16-byte load into registers,
@@ -365,14 +403,8 @@ __device__ __forceinline__ int walk_bytes(const Tables& t, Walker& w, const Spel
     }
     w.q = nq;
     w.lx = lex_step(t, w.lx, b, w.pc, w.wc);
-    uint32_t L[4];
-    live_prime(t, w.q, w.pc, L);
-    bool any;
-    if (const uint32_t* A = w.Acur)
-      any = (L[0] & (A[0] | t.ignored[0])) | (L[1] & (A[1] | t.ignored[1])) | (L[2] & (A[2] | t.ignored[2])) |
-            (L[3] & (A[3] | t.ignored[3]));
-    else
-      any = L[0] | L[1] | L[2] | L[3];
+    const Bits4 L = live_prime(t, w.q, w.pc);
+    const bool any = w.Acur ? (L & (Bits4::load(w.Acur) | t.ign)).any() : L.any();
     if (!any) {
       rej = i;
       return 0;
@@ -400,54 +432,46 @@ __device__ __forceinline__ int class_id(const Tables& t, int kind, int q, uint32
 }
 
 // Terminal set of a class id (for the per-row class selection).
-__device__ __forceinline__ void class_set(const Tables& t, int cls, uint32_t out[4]) {
+__device__ __forceinline__ Bits4 class_set(const Tables& t, int cls) {
   const int hi = cls >> t.n_cat;
   const uint32_t cats = (uint32_t)cls & ((1u << t.n_cat) - 1u);
   const int kind = hi / t.Q, q = hi - kind * t.Q;
-  lex_filter(t, kind ? t.acc : t.live, q, cats, out);
+  return lex_filter(t, kind ? t.acc : t.live, q, cats);
 }
 
 // Sec. 4.2 CI/CD classification of one spelling from lexer state (q, lx),
-// with the stack abstracted to its allowed set A.  Emissions whose first
-// candidate is ignored leave the stack alone; an emission whose first candidate
-// is a parser terminal, or the final liveness test, is a stack-dependent event.
-//   one event  -> CI class (verdict = class set meets A u I)
-//   two events -> kClsCD2 with pair = key1 << 16 | key2: the first event picks
-//                 tau1 = lowest(set(key1) & A) and the second is decided by the
-//                 allowed set after shifting tau1 (verdict-equivalent spellings
-//                 share the pair; GRID Sec. 4.2 "verdict-equivalence grouping")
-//   more       -> kClsCD, walked against the live stack.
-// For kClsCD, `first_key` is the class of the first event (0xFFFF if that
-// event always succeeds): the walk is skipped when that class is not selected.
+// with the stack abstracted away.  Emissions whose first candidate is ignored
+// leave the stack alone and are dropped; every other emission, and the final
+// liveness test, is a stack-dependent event.
+//   no event but the final test      -> CI live class / kClsAcc / kClsRej
+//   one emission, then ignored bytes -> CI candidate class (or kClsAcc)
+//   otherwise                        -> kClsVC with its event record `rec`
+//                                       (kClsCD when it has more than kMaxEv
+//                                       emissions; then `first_key` is the
+//                                       class of the first one, 0xFFFF if that
+//                                       emission always succeeds)
 __device__ __forceinline__ uint16_t classify(const Tables& t, int q, int lx, const uint8_t* bytes, int len,
-                                             uint16_t& first_key, uint32_t& pair) {
+                                             uint16_t& first_key, uint16_t* rec) {
   first_key = 0xFFFF;
-  pair = 0u;
   uint32_t pc = lx == 0 ? t.root_pc : 0u, wc = lx == 0 ? t.root_wc : 0u;
-  int key1 = -1, key2 = -1;
-  bool ign1 = false, ign2 = false;
+  int n = 0;
+  bool first_ign = false, overflow = false;
   for (int i = 0; i < len; ++i) {
     const int b = bytes[i];
     const int c = t.byte_class[b];
     int nq = t.next[q * t.C + c];
     if (nq == kDead) {
       if (q == kStart) return kClsRej;
-      uint32_t K[4];
-      cands(t, q, wc, K);
-      const int first = lowest4(K);
+      const Bits4 K = cands(t, q, wc);
+      const int first = K.lowest();
       if (first < 0) return kClsRej;
-      if (!bit4(t.ignored, first)) {
-        const bool kign = (K[0] & t.ignored[0]) | (K[1] & t.ignored[1]) | (K[2] & t.ignored[2]) | (K[3] & t.ignored[3]);
-        if (key1 < 0) {
-          key1 = class_id(t, 1, q, wc);
-          ign1 = kign;
-        } else if (key2 < 0 && !ign1) {
-          key2 = class_id(t, 1, q, wc);
-          ign2 = kign;
-        } else {
-          first_key = ign1 ? 0xFFFF : (uint16_t)key1;
-          return kClsCD;
-        }
+      if (!t.ign.has(first)) {
+        if (n == 0) first_ign = (K & t.ign).any();
+        if (n < kMaxEv)
+          rec[2 + n] = (uint16_t)class_id(t, 1, q, wc);
+        else
+          overflow = true;
+        ++n;
       }
       q = kStart;
       lx = 0;
@@ -459,33 +483,31 @@ __device__ __forceinline__ uint16_t classify(const Tables& t, int q, int lx, con
     q = nq;
     lx = lex_step(t, lx, b, pc, wc);
   }
-  uint32_t L[4];
-  live_prime(t, q, pc, L);
-  const bool lign = (L[0] & t.ignored[0]) | (L[1] & t.ignored[1]) | (L[2] & t.ignored[2]) | (L[3] & t.ignored[3]);
-  const bool lany = L[0] | L[1] | L[2] | L[3];
-  if (key1 < 0) {
-    if (lign) return kClsAcc;
-    if (!lany) return kClsRej;
-    return (uint16_t)class_id(t, 0, q, pc);
+  const Bits4 L = live_prime(t, q, pc);
+  const bool lign = (L & t.ign).any();
+  if (!L.any()) return kClsRej;
+  if (n == 0) return lign ? kClsAcc : (uint16_t)class_id(t, 0, q, pc);
+  if (n == 1 && lign) return first_ign ? kClsAcc : rec[2];
+  if (overflow) {
+    first_key = first_ign ? 0xFFFF : rec[2];
+    return kClsCD;
   }
-  if (key2 < 0) {
-    if (lign) return ign1 ? kClsAcc : (uint16_t)key1;
-    if (!lany) return kClsRej;
-    if (ign1) {
-      first_key = 0xFFFF;
-      return kClsCD;
-    }
-    pair = ((uint32_t)key1 << 16) | (uint32_t)class_id(t, 0, q, pc);
-    return kClsCD2;
+  rec[0] = (uint16_t)n;
+  rec[1] = lign ? kClsAcc : (uint16_t)class_id(t, 0, q, pc);
+  return kClsVC;
+}
+
+// Verdict of an event record at the walker's stack: each event is an emission
+// with the recorded candidate set, then the final liveness test.  1 / 0 / -1.
+__device__ __forceinline__ int eval_record(const Tables& t, Walker& w, const uint16_t* rec, int max_chain) {
+  const int n = rec[0];
+  for (int i = 0; i < n; ++i) {
+    const int e = emit_set(t, w, class_set(t, rec[2 + i]), max_chain);
+    if (e <= 0) return e;
   }
-  if (lign) {
-    if (ign2) return (uint16_t)key1;
-    pair = ((uint32_t)key1 << 16) | (uint32_t)key2;
-    return kClsCD2;
-  }
-  if (!lany) return kClsRej;
-  first_key = (uint16_t)key1;
-  return kClsCD;
+  const uint16_t f = rec[1];
+  if (f == kClsAcc) return 1;
+  return trailing_set(t, w, class_set(t, f), max_chain);
 }
 
 }  // namespace grid

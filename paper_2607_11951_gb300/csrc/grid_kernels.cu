@@ -15,7 +15,9 @@
 //            first-byte ranges that continue the pending lexeme
 //   k_succ   per row, context and allowed terminal tau: the allowed set after
 //            shifting tau, so walks simulate nothing before their second shift
-//   k_walk   CD spellings only: lanes walk token bytes through the DFA and the
+//   k_filter per row and context: the CD spellings whose first stack-dependent
+//            emission can succeed (the others are rejected without a walk)
+//   k_walk   surviving CD spellings only: lanes walk token bytes through the DFA and the
 //            identifier trie, emissions pick the highest-priority parser-viable
 //            candidate on a copy-on-write overlay; a rejected prefix skips its
 //            whole trie subtree (Sec. 4.1)
@@ -30,6 +32,7 @@
 #include <algorithm>
 #include <cstring>
 #include <string>
+#include <unordered_map>
 #include <vector>
 
 #include "grid_device.cuh"
@@ -65,8 +68,9 @@ struct RowCtx {
   int32_t emit_ok, eos_ok, status, complete;
   uint32_t nonempty, done_blocks;
   int32_t keep1, m1;
-  int32_t work0, total0;  // chunk counter / chunks of the row's walk queue
-  int32_t total1;         // leading chunks of the queue that belong to sigma' 
+  int32_t work0;          // next item of the row's walk queue
+  int32_t nrange;         // items over the continuing first-byte ranges (rows without a CI table)
+  int32_t nsurv[2];       // CD spellings that survived k_filter, per context (0: sigma, 1: sigma')
   int32_t nrng;
   uint32_t kill[8];  // bit b: first byte b ends the pending lexeme
   uint16_t ovl1[kMaxOvl];
@@ -100,33 +104,68 @@ __global__ void k_reset(DevConfigs c, int B, int D) {
 
 // ---------------- specialization ----------------
 __global__ void k_classify(Tables t, uint16_t* __restrict__ cls_sp, uint16_t* __restrict__ key_sp,
-                           uint32_t* __restrict__ pair_sp, int32_t* __restrict__ cd_count) {
+                           int32_t* __restrict__ counts) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
   const int tbl = blockIdx.y;
   const int q0 = t.tbl_q[tbl];
   const int lx0 = q0 == kStart ? 0 : -1;
-  int cd = 0;
+  int ncd = 0, nvc = 0;
+  uint16_t rec[kRecLen];
   for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < t.NS; s += gridDim.x * blockDim.x) {
     const int off = t.spell_off[s];
     const int len = t.spell_off[s + 1] - off;
     const uint8_t* by = t.spell_bytes + off;
     uint16_t code, key = 0xFFFF;
-    uint32_t pair = 0u;
     if (!t.ci_on)
       code = kClsCD;
     else if (q0 != kStart && ts.next[q0 * ts.C + ts.byte_class[by[0]]] == kDead)
       code = kClsNA;
     else
-      code = classify(ts, q0, lx0, by, len, key, pair);
+      code = classify(ts, q0, lx0, by, len, key, rec);
     cls_sp[(size_t)tbl * t.NS + s] = code;
     key_sp[(size_t)tbl * t.NS + s] = key;
-    pair_sp[(size_t)tbl * t.NS + s] = pair;
-    cd += code == kClsCD;
+    ncd += code == kClsCD;
+    nvc += code == kClsVC;
   }
-  cd = __reduce_add_sync(0xffffffffu, cd);
-  if ((threadIdx.x & 31) == 0 && cd) atomicAdd(&cd_count[tbl], cd);
+  ncd = __reduce_add_sync(0xffffffffu, ncd);
+  nvc = __reduce_add_sync(0xffffffffu, nvc);
+  if ((threadIdx.x & 31) == 0) {
+    if (ncd) atomicAdd(&counts[2 * tbl], ncd);
+    if (nvc) atomicAdd(&counts[2 * tbl + 1], nvc);
+  }
+}
+
+// Event records of the kClsVC spellings, appended per table in any order:
+// slot -> (table, spelling, record).
+__global__ void k_events(Tables t, const uint16_t* __restrict__ cls_sp, const int32_t* __restrict__ vc_base,
+                         int32_t* __restrict__ fill, int32_t* __restrict__ slot_tbl, int32_t* __restrict__ slot_sp,
+                         uint16_t* __restrict__ slot_rec) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ Tables ts;
+  stage_tables(t, ts, smem);
+  const int tbl = blockIdx.y;
+  const int q0 = t.tbl_q[tbl];
+  const int lx0 = q0 == kStart ? 0 : -1;
+  uint16_t rec[kRecLen];
+  for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < t.NS; s += gridDim.x * blockDim.x) {
+    if (cls_sp[(size_t)tbl * t.NS + s] != kClsVC) continue;
+    const int off = t.spell_off[s];
+    uint16_t key;
+    for (int k = 0; k < kRecLen; ++k) rec[k] = 0;
+    classify(ts, q0, lx0, t.spell_bytes + off, t.spell_off[s + 1] - off, key, rec);
+    const int slot = vc_base[tbl] + atomicAdd(&fill[tbl], 1);
+    slot_tbl[slot] = tbl;
+    slot_sp[slot] = s;
+    for (int k = 0; k < kRecLen; ++k) slot_rec[(size_t)slot * kRecLen + k] = rec[k];
+  }
+}
+
+__global__ void k_scatter_vc(const int32_t* __restrict__ slot_tbl, const int32_t* __restrict__ slot_sp,
+                             const int32_t* __restrict__ slot_vc, int nslot, int NS, uint32_t* __restrict__ vc_sp) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < nslot) vc_sp[(size_t)slot_tbl[i] * NS + slot_sp[i]] = (uint32_t)slot_vc[i];
 }
 
 // One block per table: ordered stream compaction of the CD spellings.
@@ -162,40 +201,28 @@ __global__ void k_compact(const uint16_t* __restrict__ cls_sp, const uint16_t* _
   }
 }
 
-__global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const uint32_t* __restrict__ pair_sp,
-                          uint16_t* __restrict__ cls_by_id, uint32_t* __restrict__ pair_by_id,
+__global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const uint32_t* __restrict__ vc_sp,
+                          uint16_t* __restrict__ cls_by_id, uint32_t* __restrict__ vc_by_id,
                           uint8_t* __restrict__ fb_by_id) {
   const int id = blockIdx.x * blockDim.x + threadIdx.x;
   if (id >= t.V) return;
   const int s = t.spell_of_id[id];
   fb_by_id[id] = s >= 0 ? t.spell_bytes[t.spell_off[s]] : 0;
   for (int k = 0; k < t.n_tbl; ++k) {
-    cls_by_id[(size_t)k * t.V + id] = s >= 0 ? cls_sp[(size_t)k * t.NS + s] : kClsNA;
-    pair_by_id[(size_t)k * t.V + id] = s >= 0 ? pair_sp[(size_t)k * t.NS + s] : 0u;
+    const uint16_t c = s >= 0 ? cls_sp[(size_t)k * t.NS + s] : kClsNA;
+    cls_by_id[(size_t)k * t.V + id] = c;
+    vc_by_id[(size_t)k * t.V + id] = c == kClsVC ? vc_sp[(size_t)k * t.NS + s] : 0xFFFFFFFFu;
   }
 }
 
 // ---------------- mask step ----------------
-// Class selection for allowed set A: bit c = set(c) meets A u I.  With `pick`,
-// also the first terminal of set(c) & A (0xFF if none), i.e. the terminal a
-// first stack-dependent emission of class c shifts.
-__device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* out, uint8_t* pick, int lane) {
-  uint32_t AI[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) AI[k] = A[k] | t.ignored[k];
+// Class selection for allowed set A: bit c = set(c) meets A u I.
+__device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, int lane) {
+  const Bits4 AI = A | t.ign;
   for (int w0 = 0; w0 < t.nselw; ++w0) {
     const int cls = w0 * 32 + lane;
     bool v = false;
-    if (cls < t.ncls) {
-      uint32_t S[4];
-      class_set(t, cls, S);
-      v = (S[0] & AI[0]) | (S[1] & AI[1]) | (S[2] & AI[2]) | (S[3] & AI[3]);
-      if (pick) {
-        const uint32_t SA[4] = {S[0] & A[0], S[1] & A[1], S[2] & A[2], S[3] & A[3]};
-        const int f = lowest4(SA);
-        pick[cls] = f < 0 ? 0xFF : (uint8_t)f;
-      }
-    }
+    if (cls < t.ncls) v = (class_set(t, cls) & AI).any();
     const uint32_t word = __ballot_sync(0xffffffffu, v);
     if (lane == 0) out[w0] = word;
   }
@@ -203,20 +230,23 @@ __device__ void select_classes(const Tables& t, const uint32_t A[4], uint32_t* o
 
 // A(sigma) for the virtual stack base[0:keep] ++ ovl[0:m]: lane l simulates
 // terminals l, l+32, ...; `scr` is the lane's scratch (kMaxOvl entries).
-__device__ void allowed_set(const Tables& t, const uint16_t* base, int keep, const uint16_t* ovl, int m,
-                            uint32_t A[4], int& status, int lane, LArr scr) {
+__device__ Bits4 allowed_set(const Tables& t, const uint16_t* base, int keep, const uint16_t* ovl, int m,
+                             int& status, int lane, LArr scr) {
   const int mc = max_chain_of(t);
+  uint32_t wds[4];
+#pragma unroll
   for (int wd = 0; wd < 4; ++wd) {
     const int tau = wd * 32 + lane;
     bool ok = false;
-    if (tau < t.n_term && !bit4(t.ignored, tau)) {
+    if (tau < t.n_term && !t.ign.has(tau)) {
       int keep_o, m_o, ns;
       int a = simulate(t, base, keep, ovl, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
       ok = a > 0 && a != kAccept;
       if (a < 0) status = GRID_ST_BOUND;
     }
-    A[wd] = __ballot_sync(0xffffffffu, ok);
+    wds[wd] = __ballot_sync(0xffffffffu, ok);
   }
+  return Bits4{wds[0], wds[1], wds[2], wds[3]};
 }
 
 __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
@@ -226,6 +256,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   __shared__ uint16_t s_ovl[kPrepWarps][kMaxOvl];
   __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
   __shared__ uint16_t s_scr[kPrepWarps][kMaxOvl * 32];
+  __shared__ uint32_t s_A0[kPrepWarps][4];
   __shared__ int s_km[kPrepWarps][3];
   const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
   if ((int)blockIdx.x >= row_blocks) {
@@ -263,16 +294,23 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   }
   const int mc = max_chain_of(t);
   int status = complete ? GRID_ST_COMPLETE : GRID_ST_OK;
-  uint32_t A0[4] = {0, 0, 0, 0}, A1[4] = {0, 0, 0, 0};
+  Bits4 A0 = Bits4::zero(), A1 = Bits4::zero();
   const LArr scr{s_scr[warp] + lane, 32};
-  if (!complete) allowed_set(ts, base, depth, nullptr, 0, A0, status, lane, scr);
+  if (!complete) A0 = allowed_set(ts, base, depth, nullptr, 0, status, lane, scr);
+  if (lane == 0) {
+    s_A0[warp][0] = A0.x;
+    s_A0[warp][1] = A0.y;
+    s_A0[warp][2] = A0.z;
+    s_A0[warp][3] = A0.w;
+  }
+  __syncwarp();
   // forced emission of the pending lexeme + EOS gate (lane 0)
   if (lane == 0) {
     int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
     if (!complete) {
       Walker w;
       uint16_t lo[kMaxOvl], ls[kMaxOvl];
-      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, A0, nullptr);
+      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, s_A0[warp], nullptr);
       if (q == kStart) {
         emit_ok = 1;
       } else {
@@ -284,7 +322,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
         for (int i = 0; i < m1; ++i) s_ovl[warp][i] = w.ovl[i];
       }
       Walker w2;
-      walker_init(w2, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, A0, nullptr);
+      walker_init(w2, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, s_A0[warp], nullptr);
       int g = eos_gate(ts, w2, mc);
       if (g < 0) status = GRID_ST_BOUND;
       eos = g > 0;
@@ -297,21 +335,17 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   __syncwarp();
   const int emit_ok = s_km[warp][0], keep1 = s_km[warp][1], m1 = s_km[warp][2];
   if (!complete && emit_ok) {
-    if (keep1 == depth && m1 == 0) {
-      for (int k = 0; k < 4; ++k) A1[k] = A0[k];
-    } else {
-      allowed_set(ts, base, keep1, s_ovl[warp], m1, A1, status, lane, scr);
-    }
+    if (keep1 == depth && m1 == 0)
+      A1 = A0;
+    else
+      A1 = allowed_set(ts, base, keep1, s_ovl[warp], m1, status, lane, scr);
   }
   status = __reduce_max_sync(0xffffffffu, status);
   const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
   // continuing first-byte ranges (rows without a CI table for q)
   int total0 = 0, nrng = 0;
   if (!complete && q != kStart) {
-    if (tbl0 >= 0) {
-      const int len = t.cd_off[tbl0 + 1] - t.cd_off[tbl0];
-      total0 = (len + kSpan - 1) / kSpan;
-    } else {
+    if (tbl0 < 0) {
       RowRanges& R = rng[b];
       for (int b0 = 0; b0 < 256; b0 += 32) {
         const int by = b0 + lane;
@@ -343,13 +377,15 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     const uint32_t word = __ballot_sync(0xffffffffu, kill);
     if (lane == 0) r.kill[b0 >> 5] = word;
   }
-  const int start_len = t.cd_off[1] - t.cd_off[0];
-  const int total1 = (!complete && emit_ok) ? (start_len + kSpan - 1) / kSpan : 0;
   if (lane == 0) {
-    for (int k = 0; k < 4; ++k) {
-      r.A0[k] = A0[k];
-      r.A1[k] = A1[k];
-    }
+    r.A0[0] = A0.x;
+    r.A0[1] = A0.y;
+    r.A0[2] = A0.z;
+    r.A0[3] = A0.w;
+    r.A1[0] = A1.x;
+    r.A1[1] = A1.y;
+    r.A1[2] = A1.z;
+    r.A1[3] = A1.w;
     r.q = q;
     r.lx = lx;
     r.pc0 = pc0;
@@ -364,8 +400,9 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     r.keep1 = keep1;
     r.m1 = m1;
     r.work0 = 0;
-    r.total0 = total1 + total0;
-    r.total1 = total1;
+    r.nrange = total0;
+    r.nsurv[0] = 0;
+    r.nsurv[1] = 0;
     r.nrng = nrng;
   }
   for (int i = lane; i < m1; i += 32) r.ovl1[i] = s_ovl[warp][i];
@@ -375,13 +412,11 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
 // grid = (B, 2, kSuccSlots): row b, context cx (0: sigma, 1: sigma' after the
 // forced emission).  Jobs j = 0..n_term of a (row, context) are spread over
 // its kSuccSlots * kSuccWarps warps.  Job tau < n_term, for tau allowed in the
-// context: the allowed set after tau's reduce chain and shift (A2) and its
-// class selection (sel2), so that walks simulate nothing before their second
-// shift and two-event spellings need no walk.  Job n_term: the context's own
-// class selection and, per emission class, the terminal it would shift (pick).
+// context: the allowed set after tau's reduce chain and shift (A2), so that a
+// walk or verdict-class evaluation simulates nothing before its second shift.
+// Job n_term: the context's CI class selection.
 __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c, const RowCtx* __restrict__ ctx,
-                                                          uint32_t* __restrict__ A2, uint32_t* __restrict__ sel2,
-                                                          uint32_t* __restrict__ sel, uint8_t* __restrict__ pick) {
+                                                          uint32_t* __restrict__ A2, uint32_t* __restrict__ sel) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   __shared__ uint16_t s_win[kWalkWin];
@@ -404,8 +439,7 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   }
   __syncthreads();
   const int keep = cx ? r.keep1 : depth;
-  uint32_t A[4];
-  for (int k = 0; k < 4; ++k) A[k] = cx ? r.A1[k] : r.A0[k];
+  const Bits4 A = Bits4::load(cx ? r.A1 : r.A0);
   const int mc = max_chain_of(t);
   uint32_t* out = A2 + ((size_t)b * 2 + cx) * t.T1 * 4;
   int status = GRID_ST_OK;
@@ -413,11 +447,11 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   for (int j = blockIdx.z * kSuccWarps + warp; j <= t.n_term; j += nw) {
     if (j == t.n_term) {
       if (t.ci_on && (cx == 1 || r.tbl0 >= 0))
-        select_classes(ts, A, sel + ((size_t)b * 2 + cx) * t.nselw, pick + ((size_t)b * 2 + cx) * t.ncls, lane);
+        select_classes(ts, A, sel + ((size_t)b * 2 + cx) * t.nselw, lane);
       continue;
     }
     const int tau = j;
-    if (!bit4(A, tau)) continue;
+    if (!A.has(tau)) continue;
     const LArr scr{s_scr[warp] + lane, 32};
     if (lane == 0) {
       int keep_o, m_o, ns;
@@ -434,29 +468,84 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
     }
     __syncwarp();
     const int m2 = s_m2[warp];
-    uint32_t An[4] = {0, 0, 0, 0};
+    Bits4 An = Bits4::zero();
     if (m2 > 0)
-      allowed_set(ts, base, s_keep2[warp], s_ovl2[warp], m2, An, status, lane, scr);
+      An = allowed_set(ts, base, s_keep2[warp], s_ovl2[warp], m2, status, lane, scr);
     else
       status = GRID_ST_BOUND;
-    if (lane == 0)
-      for (int k = 0; k < 4; ++k) out[tau * 4 + k] = An[k];
-    if (t.ci_on) select_classes(ts, An, sel2 + (((size_t)b * 2 + cx) * t.T1 + tau) * t.nselw, nullptr, lane);
+    if (lane == 0) {
+      out[tau * 4 + 0] = An.x;
+      out[tau * 4 + 1] = An.y;
+      out[tau * 4 + 2] = An.z;
+      out[tau * 4 + 3] = An.w;
+    }
     __syncwarp();
   }
   status = __reduce_max_sync(0xffffffffu, status);
   if (lane == 0 && status != GRID_ST_OK) atomicCAS(const_cast<int32_t*>(&ctx[b].status), GRID_ST_OK, status);
 }
 
-// Persistent walk.  Every row owns one work queue of items: items
-// [0, total1) cover the start state's CD list under sigma' (tokens whose first
-// byte ends the pending lexeme), items [total1, total) the spellings that
-// continue the pending lexeme (the CD list of its lexer state, or its
-// continuing first-byte ranges).  Warps start at different rows, drain a row's
+// grid = (ceil(maxlen/256), B, 2): compact, per row and context, the CD
+// spellings that a walk could admit: the class of the first stack-dependent
+// emission must be selected for the context's allowed set and, for sigma',
+// the first byte must end the pending lexeme.  Survivors go to
+// surv[(b*2 + cx) * cap ...] in any order (list walks do not skip).
+__global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
+                                                int32_t* __restrict__ surv, int cap) {
+  __shared__ int s_warp[8];
+  __shared__ int s_base;
+  const int b = blockIdx.y, cx = blockIdx.z;
+  RowCtx& r = ctx[b];
+  const int q = r.q, tbl0 = r.tbl0;
+  if (r.complete) return;
+  if (cx == 1 && !r.emit_ok) return;
+  if (cx == 0 && (q == kStart || tbl0 < 0)) return;
+  const int tb = cx ? 0 : tbl0;
+  const int len = t.cd_off[tb + 1] - t.cd_off[tb];
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t* csel = sel + ((size_t)b * 2 + cx) * t.nselw;
+  bool pass = false;
+  int s = -1;
+  if (i < len) {
+    s = t.cd_list[t.cd_off[tb] + i];
+    const uint16_t k = t.cd_key[t.cd_off[tb] + i];
+    pass = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
+    if (pass && cx == 1 && q != kStart) {
+      const int b0 = (int)(__ldg(&t.spell16[s]).x & 0xFFu);
+      pass = t.next[q * t.C + t.byte_class[b0]] == kDead;
+    }
+  }
+  const uint32_t bal = __ballot_sync(0xffffffffu, pass);
+  if (lane == 0) s_warp[warp] = __popc(bal);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int tot = 0;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+      const int c = s_warp[k];
+      s_warp[k] = tot;
+      tot += c;
+    }
+    s_base = tot ? atomicAdd(&r.nsurv[cx], tot) : 0;
+  }
+  __syncthreads();
+  if (pass) surv[((size_t)b * 2 + cx) * cap + s_base + s_warp[warp] + __popc(bal & ((1u << lane) - 1u))] = s;
+}
+
+// Persistent walk.  Every row owns one work queue of items, in four segments:
+// verdict classes of the start state's table under sigma' (the context of
+// tokens whose first byte ends the pending lexeme), the start state's
+// byte-walked spellings under sigma', then the verdict classes of the pending
+// lexer state's table under sigma, and the spellings that continue the pending
+// lexeme (its table's byte-walked list, or its continuing first-byte ranges
+// when the state has no table).  Warps start at different rows, drain a row's
 // queue item by item and move on; a warp stops after finding every queue
 // empty once in a row.  A warp keeps the current row's context (allowed sets,
 // sigma' overlay, stack mirror) until it moves to another row.
 //
+// Verdict-class items: 32 distinct event records, one per lane, each
+// evaluated once against the row's stack; a ballot word of verdicts goes to
+// vcbits, read back per token id by k_pack.
 // List items (kSpan CD spellings): a spelling is walked only if the class of
 // its first stack-dependent emission is selected for the context's allowed
 // set (otherwise that emission, and so the spelling, fails) and, for sigma',
@@ -467,10 +556,11 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
 // contiguous in DFS order).  Both kinds share one call of walk_bytes.
 __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* __restrict__ ctx,
                                                              const RowRanges* __restrict__ rng, const uint16_t* stacks,
-                                                             const uint32_t* __restrict__ sel,
+                                                             const int32_t* __restrict__ surv, int cap,
                                                              const uint32_t* __restrict__ A2,
                                                              uint32_t* __restrict__ verd0,
-                                                             uint32_t* __restrict__ verd1, int words_ns, int B) {
+                                                             uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
+                                                             int vcw, int words_ns, int B) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
   __shared__ uint16_t s_win[kWalkWarps][kWalkWin];
@@ -480,27 +570,36 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   stage_tables(t, ts, smem);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWalkWarps + warp;
-  const int start_len = t.cd_off[1] - t.cd_off[0];
-  const int32_t* start_list = t.cd_list + t.cd_off[0];
-  const uint16_t* start_keys = t.cd_key + t.cd_off[0];
   const int mc = max_chain_of(t);
   const LArr lo{s_lane[warp] + lane, 32}, ls{s_lane[warp] + kLaneOvl * 32 + lane, 32};
   int row = gw % B;
   int fails = 0;
   int bound = 0, bound_row = -1;
   int cur = -1;  // row whose context is cached below
-  int total1 = 0, tbl0 = -1, depth = 0, q = 0, lx = 0, keep1 = 0, m1 = 0, nrng = 0;
+  int tbl0 = -1, depth = 0, q = 0, lx = 0, keep1 = 0, m1 = 0, nrng = 0;
   uint32_t pc0 = 0, wc0 = 0;
   const uint16_t* base = stacks;
   while (fails < B) {
     RowCtx& r = ctx[row];
-    int cidx = 0, total = 0;
+    // queue layout: [A: sigma' verdict classes][B: sigma' walked CD spellings]
+    //               [C: sigma verdict classes][D: sigma walked CD spellings, or ranges]
+    int cidx = 0, total = 0, ea = 0, eb = 0, ec = 0;
     if (lane == 0) {
-      total = r.total0;
+      const int t0 = r.tbl0;
+      const int nv1 = r.emit_ok ? t.vc_off[1] - t.vc_off[0] : 0;
+      const int nv0 = t0 >= 0 ? t.vc_off[t0 + 1] - t.vc_off[t0] : 0;
+      ea = (nv1 + 31) >> 5;
+      eb = ea + (r.nsurv[1] + kSpan - 1) / kSpan;
+      ec = eb + ((nv0 + 31) >> 5);
+      total = ec + (t0 >= 0 ? (r.nsurv[0] + kSpan - 1) / kSpan : r.nrange);
+      if (r.complete) total = 0;
       cidx = *((volatile int32_t*)&r.work0) < total ? atomicAdd(&r.work0, 1) : total;
     }
     cidx = __shfl_sync(0xffffffffu, cidx, 0);
     total = __shfl_sync(0xffffffffu, total, 0);
+    ea = __shfl_sync(0xffffffffu, ea, 0);
+    eb = __shfl_sync(0xffffffffu, eb, 0);
+    ec = __shfl_sync(0xffffffffu, ec, 0);
     if (cidx >= total) {
       ++fails;
       row = row + 1 == B ? 0 : row + 1;
@@ -509,7 +608,6 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     fails = 0;
     if (cur != row) {
       cur = row;
-      total1 = r.total1;
       tbl0 = r.tbl0;
       depth = r.depth;
       q = r.q;
@@ -533,7 +631,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
       __syncwarp();
     }
     // ---- the item: context and source
-    const bool c1 = cidx < total1;
+    const bool c1 = cidx < eb;
+    const bool is_vc = cidx < ea || (cidx >= eb && cidx < ec);
     if (c1 && m1 > kLaneOvl) {  // sigma' overlay larger than a walk lane holds: flag the row
       bound = 1;
       bound_row = bound_row < 0 ? row : bound_row;
@@ -544,25 +643,33 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     const int ckeep = c1 ? keep1 : depth, cm = c1 ? m1 : 0;
     const int cq = c1 ? kStart : q, clx = c1 ? 0 : lx;
     const uint32_t cpc = c1 ? t.root_pc : pc0, cwc = c1 ? t.root_wc : wc0;
-    const int kill_q = (c1 && q != kStart) ? q : -1;
+    if (is_vc) {  // 32 verdict classes of the context's table, one per lane
+      const int tb = c1 ? 0 : tbl0;
+      const int item = c1 ? cidx : cidx - eb;
+      const int v = item * 32 + lane;
+      const int nv = t.vc_off[tb + 1] - t.vc_off[tb];
+      int res = 0;
+      if (v < nv) {
+        Walker w;
+        walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
+        res = eval_record(ts, w, ts.vc_rec + (size_t)(t.vc_off[tb] + v) * kRecLen, mc);
+        if (res < 0 && bound_row < 0) bound_row = row;
+        if (res < 0) bound = 1;
+      }
+      const uint32_t word = __ballot_sync(0xffffffffu, res > 0);
+      if (lane == 0) vcbits[((size_t)row * 2 + (c1 ? 1 : 0)) * vcw + item] = word;
+      continue;
+    }
     uint32_t* vb = (c1 ? verd1 : verd0) + (size_t)row * words_ns;
     const int32_t* list = nullptr;
-    const uint16_t* keys = nullptr;
-    const uint32_t* csel = sel + ((size_t)row * 2 + (c1 ? 1 : 0)) * t.nselw;
     int p0, p1;
-    if (c1) {
-      list = start_list;
-      keys = start_keys;
-      p0 = cidx * kSpan;
-      p1 = min(start_len, p0 + kSpan);
-    } else if (tbl0 >= 0) {
-      const int c0 = cidx - total1;
-      list = t.cd_list + t.cd_off[tbl0];
-      keys = t.cd_key + t.cd_off[tbl0];
-      p0 = c0 * kSpan;
-      p1 = min(t.cd_off[tbl0 + 1] - t.cd_off[tbl0], p0 + kSpan);
+    if (c1 || tbl0 >= 0) {  // survivors of k_filter
+      const int n = c1 ? r.nsurv[1] : r.nsurv[0];
+      list = surv + ((size_t)row * 2 + (c1 ? 1 : 0)) * cap;
+      p0 = (c1 ? cidx - ea : cidx - ec) * kSpan;
+      p1 = min(n, p0 + kSpan);
     } else {
-      const int c0 = cidx - total1;
+      const int c0 = cidx - ec;
       const RowRanges& R = rng[row];
       int a = 0, z = nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
       while (z - a > 1) {
@@ -580,41 +687,19 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     for (bool first = true;; first = false) {
       int s = -1;
       bool go = false;
-      Spell sp;
       if (list) {
         if (!first) break;
         const int i = p0 + lane;
-        bool pass = false;
-        if (i < p1) {
-          s = list[i];
-          const uint16_t k = keys[i];
-          pass = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
-          if (pass) {
-            sp = load_spell(ts, s);
-            if (kill_q >= 0) pass = ts.next[kill_q * ts.C + ts.byte_class[sp.at(0)]] == kDead;
-          }
-        }
-        const uint32_t bal = __ballot_sync(0xffffffffu, pass);
-        if (!bal) break;
-        uint32_t rest = bal;  // lane d takes the d-th survivor
-        for (int d = 0; d < lane && rest; ++d) rest &= rest - 1;
-        const int src = rest ? __ffs(rest) - 1 : 0;
-        s = __shfl_sync(0xffffffffu, s, src);
-        sp.head.x = __shfl_sync(0xffffffffu, sp.head.x, src);
-        sp.head.y = __shfl_sync(0xffffffffu, sp.head.y, src);
-        sp.head.z = __shfl_sync(0xffffffffu, sp.head.z, src);
-        sp.head.w = __shfl_sync(0xffffffffu, sp.head.w, src);
-        sp.len = __shfl_sync(0xffffffffu, sp.len, src);
-        go = lane < __popc(bal);
-        if (go) sp.all = ts.spell_bytes + ts.spell_off[s];
+        go = i < p1;
+        if (go) s = list[i];
       } else {
         if (pos >= p1) break;
         s = pos + lane;
         go = s < p1;
-        if (go) sp = load_spell(ts, s);
       }
       int res = 0, rej = -1;
       if (go) {
+        const Spell sp = load_spell(ts, s);
         Walker w;
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
         res = walk_bytes(ts, w, sp, mc, rej);
@@ -644,24 +729,13 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
 }
 
-// Verdict of a kClsCD2 spelling in context cx of row b: its first emission
-// shifts pick[key1] (none: rejected); the second event is decided by the class
-// selection after that shift.
-__device__ __forceinline__ bool cd2_bit(const Tables& t, const uint8_t* __restrict__ pick,
-                                        const uint32_t* __restrict__ sel2, int b, int cx, uint32_t pair) {
-  const uint32_t key1 = pair >> 16, key2 = pair & 0xFFFFu;
-  const int tau = pick[((size_t)b * 2 + cx) * t.ncls + key1];
-  if (tau == 0xFF) return false;
-  return (sel2[(((size_t)b * 2 + cx) * t.T1 + tau) * t.nselw + (key2 >> 5)] >> (key2 & 31)) & 1u;
-}
-
 // grid = (ceil(V/256), ceil(B/kPackRows)), 256 threads: one token id per
 // thread and kPackRows rows per block.  The per-id data (spelling, first byte,
 // start-state class) is loaded once; each warp writes one mask word per row.
 // The last block to finish writes every row's status (EMPTY_MASK for a viable
 // row with no bit set).
 __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
-                                              const uint8_t* __restrict__ pick, const uint32_t* __restrict__ sel2,
+                                              const uint32_t* __restrict__ vcbits, int vcw,
                                               const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
                                               int words_ns, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
                                               int B) {
@@ -685,13 +759,13 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) s_sel[i] = sel[(size_t)r0 * 2 * nw + i];
   int s = -1, b0 = 0;
   uint16_t cl_start = kClsNA;
-  uint32_t pair_start = 0u;
+  uint32_t vc_start = 0u;
   if (id < t.V && id != t.eos) {
     s = t.spell_of_id[id];
     if (s >= 0) {
       b0 = t.first_byte_by_id[id];
       cl_start = t.cls_by_id[id];
-      if (cl_start == kClsCD2) pair_start = t.pair_by_id[id];
+      if (cl_start == kClsVC) vc_start = t.vc_by_id[id];
     }
   }
   __syncthreads();
@@ -712,8 +786,8 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
               bit = true;
             else if (cl == kClsCD)
               bit = (verd1[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-            else if (cl == kClsCD2)
-              bit = cd2_bit(t, pick, sel2, b, 1, pair_start);
+            else if (cl == kClsVC)
+              bit = (vcbits[((size_t)b * 2 + 1) * vcw + (vc_start >> 5)] >> (vc_start & 31)) & 1u;
           }
         } else {
           const int tbl0 = s_tbl[k];
@@ -725,8 +799,10 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
               bit = true;
             else if (cl == kClsCD)
               bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-            else if (cl == kClsCD2)
-              bit = cd2_bit(t, pick, sel2, b, 0, t.pair_by_id[(size_t)tbl0 * t.V + id]);
+            else if (cl == kClsVC) {
+              const uint32_t v = t.vc_by_id[(size_t)tbl0 * t.V + id];
+              bit = (vcbits[(size_t)b * 2 * vcw + (v >> 5)] >> (v & 31)) & 1u;
+            }
           } else {
             bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
           }
@@ -954,6 +1030,9 @@ struct grid_spec {
   int sms = 152;
   int n1 = 0;  // walk chunks of the start state's CD list
   int walk_blocks = 0;  // persistent k_walk grid: resident blocks per SM x SMs
+  int max_cd = 0;       // longest CD list of a table
+  int vcw = 0;          // words of the largest table's verdict-class bitset
+  int n_vc = 0;         // verdict classes over all tables
 };
 
 struct grid_configs {
@@ -965,8 +1044,9 @@ struct grid_configs {
   uint32_t* verd0 = nullptr;
   uint32_t* verd1 = nullptr;
   uint32_t* A2 = nullptr;
-  uint8_t* pick = nullptr;
-  uint32_t* sel2 = nullptr;
+  uint32_t* vcbits = nullptr;
+  int32_t* surv = nullptr;
+  int cap = 0;
   Arena mem;
 };
 
@@ -976,6 +1056,11 @@ struct grid_configs {
 static int set_smem_limits() {
   const int dyn = kMaxStage;
   GRID_CUDA(cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_events, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  // k_pack: the class selections of kPackRows rows, two contexts, at most
+  // kClsFirstCode class ids
+  GRID_CUDA(cudaFuncSetAttribute(k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kPackRows * 2 * ((kClsFirstCode + 31) / 32) * 4));
   GRID_CUDA(cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_succ, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
@@ -1008,10 +1093,8 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   t.eos = hv.eos;
   t.W = (hv.V + 31) / 32;
   t.D = h.max_depth;
-  for (int k = 0; k < 4; ++k) {
-    t.ignored[k] = h.ignored[k];
-    t.catmask[k] = h.catmask[k];
-  }
+  t.ign = Bits4{h.ignored[0], h.ignored[1], h.ignored[2], h.ignored[3]};
+  t.cm = Bits4{h.catmask[0], h.catmask[1], h.catmask[2], h.catmask[3]};
   for (int c = 0; c < h.n_cat; ++c) t.cat_term[c] = h.cat_term[c];
   auto fail = [&](int rc) {
     s->mem.release();
@@ -1116,46 +1199,103 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   cudaGetDevice(&dev);
   s->device = dev;
   cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
-  // CI classification on the device
+  // CI classification on the device (temporaries live in `tmp`)
+  Arena tmp;
+  auto fail_tmp = [&](int code) {
+    tmp.release();
+    return fail(code);
+  };
   uint16_t* cls_sp = nullptr;
   uint16_t* key_sp = nullptr;
-  uint32_t* pair_sp = nullptr;
-  uint32_t* pair_by_id = nullptr;
-  int32_t* cd_count = nullptr;
+  int32_t* counts_d = nullptr;
   uint16_t* cls_by_id = nullptr;
+  uint32_t* vc_by_id = nullptr;
   uint8_t* fb = nullptr;
-  if ((rc = a.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&cls_sp)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&key_sp)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.NS * 4, (void**)&pair_sp)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.V * 4, (void**)&pair_by_id)) ||
-      (rc = a.alloc((size_t)t.n_tbl * 4, (void**)&cd_count)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.V * 2, (void**)&cls_by_id)) || (rc = a.alloc((size_t)t.V, (void**)&fb)))
-    return fail(rc);
+  if ((rc = tmp.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&cls_sp)) ||
+      (rc = tmp.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&key_sp)) ||
+      (rc = tmp.alloc((size_t)t.n_tbl * 8, (void**)&counts_d)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.V * 2, (void**)&cls_by_id)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.V * 4, (void**)&vc_by_id)) || (rc = a.alloc((size_t)t.V, (void**)&fb)))
+    return fail_tmp(rc);
   t.cls_by_id = cls_by_id;
-  t.pair_by_id = pair_by_id;
+  t.vc_by_id = vc_by_id;
   t.first_byte_by_id = fb;
-  GRID_CUDA(cudaMemsetAsync(cd_count, 0, (size_t)t.n_tbl * 4, st));
-  {
-    dim3 grid(std::max(1, std::min((t.NS + 255) / 256, 4 * s->sms)), t.n_tbl);
-    k_classify<<<grid, 256, t.blob_bytes, st>>>(t, cls_sp, key_sp, pair_sp, cd_count);
-  }
-  std::vector<int32_t> counts(t.n_tbl);
-  GRID_CUDA(cudaMemcpyAsync(counts.data(), cd_count, t.n_tbl * 4, cudaMemcpyDeviceToHost, st));
+  GRID_CUDA(cudaMemsetAsync(counts_d, 0, (size_t)t.n_tbl * 8, st));
+  const dim3 cgrid(std::max(1, std::min((t.NS + 255) / 256, 4 * s->sms)), t.n_tbl);
+  k_classify<<<cgrid, 256, t.blob_bytes, st>>>(t, cls_sp, key_sp, counts_d);
+  std::vector<int32_t> counts2(2 * t.n_tbl);
+  GRID_CUDA(cudaMemcpyAsync(counts2.data(), counts_d, t.n_tbl * 8, cudaMemcpyDeviceToHost, st));
   GRID_CUDA(cudaStreamSynchronize(st));
-  std::vector<int32_t> cdoff(t.n_tbl + 1, 0);
-  for (int k = 0; k < t.n_tbl; ++k) cdoff[k + 1] = cdoff[k] + counts[k];
+  std::vector<int32_t> counts(t.n_tbl), cdoff(t.n_tbl + 1, 0), vcbase(t.n_tbl + 1, 0);
+  for (int k = 0; k < t.n_tbl; ++k) {
+    counts[k] = counts2[2 * k];
+    cdoff[k + 1] = cdoff[k] + counts2[2 * k];
+    vcbase[k + 1] = vcbase[k] + counts2[2 * k + 1];
+  }
+  // CD spellings walked byte by byte (more than kMaxEv events)
   int32_t* cd_list = nullptr;
   uint16_t* cd_key = nullptr;
   if ((rc = a.upload(cdoff, &t.cd_off)) || (rc = a.alloc((size_t)cdoff.back() * 4, (void**)&cd_list)) ||
       (rc = a.alloc((size_t)cdoff.back() * 2, (void**)&cd_key)))
-    return fail(rc);
+    return fail_tmp(rc);
   t.cd_list = cd_list;
   t.cd_key = cd_key;
   k_compact<<<t.n_tbl, 1024, 0, st>>>(cls_sp, key_sp, t.NS, t.cd_off, cd_list, cd_key);
-  k_permute<<<(t.V + 255) / 256, 256, 0, st>>>(t, cls_sp, pair_sp, cls_by_id, pair_by_id, fb);
+  // event records of the verdict-class spellings -> distinct records per table
+  const int nslot = vcbase.back();
+  const int32_t* vcbase_d = nullptr;
+  int32_t *fill = nullptr, *slot_tbl = nullptr, *slot_sp = nullptr;
+  uint16_t* slot_rec = nullptr;
+  uint32_t* vc_sp = nullptr;
+  if ((rc = tmp.upload(vcbase, &vcbase_d)) || (rc = tmp.alloc((size_t)t.n_tbl * 4, (void**)&fill)) ||
+      (rc = tmp.alloc((size_t)nslot * 4, (void**)&slot_tbl)) || (rc = tmp.alloc((size_t)nslot * 4, (void**)&slot_sp)) ||
+      (rc = tmp.alloc((size_t)nslot * kRecLen * 2, (void**)&slot_rec)) ||
+      (rc = tmp.alloc((size_t)t.n_tbl * t.NS * 4, (void**)&vc_sp)))
+    return fail_tmp(rc);
+  GRID_CUDA(cudaMemsetAsync(fill, 0, (size_t)t.n_tbl * 4, st));
+  if (nslot > 0) k_events<<<cgrid, 256, t.blob_bytes, st>>>(t, cls_sp, vcbase_d, fill, slot_tbl, slot_sp, slot_rec);
+  std::vector<int32_t> h_tbl(nslot);
+  std::vector<uint16_t> h_rec((size_t)nslot * kRecLen);
+  if (nslot > 0) {
+    GRID_CUDA(cudaMemcpyAsync(h_tbl.data(), slot_tbl, (size_t)nslot * 4, cudaMemcpyDeviceToHost, st));
+    GRID_CUDA(cudaMemcpyAsync(h_rec.data(), slot_rec, (size_t)nslot * kRecLen * 2, cudaMemcpyDeviceToHost, st));
+  }
+  GRID_CUDA(cudaStreamSynchronize(st));
+  std::vector<int32_t> vcoff(t.n_tbl + 1, 0), h_vc(nslot);
+  std::vector<uint16_t> recs;
+  {
+    std::vector<std::unordered_map<std::string, int32_t>> seen(t.n_tbl);
+    std::vector<std::vector<uint16_t>> per(t.n_tbl);
+    for (int i = 0; i < nslot; ++i) {
+      const int k = h_tbl[i];
+      const uint16_t* r = h_rec.data() + (size_t)i * kRecLen;
+      std::string key(reinterpret_cast<const char*>(r), kRecLen * 2);
+      auto it = seen[k].find(key);
+      if (it == seen[k].end()) {
+        it = seen[k].emplace(key, (int32_t)(per[k].size() / kRecLen)).first;
+        per[k].insert(per[k].end(), r, r + kRecLen);
+      }
+      h_vc[i] = it->second;
+    }
+    for (int k = 0; k < t.n_tbl; ++k) {
+      vcoff[k + 1] = vcoff[k] + (int32_t)(per[k].size() / kRecLen);
+      recs.insert(recs.end(), per[k].begin(), per[k].end());
+      s->vcw = std::max(s->vcw, (int)((per[k].size() / kRecLen + 31) / 32));
+    }
+  }
+  const int32_t* slot_vc_c = nullptr;
+  if ((rc = a.upload(vcoff, &t.vc_off)) || (rc = a.upload(recs, &t.vc_rec)) ||
+      (rc = tmp.upload(h_vc, &slot_vc_c)))
+    return fail_tmp(rc);
+  if (nslot > 0)
+    k_scatter_vc<<<(nslot + 255) / 256, 256, 0, st>>>(slot_tbl, slot_sp, slot_vc_c, nslot, t.NS, vc_sp);
+  k_permute<<<(t.V + 255) / 256, 256, 0, st>>>(t, cls_sp, vc_sp, cls_by_id, vc_by_id, fb);
   GRID_CUDA(cudaGetLastError());
   GRID_CUDA(cudaStreamSynchronize(st));
+  tmp.release();
+  s->n_vc = vcoff.back();
   s->n1 = (counts[0] + kSpan - 1) / kSpan;
+  s->max_cd = *std::max_element(counts.begin(), counts.end());
   int per_sm = 0;
   GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, 0));
   s->walk_blocks = std::max(1, per_sm) * s->sms;
@@ -1173,7 +1313,7 @@ extern "C" int grid_spec_info(const grid_spec* s, int64_t out[8]) {
   out[2] = off[1] - off[0];
   out[3] = off[t.n_tbl];
   out[4] = t.blob_bytes;
-  out[5] = s->n1;
+  out[5] = s->n_vc;
   out[6] = t.ci_on;
   out[7] = t.NS;
   return GRID_OK;
@@ -1192,6 +1332,7 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
   c->B = B;
   c->D = s->t.D;
   c->words_ns = (s->t.NS + 31) / 32 + 1;
+  c->cap = std::max(1, s->max_cd);
   Arena& a = c->mem;
   int rc;
   if ((rc = a.alloc((size_t)B * c->D * sizeof(uint16_t), (void**)&c->c.stack)) ||
@@ -1203,8 +1344,8 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
       (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd0)) ||
       (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd1)) ||
       (rc = a.alloc((size_t)B * 2 * s->t.T1 * 16, (void**)&c->A2)) ||
-      (rc = a.alloc((size_t)B * 2 * std::max(1, s->t.ncls), (void**)&c->pick)) ||
-      (rc = a.alloc((size_t)B * 2 * s->t.T1 * std::max(1, s->t.nselw) * 4, (void**)&c->sel2))) {
+      (rc = a.alloc((size_t)B * 2 * std::max(1, s->vcw) * 4, (void**)&c->vcbits)) ||
+      (rc = a.alloc((size_t)B * 2 * std::max(1, s->max_cd) * 4, (void**)&c->surv))) {
     grid_configs_free(c);
     return rc;
   }
@@ -1251,15 +1392,16 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
   const int zero_blocks = std::min(128, (int)(((size_t)B * c->words_ns / 4 + 1023) / 1024) + 1);
   k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(
       t, c->c, c->ctx, c->rng, c->verd0, c->verd1, B, c->words_ns);
-  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c->c, c->ctx, c->A2, c->sel2, c->sel,
-                                                                        c->pick);
+  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c->c, c->ctx, c->A2, c->sel);
   Tables tw = t;  // the walk reads the small tables through L1; its shared memory holds lane overlays
   tw.blob_bytes = 0;
-  k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, c->ctx, c->rng, c->c.stack, c->sel, c->A2, c->verd0,
-                                                     c->verd1, c->words_ns, B);
+  k_filter<<<dim3((s->max_cd + 255) / 256 + (s->max_cd == 0), B, 2), 256, 0, st>>>(t, c->ctx, c->sel, c->surv, c->cap);
+  k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, c->ctx, c->rng, c->c.stack, c->surv, c->cap, c->A2,
+                                                     c->verd0, c->verd1, c->vcbits, std::max(1, s->vcw),
+                                                     c->words_ns, B);
   k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
            st>>>(
-      t, c->ctx, c->sel, c->pick, c->sel2, c->verd0, c->verd1, c->words_ns, d_mask, d_status, B);
+      t, c->ctx, c->sel, c->vcbits, std::max(1, s->vcw), c->verd0, c->verd1, c->words_ns, d_mask, d_status, B);
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }

@@ -182,7 +182,7 @@ def grid_specialize(g, v, stream=None):
 def grid_spec_info(spec):
     out = (ctypes.c_int64 * 8)()
     _check(lib().grid_spec_info(spec, out))
-    keys = ["ci_tables", "ci_classes", "cd_start", "cd_total", "staged_bytes", "walk_blocks_start",
+    keys = ["ci_tables", "ci_classes", "cd_start", "cd_total", "staged_bytes", "verdict_classes",
             "ci_on", "spellings"]
     return dict(zip(keys, list(out)))
 
