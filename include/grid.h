@@ -203,6 +203,36 @@ int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
 int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
                void* stream);
 
+/* grid_masks without any allocation.  The paper has no counterpart: this is
+ * an interface for callers that cannot allocate device memory when they need
+ * a mask, e.g. a serving engine whose memory pool has reserved the device up
+ * front, or that cannot pay for the device-wide synchronization of freeing
+ * memory in the middle of a decoding step.  Such a caller keeps the B parser
+ * configurations in device memory it owns and passes them as arrays with the
+ * layout grid_configs_export reports for one row:
+ *   d_stack     uint16 LALR(1) states, row b at d_stack[b*stack_stride ...],
+ *               bottom first, d_depth[b] entries used;
+ *               stack_stride must equal the grammar's max_depth
+ *   d_depth, d_dfa_state, d_lex_node, d_flags   int32[B] (flags bit 0 =
+ *               complete)
+ * Each row must hold a configuration this library produced (read back with
+ * grid_configs_export, or copied from such a row); other contents are not
+ * checked.  Outputs and status codes are those of grid_masks.
+ *
+ * The step's scratch is one fixed 8 MiB array in the library's device image,
+ * reserved on every device that loads the library until the process exits;
+ * a (spec, B) whose scratch does not fit is rejected with GRID_E_TOO_LARGE
+ * before anything is enqueued (about 45 KB per row at V = 151,936).  The
+ * first call on a device looks up the array's device address (set-up, once per
+ * device, with that device current); make that first call before any stream
+ * capture.  Every call on a device shares the array: calls whose kernels
+ * overlap on the GPU (other streams, other threads) race and corrupt each
+ * other's masks, so serialize them.  Each call clears what must start at zero
+ * itself.  The spec must live on the current device.  Enqueue only. */
+int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, const int32_t* d_depth,
+                      const int32_t* d_dfa_state, const int32_t* d_lex_node, const int32_t* d_flags, int32_t B,
+                      int32_t stack_stride, uint32_t* d_mask, int32_t* d_status, void* stream);
+
 /* Sec. 2 masked decoding: for b < B, t < V, set d_logits[b*row_stride + t] to
  * -inf (fp32 0xFF800000 / bf16 0xFF80) where mask bit t of row b is 0; accepted
  * values are left bit-identical.  d_logits is device memory of `dtype`

@@ -31,6 +31,7 @@
 
 #include <algorithm>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <unordered_map>
 #include <vector>
@@ -1402,6 +1403,126 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
   k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
            st>>>(
       t, c->ctx, c->sel, c->vcbits, std::max(1, s->vcw), c->verd0, c->verd1, c->words_ns, d_mask, d_status, B);
+  GRID_CUDA(cudaGetLastError());
+  return GRID_OK;
+}
+
+// ---------------------------------------------------------------------------
+// grid_masks_static: the mask step without any allocation.
+//
+// Some callers cannot allocate device memory when they need a mask: a serving
+// engine whose own pool has reserved the device memory up front (a driver
+// allocation would fail, or fragment the pool), or one that cannot afford the
+// device-wide synchronization that freeing memory implies in the middle of a
+// decoding step.  Such a caller keeps the parser configurations in device
+// memory it already owns and passes them in; the scratch of the step (row
+// contexts, class selections, survivor lists, verdict bitmaps) comes from the
+// fixed array below instead of from a grid_configs.  The array is part of the
+// library's device image: the CUDA runtime reserves it on every device where
+// the library's kernels are loaded and keeps it until the process exits.
+constexpr size_t kStaticScratchBytes = size_t(8) << 20;
+constexpr int kStaticMaxDevices = 64;
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+namespace {
+// In host code `g_static_scratch` names a host-side shadow of the array, not
+// device memory; kernels get the device address found at set-up.
+std::mutex g_static_mu;
+uint8_t* g_static_dev[kStaticMaxDevices] = {};
+
+// Offsets of the step's buffers inside the array (each 256-byte aligned),
+// sized exactly as grid_configs_create sizes the same buffers.
+struct StaticCarve {
+  size_t ctx, rng, sel, verd0, verd1, A2, vcbits, surv, total;
+};
+
+StaticCarve carve_static(const grid_spec* s, int B, int words_ns) {
+  StaticCarve c{};
+  size_t at = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = at;
+    at += (std::max<size_t>(bytes, 16) + 255) & ~size_t(255);
+    return o;
+  };
+  c.ctx = take((size_t)B * sizeof(RowCtx));
+  c.rng = take((size_t)B * sizeof(RowRanges));
+  c.sel = take((size_t)B * 2 * std::max(1, s->t.nselw) * 4);
+  c.verd0 = take((size_t)B * words_ns * 4);
+  c.verd1 = take((size_t)B * words_ns * 4);
+  c.A2 = take((size_t)B * 2 * s->t.T1 * 16);
+  c.vcbits = take((size_t)B * 2 * std::max(1, s->vcw) * 4);
+  c.surv = take((size_t)B * 2 * std::max(1, s->max_cd) * 4);
+  c.total = at;
+  return c;
+}
+}  // namespace
+
+extern "C" int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, const int32_t* d_depth,
+                                 const int32_t* d_dfa_state, const int32_t* d_lex_node, const int32_t* d_flags,
+                                 int32_t B, int32_t stack_stride, uint32_t* d_mask, int32_t* d_status,
+                                 void* stream) {
+  if (!s || !d_stack || !d_depth || !d_dfa_state || !d_lex_node || !d_flags || !d_mask || !d_status || B <= 0)
+    return set_error(GRID_E_INVALID_ARG, "grid_masks_static: bad arguments");
+  const Tables& t = s->t;
+  if (stack_stride != t.D)
+    return set_error(GRID_E_INVALID_ARG, "grid_masks_static: stack_stride " + std::to_string(stack_stride) +
+                                             " differs from the grammar's max_depth " + std::to_string(t.D));
+  int dev = 0;
+  GRID_CUDA(cudaGetDevice(&dev));
+  if (dev != s->device)
+    return set_error(GRID_E_INVALID_ARG, "grid_masks_static: the spec lives on device " + std::to_string(s->device) +
+                                             ", the current device is " + std::to_string(dev));
+  if (dev < 0 || dev >= kStaticMaxDevices)
+    return set_error(GRID_E_INVALID_ARG, "grid_masks_static: device ordinal " + std::to_string(dev) +
+                                             " is beyond the " + std::to_string(kStaticMaxDevices) + " supported");
+  const int words_ns = (t.NS + 31) / 32 + 1;
+  const StaticCarve cv = carve_static(s, B, words_ns);
+  if (cv.total > kStaticScratchBytes)
+    return set_error(GRID_E_TOO_LARGE, "grid_masks_static: B=" + std::to_string(B) + " needs " +
+                                           std::to_string(cv.total) + " bytes of scratch with this spec, more than "
+                                           "the " + std::to_string(kStaticScratchBytes) +
+                                           "-byte static area; use grid_masks with a grid_configs instead");
+  uint8_t* area = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    if (!g_static_dev[dev]) {  // set-up, once per device
+      void* p = nullptr;
+      const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+      if (e != cudaSuccess || !p)
+        return set_error(GRID_E_CUDA, std::string("grid_masks_static: cudaGetSymbolAddress: ") +
+                                          cudaGetErrorString(e));
+      g_static_dev[dev] = static_cast<uint8_t*>(p);
+    }
+    area = g_static_dev[dev];
+  }
+  RowCtx* ctx = reinterpret_cast<RowCtx*>(area + cv.ctx);
+  RowRanges* rng = reinterpret_cast<RowRanges*>(area + cv.rng);
+  uint32_t* sel = reinterpret_cast<uint32_t*>(area + cv.sel);
+  uint32_t* verd0 = reinterpret_cast<uint32_t*>(area + cv.verd0);
+  uint32_t* verd1 = reinterpret_cast<uint32_t*>(area + cv.verd1);
+  uint32_t* A2 = reinterpret_cast<uint32_t*>(area + cv.A2);
+  uint32_t* vcbits = reinterpret_cast<uint32_t*>(area + cv.vcbits);
+  int32_t* surv = reinterpret_cast<int32_t*>(area + cv.surv);
+  const int cap = std::max(1, s->max_cd);
+  // the kernels only read the configurations
+  DevConfigs c{const_cast<uint16_t*>(d_stack), const_cast<int32_t*>(d_depth), const_cast<int32_t*>(d_dfa_state),
+               const_cast<int32_t*>(d_lex_node), const_cast<int32_t*>(d_flags)};
+  cudaStream_t st = (cudaStream_t)stream;
+  // What must start at zero is cleared by k_prep itself on every call: both
+  // verdict bitmaps (its clearing blocks) and each row's queue, survivor and
+  // completion counters.  The other buffers are written before they are read
+  // within the call, so the previous call's contents do not matter.
+  const int zero_blocks = std::min(128, (int)(((size_t)B * words_ns / 4 + 1023) / 1024) + 1);
+  k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(t, c, ctx, rng, verd0,
+                                                                                               verd1, B, words_ns);
+  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c, ctx, A2, sel);
+  Tables tw = t;
+  tw.blob_bytes = 0;
+  k_filter<<<dim3((s->max_cd + 255) / 256 + (s->max_cd == 0), B, 2), 256, 0, st>>>(t, ctx, sel, surv, cap);
+  k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, ctx, rng, d_stack, surv, cap, A2, verd0, verd1, vcbits,
+                                                     std::max(1, s->vcw), words_ns, B);
+  k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
+           st>>>(t, ctx, sel, vcbits, std::max(1, s->vcw), verd0, verd1, words_ns, d_mask, d_status, B);
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
