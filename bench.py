@@ -31,6 +31,11 @@ N_BATCHES = 16
 METRIC = "cold full-vocab masks/s (batch-32 mask step at V=151,936)"
 
 
+MASK_KERNELS = ["k_prep", "k_succ", "k_filter", "k_walk", "k_pack"]
+WALK_PROFILE = os.path.join(ROOT, "profiles", "k_walk_sql_select_only.md")
+SMSP_PER_SM = 4  # warp schedulers per SM, each issuing at most one warp instruction per clock
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -38,6 +43,32 @@ def _peaks():
         return float(p["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def _source_sha():
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("grid_kernels.cu", "grid_device.cuh"):
+        with open(os.path.join(ROOT, "paper_2607_11951_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def _walk_counters():
+    """Per-launch counters of the walk kernel from the committed ncu summary of
+    this workload, if they were taken on the current kernel sources."""
+    try:
+        kv = {}
+        with open(WALK_PROFILE) as f:
+            for line in f:
+                if line.startswith("- ") and ":" in line:
+                    k, v = line[2:].split(":", 1)
+                    kv[k.strip()] = v.strip().strip("`")
+        if kv.get("source_sha") != _source_sha():
+            return None
+        return {"inst": float(kv["warp_inst_per_launch"]), "dram": float(kv["dram_bytes_per_launch"])}
+    except Exception:
+        return None
 
 
 class ClockSampler:
@@ -84,6 +115,15 @@ class ClockSampler:
         reasons = sorted({names[k] for r in self.rows for k in range(4) if r[3 + k].lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
                 "reasons": reasons, "samples": len(self.rows)}
+
+
+def _gpu_index(local):
+    """nvidia-smi index of this process's GPU (CUDA_VISIBLE_DEVICES applied)."""
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")
+    vis = [v.strip() for v in vis if v.strip()]
+    if local < len(vis) and vis[local].isdigit():
+        return int(vis[local])
+    return local
 
 
 def _dist():
@@ -234,16 +274,16 @@ def main():
     def step(k, ev=None):
         i = k % N_BATCHES
         if ev:
-            ev[0].record()
+            ev[0].record(stream)
         G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
         if ev:
-            ev[1].record()
+            ev[1].record(stream)
         G.grid_masks(spec.h, scratch.h, mask, status, stream)
         if ev:
-            ev[2].record()
+            ev[2].record(stream)
         G.grid_apply_mask(mask, logits[i], stream)
         if ev:
-            ev[3].record()
+            ev[3].record(stream)
 
     for k in range(args.warmup):
         step(k)
@@ -251,28 +291,55 @@ def main():
     if ws > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
-    clk = ClockSampler(local if ws > 1 else int(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or 0)
-                       if False else 0)
+    # Three passes of K steps each, back to back:
+    #   A  the timed region of `value`: events only at its two ends
+    #   B  per-step events around the three calls (p50/p99, per-call means)
+    #   C  events recorded by the library around each kernel of grid_masks
+    # Events cost the GPU a little time each, so A carries none between steps.
+    ev_b = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    ev_c = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    for ev in ev_b + ev_c:  # create each event by a first record, before the library sees its handle
+        for e in ev:
+            e.record(stream)
+    torch.cuda.synchronize()
+    clk = ClockSampler(_gpu_index(local))
     clk.start()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    t_start.record()
-    for k in range(args.steps):
-        step(args.warmup + k, evs[k])
-    t_end.record()
+    if ws > 1:
+        torch.distributed.barrier()
     torch.cuda.synchronize()
-    clocks = clk.stop()
+    torch.cuda.nvtx.range_push("timed")
+    t_start.record(stream)
+    for k in range(args.steps):
+        step(args.warmup + k)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
     total_ms = t_start.elapsed_time(t_end)
+    for k in range(args.steps):  # pass B
+        step(args.warmup + k, ev_b[k])
+    for k in range(args.steps):  # pass C
+        G.grid_configs_set_events(scratch.h, ev_c[k])
+        step(args.warmup + k)
+    torch.cuda.synchronize()
+    G.grid_configs_set_events(scratch.h, [])
+    clocks = clk.stop()
     if ws > 1:
         tt = torch.tensor([total_ms], device=dev)
         torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
         total_ms = float(tt.item())
         torch.distributed.barrier()
-    per_step = [e[0].elapsed_time(e[3]) * 1e3 for e in evs]
-    adv_us = statistics.mean(e[0].elapsed_time(e[1]) * 1e3 for e in evs)
-    masks_us = statistics.mean(e[1].elapsed_time(e[2]) * 1e3 for e in evs)
-    apply_us = statistics.mean(e[2].elapsed_time(e[3]) * 1e3 for e in evs)
+    per_step = [e[0].elapsed_time(e[3]) * 1e3 for e in ev_b]
+    adv_us = statistics.mean(e[0].elapsed_time(e[1]) * 1e3 for e in ev_b)
+    masks_us = statistics.mean(e[1].elapsed_time(e[2]) * 1e3 for e in ev_b)
+    apply_us = statistics.mean(e[2].elapsed_time(e[3]) * 1e3 for e in ev_b)
+    kern_us = {"k_advance": adv_us, "k_apply": apply_us}
+    for j, name in enumerate(MASK_KERNELS):
+        kern_us[name] = statistics.mean(e[j].elapsed_time(e[j + 1]) * 1e3 for e in ev_c)
     per_step.sort()
     p50 = per_step[len(per_step) // 2]
     p99 = per_step[min(len(per_step) - 1, int(math.ceil(0.99 * len(per_step))) - 1)]
@@ -316,12 +383,35 @@ def main():
         e2e = {"value": ws * B * args.steps / (e_ms / 1e3), "unit": "masks/s",
                "h2d_bytes_per_step": B * 4 + B * V * 4, "d2h_bytes_per_step": B * W * 4 + B * 4}
 
-    # ---- roofline of the mask-apply kernel (HBM-bound, write-mostly) ----
-    peak, peak_kind = _peaks()
+    # ---- rooflines ----
+    # mask apply: HBM-bound, write-mostly; algorithmic bytes = the mask read
+    # once + every logit written once (the reject fill touches every sector)
+    hbm_peak, peak_kind = _peaks()
     apply_bytes = B * W * 4 + B * V * 4
-    roof = {"kernel": "k_apply (grid_apply_mask)", "bound": "hbm", "achieved": apply_bytes / (apply_us * 1e-6) / 1e9,
-            "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "traffic": None}
-    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof_apply = {"kernel": "k_apply (grid_apply_mask)", "bound": "hbm",
+                  "achieved": apply_bytes / (apply_us * 1e-6) / 1e9, "peak": hbm_peak,
+                  "peak_kind": peak_kind + " copy bandwidth", "unit": "GB/s", "traffic": None,
+                  "bytes_per_launch": apply_bytes}
+    roof_apply["frac"] = roof_apply["achieved"] / roof_apply["peak"]
+    # walk: integer work without a memory stream (tables stay in L1/L2), so
+    # its ceiling is the warp-instruction issue rate: SMs x 4 schedulers x
+    # 1 instruction per clock at the SM clock sampled during the timed region
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    mhz = clocks.get("sm_mhz") or 2070.0
+    issue_peak = sms * SMSP_PER_SM * mhz * 1e6 / 1e9
+    wc = _walk_counters()
+    walk_us = kern_us["k_walk"]
+    roof_walk = {"kernel": "k_walk (grid_masks)", "bound": "alu", "unit": "G warp-inst/s",
+                 "peak": issue_peak, "peak_kind": "derived: %d SMs x %d schedulers x %.0f MHz sampled" %
+                 (sms, SMSP_PER_SM, mhz),
+                 "achieved": None, "frac": None, "traffic": None,
+                 "counters": "ncu, " + os.path.relpath(WALK_PROFILE, ROOT) if wc else "stale or missing"}
+    if wc:
+        roof_walk["achieved"] = wc["inst"] / (walk_us * 1e-6) / 1e9
+        roof_walk["frac"] = roof_walk["achieved"] / issue_peak
+        roof_walk["traffic"] = wc["dram"]
+    dominant = max(kern_us, key=kern_us.get)
+    roof = roof_walk if dominant == "k_walk" else roof_apply
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "masks/s", "n_gpus": ws, "steps": args.steps,
@@ -333,9 +423,13 @@ def main():
                            "step": "grid_advance + grid_masks + grid_apply_mask"},
                 "p50_us": p50, "p99_us": p99,
                 "token_checks_per_s": value * V,
-                "kernel_us": {"grid_advance": adv_us, "grid_masks": masks_us, "grid_apply_mask": apply_us},
-                "roofline": roof, "cpu_baseline": cpu_base, "e2e": e2e,
-                "gpu_launches": args.steps * 5, "clocks": clocks}
+                "call_us": {"grid_advance": adv_us, "grid_masks": masks_us, "grid_apply_mask": apply_us},
+                "kernel_us": kern_us, "dominant_kernel": dominant,
+                "roofline": roof, "roofline_apply": roof_apply, "cpu_baseline": cpu_base, "e2e": e2e,
+                "gpu_launches": args.steps * (2 + len(MASK_KERNELS)), "clocks": clocks,
+                "timing": "value: K steps between two events; p50/p99 and call_us: a second pass of K "
+                          "steps with events around each call; kernel_us: a third pass with events "
+                          "around each kernel of grid_masks"}
         print(json.dumps(line), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()

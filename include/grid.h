@@ -203,6 +203,16 @@ int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
 int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
                void* stream);
 
+/* Measurement hook: with n_events == 6, every later grid_masks on `c` records
+ * events[0..5] (cudaEvent_t, created by the caller) on its stream before its
+ * first kernel and after each of its five kernels (allowed sets and EOS gate;
+ * allowed sets after the first shift and class selections; byte-walk
+ * candidate filter; walk and verdict classes; id-order packing), so that
+ * cudaEventElapsedTime between neighbours gives each kernel's duration.
+ * n_events == 0 stops the recording.  The caller keeps the events alive while
+ * they are set. */
+int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events);
+
 /* grid_masks without any allocation.  The paper has no counterpart: this is
  * an interface for callers that cannot allocate device memory when they need
  * a mask, e.g. a serving engine whose memory pool has reserved the device up
@@ -222,10 +232,12 @@ int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int3
  * The step's scratch is one fixed 8 MiB array in the library's device image,
  * reserved on every device that loads the library until the process exits;
  * a (spec, B) whose scratch does not fit is rejected with GRID_E_TOO_LARGE
- * before anything is enqueued (about 45 KB per row at V = 151,936).  The
- * first call on a device looks up the array's device address (set-up, once per
- * device, with that device current); make that first call before any stream
- * capture.  Every call on a device shares the array: calls whose kernels
+ * before anything is enqueued (the scratch grows with B and with the spec:
+ * two V-bit verdict bitmaps and the verdict-class survivor lists per row,
+ * about 175 KB per row for the SQL grammar at V = 151,936, so about 48 rows).
+ * The first call on a device looks up the array's device address (set-up,
+ * once per device, with that device current); make that first call before any
+ * stream capture.  Every call on a device shares the array: calls whose kernels
  * overlap on the GPU (other streams, other threads) race and corrupt each
  * other's masks, so serialize them.  Each call clears what must start at zero
  * itself.  The spec must live on the current device.  Enqueue only. */

@@ -128,6 +128,7 @@ struct Tables {
   // verdict classes: table k owns records vc_off[k] .. vc_off[k+1] of vc_rec
   const int32_t* vc_off;
   const uint16_t* vc_rec;     // kRecLen per verdict class
+  const uint16_t* vc_first;   // class id of each verdict class's first event
   const uint32_t* vc_by_id;   // n_tbl * V: verdict class (within its table) of kClsVC spellings
 };
 
@@ -266,6 +267,7 @@ struct Walker {
   uint32_t pc, wc;  // category bits of trie node lx (0 if lx < 0)
   int nshift;
   bool shifted;
+  int pend;  // a first shift not yet applied to the overlay (-1: none)
   const uint32_t* Acur;
   const uint32_t* A2;
   LArr ovl, scr;  // overlay and simulation scratch, `cap` entries each
@@ -288,6 +290,7 @@ __device__ __forceinline__ void walker_init(Walker& w, LArr ovl_store, LArr scr_
   w.wc = wc;
   w.nshift = 0;
   w.shifted = false;
+  w.pend = -1;
   w.Acur = A;
   w.A2 = A2;
 }
@@ -301,16 +304,36 @@ __device__ __forceinline__ bool commit(Walker& w, int keep_o, int m_o, int ns, i
   return true;
 }
 
+// Apply a deferred first shift to the overlay.  The terminal is in the
+// allowed set of the stack it was deferred at, so it reaches SHIFT.
+__device__ __forceinline__ bool materialize(const Tables& t, Walker& w, int max_chain) {
+  int keep_o, m_o, ns;
+  const int a = simulate(t, w.base, w.keep, w.ovl, w.m, w.pend, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+  w.pend = -1;
+  if (a <= 0 || a == kAccept) return false;
+  return commit(w, keep_o, m_o, ns, a - 1);
+}
+
 // Emission of the pending lexeme (Sec. 2, contextual resolution): the first
 // candidate in priority order that is ignored or reaches SHIFT wins and is
-// shifted.  `A` (may be NULL) = allowed set of the walker's starting stack,
-// valid while nothing has been shifted.  Returns 1 ok, 0 reject, -1 bound.
+// shifted.  While the walker knows the allowed set of its stack (Acur) the
+// pick is a set test; a first shift whose successor allowed set is known (A2)
+// is only recorded, and applied to the overlay when a later step needs the
+// stack itself.  Returns 1 ok, 0 reject, -1 bound.
 __device__ __forceinline__ int emit_set(const Tables& t, Walker& w, Bits4 K, int max_chain) {
   while (K.any()) {
     const int tau = K.lowest();
     K.clear_lowest();
     if (t.ign.has(tau)) return 1;
     if (w.Acur && !bit4(w.Acur, tau)) continue;
+    if (w.Acur && w.nshift == 0 && w.A2) {
+      w.pend = tau;
+      w.shifted = true;
+      w.Acur = w.A2 + tau * 4;
+      w.nshift = 1;
+      return 1;
+    }
+    if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
     int keep_o, m_o, ns;
     int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
     if (a < 0) return -1;
@@ -333,6 +356,7 @@ __device__ __forceinline__ int emit(const Tables& t, Walker& w, int max_chain) {
 __device__ __forceinline__ int trailing_set(const Tables& t, Walker& w, Bits4 L, int max_chain) {
   if ((L & t.ign).any()) return 1;
   if (const uint32_t* A = w.Acur) return (L & Bits4::load(A)).any() ? 1 : 0;
+  if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
   while (L.any()) {
     const int tau = L.lowest();
     L.clear_lowest();
@@ -421,6 +445,7 @@ __device__ __forceinline__ int eos_gate(const Tables& t, Walker& w, int max_chai
     int e = emit(t, w, max_chain);
     if (e <= 0) return e;
   }
+  if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
   int keep_o, m_o, ns;
   int a = simulate(t, w.base, w.keep, w.ovl, w.m, t.n_term, w.scr, w.cap, keep_o, m_o, ns, max_chain);
   if (a < 0) return -1;

@@ -46,10 +46,11 @@ constexpr int kSpan = 32;        // CD list entries per walk item (one warp batc
 constexpr int kPrepWarps = 4;    // rows per k_prep block
 constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_prep/k_advance
 constexpr int kPackRows = 8;     // rows per k_pack block
-constexpr int kRangeSpan = 64;   // continuing first-byte ranges are walked in items of this many spellings
+constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
 constexpr int kSuccWarps = 8;    // warps per k_succ block
 constexpr int kSuccSlots = 4;    // k_succ blocks per (row, context)
+constexpr int kWalkRowsCached = 256;  // rows whose queue bounds k_walk keeps in shared memory
 constexpr int kLaneOvl = 32;     // overlay / scratch entries per walk lane (shared memory)
 constexpr int kMaxStage = 96 * 1024;
 
@@ -72,6 +73,7 @@ struct RowCtx {
   int32_t work0;          // next item of the row's walk queue
   int32_t nrange;         // items over the continuing first-byte ranges (rows without a CI table)
   int32_t nsurv[2];       // CD spellings that survived k_filter, per context (0: sigma, 1: sigma')
+  int32_t nvs[2];         // verdict classes that survived k_filter, per context
   int32_t nrng;
   uint32_t kill[8];  // bit b: first byte b ends the pending lexeme
   uint16_t ovl1[kMaxOvl];
@@ -163,6 +165,15 @@ __global__ void k_events(Tables t, const uint16_t* __restrict__ cls_sp, const in
   }
 }
 
+// Terminal set of every class id (events and final tests of the verdict
+// classes use nothing else of a class).
+__global__ void k_class_sets(Tables t, uint4* __restrict__ out) {
+  const int cls = blockIdx.x * blockDim.x + threadIdx.x;
+  if (cls >= t.ncls) return;
+  const Bits4 v = class_set(t, cls);
+  out[cls] = make_uint4(v.x, v.y, v.z, v.w);
+}
+
 __global__ void k_scatter_vc(const int32_t* __restrict__ slot_tbl, const int32_t* __restrict__ slot_sp,
                              const int32_t* __restrict__ slot_vc, int nslot, int NS, uint32_t* __restrict__ vc_sp) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -252,7 +263,8 @@ __device__ Bits4 allowed_set(const Tables& t, const uint16_t* base, int keep, co
 
 __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
                                                           RowRanges* __restrict__ rng, uint32_t* __restrict__ verd0,
-                                                          uint32_t* __restrict__ verd1, int B, int words_ns) {
+                                                          uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
+                                                          int n_vcbits, int B, int words_ns) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kPrepWarps][kMaxOvl];
   __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
@@ -261,7 +273,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   __shared__ int s_km[kPrepWarps][3];
   const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
   if ((int)blockIdx.x >= row_blocks) {
-    // clearing blocks: zero both verdict bitmaps of every row
+    // clearing blocks: zero both verdict bitmaps and the verdict-class bits of every row
     const size_t n = (size_t)B * words_ns;
     const size_t n4 = n >> 2;
     const size_t stride = (size_t)(gridDim.x - row_blocks) * blockDim.x;
@@ -275,6 +287,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
       verd0[i] = 0u;
       verd1[i] = 0u;
     }
+    for (size_t i = first; i < (size_t)n_vcbits; i += stride) vcbits[i] = 0u;
     return;
   }
   __shared__ Tables ts;
@@ -343,15 +356,26 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   }
   status = __reduce_max_sync(0xffffffffu, status);
   const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
-  // continuing first-byte ranges (rows without a CI table for q)
+  // continuing first-byte ranges (rows without a CI table for q).  A first
+  // byte whose lexeme has no live terminal in A0 u I (category terminals
+  // counted only while the lexeme is a prefix of one of their words) rejects
+  // every spelling it starts: liveness only shrinks along the lexeme, and any
+  // later emission picks among its live terminals.
   int total0 = 0, nrng = 0;
   if (!complete && q != kStart) {
     if (tbl0 < 0) {
       RowRanges& R = rng[b];
+      const Bits4 AI = A0 | ts.ign;
       for (int b0 = 0; b0 < 256; b0 += 32) {
         const int by = b0 + lane;
         const int lo = t.first_of_byte[by], hi = t.first_of_byte[by + 1];
-        const bool cont = hi > lo && ts.next[q * ts.C + ts.byte_class[by]] != kDead;
+        const int q2 = ts.next[q * ts.C + ts.byte_class[by]];
+        bool cont = hi > lo && q2 != kDead;
+        if (cont) {
+          uint32_t pc2 = 0u, wc2 = 0u;
+          if (lx >= 0) lex_step(ts, lx, by, pc2, wc2);
+          cont = (live_prime(ts, q2, pc2) & AI).any();
+        }
         const int chunks = cont ? (hi - lo + kRangeSpan - 1) / kRangeSpan : 0;
         const uint32_t bal = __ballot_sync(0xffffffffu, cont);
         int incl = chunks;
@@ -404,6 +428,8 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     r.nrange = total0;
     r.nsurv[0] = 0;
     r.nsurv[1] = 0;
+    r.nvs[0] = 0;
+    r.nvs[1] = 0;
     r.nrng = nrng;
   }
   for (int i = lane; i < m1; i += 32) r.ovl1[i] = s_ovl[warp][i];
@@ -486,13 +512,19 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   if (lane == 0 && status != GRID_ST_OK) atomicCAS(const_cast<int32_t*>(&ctx[b].status), GRID_ST_OK, status);
 }
 
-// grid = (ceil(maxlen/256), B, 2): compact, per row and context, the CD
-// spellings that a walk could admit: the class of the first stack-dependent
-// emission must be selected for the context's allowed set and, for sigma',
-// the first byte must end the pending lexeme.  Survivors go to
-// surv[(b*2 + cx) * cap ...] in any order (list walks do not skip).
+// grid = (cd_blocks + vc_blocks, B, 2), 256 threads: compact, per row and
+// context, what the walk has to evaluate.
+//  - blocks x < cd_blocks: the byte-walked CD spellings that a walk could
+//    admit: the class of the first stack-dependent emission must be selected
+//    for the context's allowed set and, for sigma', the first byte must end
+//    the pending lexeme; survivors go to surv[(b*2 + cx) * cap ...].
+//  - the other blocks: the verdict classes whose first event's class is
+//    selected (any other record fails at its first emission); survivors go to
+//    vsurv[(b*2 + cx) * vcap ...].
+// Both lists are in any order.
 __global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
-                                                int32_t* __restrict__ surv, int cap) {
+                                                int32_t* __restrict__ surv, int cap, int32_t* __restrict__ vsurv,
+                                                int vcap, int cd_blocks) {
   __shared__ int s_warp[8];
   __shared__ int s_base;
   const int b = blockIdx.y, cx = blockIdx.z;
@@ -502,19 +534,28 @@ __global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ c
   if (cx == 1 && !r.emit_ok) return;
   if (cx == 0 && (q == kStart || tbl0 < 0)) return;
   const int tb = cx ? 0 : tbl0;
-  const int len = t.cd_off[tb + 1] - t.cd_off[tb];
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const bool vc = (int)blockIdx.x >= cd_blocks;
+  const int bx = vc ? (int)blockIdx.x - cd_blocks : (int)blockIdx.x;
+  const int len = vc ? t.vc_off[tb + 1] - t.vc_off[tb] : t.cd_off[tb + 1] - t.cd_off[tb];
+  if (bx * (int)blockDim.x >= len) return;
+  const int i = bx * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint32_t* csel = sel + ((size_t)b * 2 + cx) * t.nselw;
   bool pass = false;
   int s = -1;
   if (i < len) {
-    s = t.cd_list[t.cd_off[tb] + i];
-    const uint16_t k = t.cd_key[t.cd_off[tb] + i];
-    pass = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
-    if (pass && cx == 1 && q != kStart) {
-      const int b0 = (int)(__ldg(&t.spell16[s]).x & 0xFFu);
-      pass = t.next[q * t.C + t.byte_class[b0]] == kDead;
+    if (vc) {
+      s = i;
+      const uint16_t k = t.vc_first[t.vc_off[tb] + i];
+      pass = (csel[k >> 5] >> (k & 31)) & 1u;
+    } else {
+      s = t.cd_list[t.cd_off[tb] + i];
+      const uint16_t k = t.cd_key[t.cd_off[tb] + i];
+      pass = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
+      if (pass && cx == 1 && q != kStart) {
+        const int b0 = (int)(__ldg(&t.spell16[s]).x & 0xFFu);
+        pass = t.next[q * t.C + t.byte_class[b0]] == kDead;
+      }
     }
   }
   const uint32_t bal = __ballot_sync(0xffffffffu, pass);
@@ -527,26 +568,47 @@ __global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ c
       s_warp[k] = tot;
       tot += c;
     }
-    s_base = tot ? atomicAdd(&r.nsurv[cx], tot) : 0;
+    s_base = tot ? atomicAdd(vc ? &r.nvs[cx] : &r.nsurv[cx], tot) : 0;
   }
   __syncthreads();
-  if (pass) surv[((size_t)b * 2 + cx) * cap + s_base + s_warp[warp] + __popc(bal & ((1u << lane) - 1u))] = s;
+  if (pass) {
+    const int at = s_base + s_warp[warp] + __popc(bal & ((1u << lane) - 1u));
+    if (vc)
+      vsurv[((size_t)b * 2 + cx) * vcap + at] = s;
+    else
+      surv[((size_t)b * 2 + cx) * cap + at] = s;
+  }
+}
+
+// Ends of the first three queue segments of a row (x, y, z) and its length
+// (w).  Segments: [sigma walked CD spellings, or ranges][sigma' verdict
+// classes][sigma' walked CD spellings][sigma verdict classes].  The byte
+// walks come first: their items are the longest, and starting them early
+// keeps them off the end of the kernel.
+__device__ __forceinline__ int4 row_queue(const Tables& t, const RowCtx& x) {
+  if (x.complete) return make_int4(0, 0, 0, 0);
+  const int ed = x.tbl0 >= 0 ? (x.nsurv[0] + kSpan - 1) / kSpan : x.nrange;
+  const int ea = ed + ((x.nvs[1] + 31) >> 5);
+  const int eb = ea + (x.nsurv[1] + kSpan - 1) / kSpan;
+  return make_int4(ed, ea, eb, eb + ((x.nvs[0] + 31) >> 5));
 }
 
 // Persistent walk.  Every row owns one work queue of items, in four segments:
-// verdict classes of the start state's table under sigma' (the context of
-// tokens whose first byte ends the pending lexeme), the start state's
-// byte-walked spellings under sigma', then the verdict classes of the pending
-// lexer state's table under sigma, and the spellings that continue the pending
-// lexeme (its table's byte-walked list, or its continuing first-byte ranges
-// when the state has no table).  Warps start at different rows, drain a row's
-// queue item by item and move on; a warp stops after finding every queue
-// empty once in a row.  A warp keeps the current row's context (allowed sets,
-// sigma' overlay, stack mirror) until it moves to another row.
+// the spellings that continue the pending lexeme under sigma (its table's
+// byte-walked list, or its continuing first-byte ranges when the state has no
+// table), the verdict classes of the start state's table under sigma' (the
+// context of tokens whose first byte ends the pending lexeme), the start
+// state's byte-walked spellings under sigma', and the verdict classes of the
+// pending lexer state's table under sigma.  Warps start at different rows and drain a
+// row's queue item by item; to find work a warp examines 32 rows at once (one
+// per lane), from its current row on, and stops when no queue has items left.
+// A warp keeps the current row's context (allowed sets, sigma' overlay, stack
+// mirror) until it moves to another row.
 //
-// Verdict-class items: 32 distinct event records, one per lane, each
-// evaluated once against the row's stack; a ballot word of verdicts goes to
-// vcbits, read back per token id by k_pack.
+// Verdict-class items: 32 of the records that k_filter kept for the row and
+// context, one per lane, each evaluated once against the row's stack; an
+// accepted record sets its bit in vcbits (cleared by k_prep), which k_pack
+// reads back per token id.
 // List items (kSpan CD spellings): a spelling is walked only if the class of
 // its first stack-dependent emission is selected for the context's allowed
 // set (otherwise that emission, and so the spelling, fails) and, for sigma',
@@ -561,52 +623,80 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
                                                              const uint32_t* __restrict__ A2,
                                                              uint32_t* __restrict__ verd0,
                                                              uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
-                                                             int vcw, int words_ns, int B) {
+                                                             int vcw, const int32_t* __restrict__ vsurv, int vcap,
+                                                             int words_ns, int B) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
   __shared__ uint16_t s_win[kWalkWarps][kWalkWin];
   __shared__ uint16_t s_lane[kWalkWarps][2 * kLaneOvl * 32];
   __shared__ uint32_t s_A[kWalkWarps][2][4];  // the cached row's A0 and A1
+  __shared__ int4 s_seg[kWalkRowsCached];
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWalkWarps + warp;
   const int mc = max_chain_of(t);
   const LArr lo{s_lane[warp] + lane, 32}, ls{s_lane[warp] + kLaneOvl * 32 + lane, 32};
+  // queue length and segment ends of every row
+  const bool cached = B <= kWalkRowsCached;
+  if (cached) {
+    for (int i = threadIdx.x; i < B; i += blockDim.x) {
+      const int4 e = row_queue(t, ctx[i]);
+      s_seg[i] = e;
+    }
+  }
+  __syncthreads();
   int row = gw % B;
-  int fails = 0;
   int bound = 0, bound_row = -1;
   int cur = -1;  // row whose context is cached below
   int tbl0 = -1, depth = 0, q = 0, lx = 0, keep1 = 0, m1 = 0, nrng = 0;
   uint32_t pc0 = 0, wc0 = 0;
   const uint16_t* base = stacks;
-  while (fails < B) {
+  for (;;) {
+    // next item of the current row; once that queue is drained, of the first
+    // row from there on with items left (32 rows examined at once, one per lane)
+    int cidx = -1;
+    int4 seg = make_int4(0, 0, 0, 0);
+    {
+      int got = 0;
+      const int4 e = cached ? s_seg[row] : row_queue(t, ctx[row]);
+      if (lane == 0 && e.w > 0) got = atomicAdd(&ctx[row].work0, 1);
+      got = __shfl_sync(0xffffffffu, got, 0);
+      if (e.w > 0 && got < e.w) {
+        cidx = got;
+        seg = e;
+      }
+    }
+    for (int off = 0; off < B && cidx < 0; off += 32) {
+      int rr = row + off + lane;
+      rr = rr >= B ? rr - B : rr;
+      int4 e = make_int4(0, 0, 0, 0);
+      bool has = false;
+      if (off + lane < B) {
+        e = cached ? s_seg[rr] : row_queue(t, ctx[rr]);
+        has = e.w > 0 && *((volatile const int32_t*)&ctx[rr].work0) < e.w;
+      }
+      uint32_t bal = __ballot_sync(0xffffffffu, has);
+      while (bal) {  // warp-uniform
+        const int l = __ffs(bal) - 1;
+        bal &= bal - 1;
+        const int rl = __shfl_sync(0xffffffffu, rr, l);
+        const int tl = __shfl_sync(0xffffffffu, e.w, l);
+        int got = 0;
+        if (lane == 0) got = atomicAdd(&ctx[rl].work0, 1);
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (got < tl) {
+          cidx = got;
+          row = rl;
+          seg = make_int4(__shfl_sync(0xffffffffu, e.x, l), __shfl_sync(0xffffffffu, e.y, l),
+                          __shfl_sync(0xffffffffu, e.z, l), tl);
+          break;
+        }
+      }
+    }
+    const int ed = seg.x, ea = seg.y, eb = seg.z;
+    if (cidx < 0) break;
     RowCtx& r = ctx[row];
-    // queue layout: [A: sigma' verdict classes][B: sigma' walked CD spellings]
-    //               [C: sigma verdict classes][D: sigma walked CD spellings, or ranges]
-    int cidx = 0, total = 0, ea = 0, eb = 0, ec = 0;
-    if (lane == 0) {
-      const int t0 = r.tbl0;
-      const int nv1 = r.emit_ok ? t.vc_off[1] - t.vc_off[0] : 0;
-      const int nv0 = t0 >= 0 ? t.vc_off[t0 + 1] - t.vc_off[t0] : 0;
-      ea = (nv1 + 31) >> 5;
-      eb = ea + (r.nsurv[1] + kSpan - 1) / kSpan;
-      ec = eb + ((nv0 + 31) >> 5);
-      total = ec + (t0 >= 0 ? (r.nsurv[0] + kSpan - 1) / kSpan : r.nrange);
-      if (r.complete) total = 0;
-      cidx = *((volatile int32_t*)&r.work0) < total ? atomicAdd(&r.work0, 1) : total;
-    }
-    cidx = __shfl_sync(0xffffffffu, cidx, 0);
-    total = __shfl_sync(0xffffffffu, total, 0);
-    ea = __shfl_sync(0xffffffffu, ea, 0);
-    eb = __shfl_sync(0xffffffffu, eb, 0);
-    ec = __shfl_sync(0xffffffffu, ec, 0);
-    if (cidx >= total) {
-      ++fails;
-      row = row + 1 == B ? 0 : row + 1;
-      continue;
-    }
-    fails = 0;
     if (cur != row) {
       cur = row;
       tbl0 = r.tbl0;
@@ -632,8 +722,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
       __syncwarp();
     }
     // ---- the item: context and source
-    const bool c1 = cidx < eb;
-    const bool is_vc = cidx < ea || (cidx >= eb && cidx < ec);
+    const bool c1 = cidx >= ed && cidx < eb;
+    const bool is_vc = (cidx >= ed && cidx < ea) || cidx >= eb;
     if (c1 && m1 > kLaneOvl) {  // sigma' overlay larger than a walk lane holds: flag the row
       bound = 1;
       bound_row = bound_row < 0 ? row : bound_row;
@@ -644,21 +734,21 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     const int ckeep = c1 ? keep1 : depth, cm = c1 ? m1 : 0;
     const int cq = c1 ? kStart : q, clx = c1 ? 0 : lx;
     const uint32_t cpc = c1 ? t.root_pc : pc0, cwc = c1 ? t.root_wc : wc0;
-    if (is_vc) {  // 32 verdict classes of the context's table, one per lane
+    if (is_vc) {  // 32 surviving verdict classes of the context's table, one per lane
       const int tb = c1 ? 0 : tbl0;
-      const int item = c1 ? cidx : cidx - eb;
-      const int v = item * 32 + lane;
-      const int nv = t.vc_off[tb + 1] - t.vc_off[tb];
-      int res = 0;
-      if (v < nv) {
+      const int cxi = c1 ? 1 : 0;
+      const int item = c1 ? cidx - ed : cidx - eb;
+      const int k = item * 32 + lane;
+      int res = 0, v = 0;
+      if (k < r.nvs[cxi]) {
+        v = vsurv[((size_t)row * 2 + cxi) * vcap + k];
         Walker w;
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
         res = eval_record(ts, w, ts.vc_rec + (size_t)(t.vc_off[tb] + v) * kRecLen, mc);
         if (res < 0 && bound_row < 0) bound_row = row;
         if (res < 0) bound = 1;
       }
-      const uint32_t word = __ballot_sync(0xffffffffu, res > 0);
-      if (lane == 0) vcbits[((size_t)row * 2 + (c1 ? 1 : 0)) * vcw + item] = word;
+      if (res > 0) atomicOr(&vcbits[((size_t)row * 2 + cxi) * vcw + (v >> 5)], 1u << (v & 31));
       continue;
     }
     uint32_t* vb = (c1 ? verd1 : verd0) + (size_t)row * words_ns;
@@ -667,10 +757,10 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     if (c1 || tbl0 >= 0) {  // survivors of k_filter
       const int n = c1 ? r.nsurv[1] : r.nsurv[0];
       list = surv + ((size_t)row * 2 + (c1 ? 1 : 0)) * cap;
-      p0 = (c1 ? cidx - ea : cidx - ec) * kSpan;
+      p0 = (c1 ? cidx - ea : cidx) * kSpan;
       p1 = min(n, p0 + kSpan);
     } else {
-      const int c0 = cidx - ec;
+      const int c0 = cidx;
       const RowRanges& R = rng[row];
       int a = 0, z = nrng;  // range k with cpre[k] <= c0 < cpre[k+1]
       while (z - a > 1) {
@@ -1034,7 +1124,10 @@ struct grid_spec {
   int max_cd = 0;       // longest CD list of a table
   int vcw = 0;          // words of the largest table's verdict-class bitset
   int n_vc = 0;         // verdict classes over all tables
+  int max_vc = 0;       // verdict classes of the largest table
 };
+
+constexpr int kMaskKernels = 5;  // k_prep, k_succ, k_filter, k_walk, k_pack
 
 struct grid_configs {
   int B = 0, D = 0, words_ns = 0;
@@ -1047,7 +1140,9 @@ struct grid_configs {
   uint32_t* A2 = nullptr;
   uint32_t* vcbits = nullptr;
   int32_t* surv = nullptr;
-  int cap = 0;
+  int32_t* vsurv = nullptr;
+  int cap = 0, vcap = 0;
+  cudaEvent_t ev[kMaskKernels + 1] = {};  // optional per-kernel timing events
   Arena mem;
 };
 
@@ -1262,6 +1357,28 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     GRID_CUDA(cudaMemcpyAsync(h_rec.data(), slot_rec, (size_t)nslot * kRecLen * 2, cudaMemcpyDeviceToHost, st));
   }
   GRID_CUDA(cudaStreamSynchronize(st));
+  // class ids with equal terminal sets are interchangeable in a record:
+  // rewrite each to the smallest such id before deduplication
+  std::vector<uint16_t> canon(std::max(1, t.ncls));
+  if (nslot > 0 && t.ncls > 0) {
+    uint4* sets_d = nullptr;
+    if ((rc = tmp.alloc((size_t)t.ncls * 16, (void**)&sets_d))) return fail_tmp(rc);
+    k_class_sets<<<(t.ncls + 255) / 256, 256, 0, st>>>(t, sets_d);
+    std::vector<uint4> sets(t.ncls);
+    GRID_CUDA(cudaMemcpyAsync(sets.data(), sets_d, (size_t)t.ncls * 16, cudaMemcpyDeviceToHost, st));
+    GRID_CUDA(cudaStreamSynchronize(st));
+    std::unordered_map<std::string, uint16_t> first;
+    for (int c = 0; c < t.ncls; ++c) {
+      std::string key(reinterpret_cast<const char*>(&sets[c]), 16);
+      canon[c] = first.emplace(key, (uint16_t)c).first->second;
+    }
+    for (int i = 0; i < nslot; ++i) {
+      uint16_t* r = h_rec.data() + (size_t)i * kRecLen;
+      if (r[1] < t.ncls) r[1] = canon[r[1]];
+      for (int e = 0; e < r[0]; ++e)
+        if (r[2 + e] < t.ncls) r[2 + e] = canon[r[2 + e]];
+    }
+  }
   std::vector<int32_t> vcoff(t.n_tbl + 1, 0), h_vc(nslot);
   std::vector<uint16_t> recs;
   {
@@ -1278,14 +1395,39 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
       }
       h_vc[i] = it->second;
     }
+    // order each table's records by event count, so that the 32 records of a
+    // walk item tend to cost alike
+    for (int k = 0; k < t.n_tbl; ++k) {
+      const int n = (int)(per[k].size() / kRecLen);
+      std::vector<int32_t> ord(n), pos(n);
+      for (int i = 0; i < n; ++i) ord[i] = i;
+      const uint16_t* R = per[k].data();
+      std::stable_sort(ord.begin(), ord.end(), [&](int x, int y) {
+        return R[(size_t)x * kRecLen] < R[(size_t)y * kRecLen];
+      });
+      std::vector<uint16_t> sorted(per[k].size());
+      for (int i = 0; i < n; ++i) {
+        pos[ord[i]] = i;
+        std::copy(R + (size_t)ord[i] * kRecLen, R + (size_t)(ord[i] + 1) * kRecLen, sorted.begin() + (size_t)i * kRecLen);
+      }
+      per[k].swap(sorted);
+      for (auto& kv : seen[k]) kv.second = pos[kv.second];
+    }
+    for (int i = 0; i < nslot; ++i) {
+      const uint16_t* r = h_rec.data() + (size_t)i * kRecLen;
+      h_vc[i] = seen[h_tbl[i]].at(std::string(reinterpret_cast<const char*>(r), kRecLen * 2));
+    }
     for (int k = 0; k < t.n_tbl; ++k) {
       vcoff[k + 1] = vcoff[k] + (int32_t)(per[k].size() / kRecLen);
       recs.insert(recs.end(), per[k].begin(), per[k].end());
       s->vcw = std::max(s->vcw, (int)((per[k].size() / kRecLen + 31) / 32));
     }
   }
+  std::vector<uint16_t> first(recs.size() / kRecLen);
+  for (size_t i = 0; i < first.size(); ++i) first[i] = recs[i * kRecLen + 2];
+  for (int k = 0; k < t.n_tbl; ++k) s->max_vc = std::max(s->max_vc, vcoff[k + 1] - vcoff[k]);
   const int32_t* slot_vc_c = nullptr;
-  if ((rc = a.upload(vcoff, &t.vc_off)) || (rc = a.upload(recs, &t.vc_rec)) ||
+  if ((rc = a.upload(vcoff, &t.vc_off)) || (rc = a.upload(recs, &t.vc_rec)) || (rc = a.upload(first, &t.vc_first)) ||
       (rc = tmp.upload(h_vc, &slot_vc_c)))
     return fail_tmp(rc);
   if (nslot > 0)
@@ -1298,7 +1440,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   s->n1 = (counts[0] + kSpan - 1) / kSpan;
   s->max_cd = *std::max_element(counts.begin(), counts.end());
   int per_sm = 0;
-  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, 0));
+  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, t.blob_bytes));
   s->walk_blocks = std::max(1, per_sm) * s->sms;
   *out = s;
   return GRID_OK;
@@ -1334,6 +1476,7 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
   c->D = s->t.D;
   c->words_ns = (s->t.NS + 31) / 32 + 1;
   c->cap = std::max(1, s->max_cd);
+  c->vcap = std::max(1, s->max_vc);
   Arena& a = c->mem;
   int rc;
   if ((rc = a.alloc((size_t)B * c->D * sizeof(uint16_t), (void**)&c->c.stack)) ||
@@ -1346,7 +1489,8 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
       (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd1)) ||
       (rc = a.alloc((size_t)B * 2 * s->t.T1 * 16, (void**)&c->A2)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->vcw) * 4, (void**)&c->vcbits)) ||
-      (rc = a.alloc((size_t)B * 2 * std::max(1, s->max_cd) * 4, (void**)&c->surv))) {
+      (rc = a.alloc((size_t)B * 2 * std::max(1, s->max_cd) * 4, (void**)&c->surv)) ||
+      (rc = a.alloc((size_t)B * 2 * c->vcap * 4, (void**)&c->vsurv))) {
     grid_configs_free(c);
     return rc;
   }
@@ -1384,26 +1528,65 @@ extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_con
   return GRID_OK;
 }
 
+// Buffers of one mask step (owned by a grid_configs, or carved out of the
+// static area of grid_masks_static).
+struct MaskScratch {
+  RowCtx* ctx;
+  RowRanges* rng;
+  uint32_t *sel, *verd0, *verd1, *A2, *vcbits;
+  int32_t *surv, *vsurv;
+  int cap, vcap, words_ns;
+};
+
+// The five kernels of one mask step on `st`; `ev` (6 events or NULL) is
+// recorded before the first kernel and after each.
+static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, int B, uint32_t* d_mask,
+                        int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev) {
+  const Tables& t = s->t;
+  const int vcw = std::max(1, s->vcw);
+  const int n_vcbits = B * 2 * vcw;
+  const size_t zero_words = (size_t)B * m.words_ns * 2 + n_vcbits;
+  const int zero_blocks = std::min(128, (int)((zero_words / 8 + 1023) / 1024) + 1);
+  if (ev) GRID_CUDA(cudaEventRecord(ev[0], st));
+  k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(
+      t, c, m.ctx, m.rng, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns);
+  if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
+  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c, m.ctx, m.A2, m.sel);
+  if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
+  const int cd_blocks = (s->max_cd + 255) / 256;
+  const int vc_blocks = (s->max_vc + 255) / 256;
+  k_filter<<<dim3(std::max(1, cd_blocks + vc_blocks), B, 2), 256, 0, st>>>(t, m.ctx, m.sel, m.surv, m.cap, m.vsurv,
+                                                                           m.vcap, cd_blocks);
+  if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
+  k_walk<<<s->walk_blocks, kWalkWarps * 32, t.blob_bytes, st>>>(t, m.ctx, m.rng, c.stack, m.surv, m.cap, m.A2,
+                                                                m.verd0, m.verd1, m.vcbits, vcw, m.vsurv, m.vcap,
+                                                                m.words_ns, B);
+  if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
+  k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
+           st>>>(t, m.ctx, m.sel, m.vcbits, vcw, m.verd0, m.verd1, m.words_ns, d_mask, d_status, B);
+  if (ev) GRID_CUDA(cudaEventRecord(ev[5], st));
+  GRID_CUDA(cudaGetLastError());
+  return GRID_OK;
+}
+
 extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
                           void* stream) {
   if (!s || !c || !d_mask || !d_status) return set_error(GRID_E_INVALID_ARG, "grid_masks: bad arguments");
-  cudaStream_t st = (cudaStream_t)stream;
-  const Tables& t = s->t;
-  const int B = c->B;
-  const int zero_blocks = std::min(128, (int)(((size_t)B * c->words_ns / 4 + 1023) / 1024) + 1);
-  k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(
-      t, c->c, c->ctx, c->rng, c->verd0, c->verd1, B, c->words_ns);
-  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c->c, c->ctx, c->A2, c->sel);
-  Tables tw = t;  // the walk reads the small tables through L1; its shared memory holds lane overlays
-  tw.blob_bytes = 0;
-  k_filter<<<dim3((s->max_cd + 255) / 256 + (s->max_cd == 0), B, 2), 256, 0, st>>>(t, c->ctx, c->sel, c->surv, c->cap);
-  k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, c->ctx, c->rng, c->c.stack, c->surv, c->cap, c->A2,
-                                                     c->verd0, c->verd1, c->vcbits, std::max(1, s->vcw),
-                                                     c->words_ns, B);
-  k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
-           st>>>(
-      t, c->ctx, c->sel, c->vcbits, std::max(1, s->vcw), c->verd0, c->verd1, c->words_ns, d_mask, d_status, B);
-  GRID_CUDA(cudaGetLastError());
+  const MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
+                      c->surv, c->vsurv, c->cap, c->vcap, c->words_ns};
+  return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr);
+}
+
+extern "C" int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events) {
+  if (!c || (n_events != 0 && n_events != kMaskKernels + 1) || (n_events && !events))
+    return set_error(GRID_E_INVALID_ARG, "grid_configs_set_events: pass 0 or 6 events");
+  for (int i = 0; i <= kMaskKernels; ++i) {
+    c->ev[i] = n_events ? static_cast<cudaEvent_t>(events[i]) : nullptr;
+    if (n_events && !c->ev[i]) {
+      for (int k = 0; k <= kMaskKernels; ++k) c->ev[k] = nullptr;
+      return set_error(GRID_E_INVALID_ARG, "grid_configs_set_events: null event");
+    }
+  }
   return GRID_OK;
 }
 
@@ -1433,7 +1616,7 @@ uint8_t* g_static_dev[kStaticMaxDevices] = {};
 // Offsets of the step's buffers inside the array (each 256-byte aligned),
 // sized exactly as grid_configs_create sizes the same buffers.
 struct StaticCarve {
-  size_t ctx, rng, sel, verd0, verd1, A2, vcbits, surv, total;
+  size_t ctx, rng, sel, verd0, verd1, A2, vcbits, surv, vsurv, total;
 };
 
 StaticCarve carve_static(const grid_spec* s, int B, int words_ns) {
@@ -1452,6 +1635,7 @@ StaticCarve carve_static(const grid_spec* s, int B, int words_ns) {
   c.A2 = take((size_t)B * 2 * s->t.T1 * 16);
   c.vcbits = take((size_t)B * 2 * std::max(1, s->vcw) * 4);
   c.surv = take((size_t)B * 2 * std::max(1, s->max_cd) * 4);
+  c.vsurv = take((size_t)B * 2 * std::max(1, s->max_vc) * 4);
   c.total = at;
   return c;
 }
@@ -1495,36 +1679,28 @@ extern "C" int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, co
     }
     area = g_static_dev[dev];
   }
-  RowCtx* ctx = reinterpret_cast<RowCtx*>(area + cv.ctx);
-  RowRanges* rng = reinterpret_cast<RowRanges*>(area + cv.rng);
-  uint32_t* sel = reinterpret_cast<uint32_t*>(area + cv.sel);
-  uint32_t* verd0 = reinterpret_cast<uint32_t*>(area + cv.verd0);
-  uint32_t* verd1 = reinterpret_cast<uint32_t*>(area + cv.verd1);
-  uint32_t* A2 = reinterpret_cast<uint32_t*>(area + cv.A2);
-  uint32_t* vcbits = reinterpret_cast<uint32_t*>(area + cv.vcbits);
-  int32_t* surv = reinterpret_cast<int32_t*>(area + cv.surv);
-  const int cap = std::max(1, s->max_cd);
+  const MaskScratch m{reinterpret_cast<RowCtx*>(area + cv.ctx),
+                      reinterpret_cast<RowRanges*>(area + cv.rng),
+                      reinterpret_cast<uint32_t*>(area + cv.sel),
+                      reinterpret_cast<uint32_t*>(area + cv.verd0),
+                      reinterpret_cast<uint32_t*>(area + cv.verd1),
+                      reinterpret_cast<uint32_t*>(area + cv.A2),
+                      reinterpret_cast<uint32_t*>(area + cv.vcbits),
+                      reinterpret_cast<int32_t*>(area + cv.surv),
+                      reinterpret_cast<int32_t*>(area + cv.vsurv),
+                      std::max(1, s->max_cd),
+                      std::max(1, s->max_vc),
+                      words_ns};
   // the kernels only read the configurations
-  DevConfigs c{const_cast<uint16_t*>(d_stack), const_cast<int32_t*>(d_depth), const_cast<int32_t*>(d_dfa_state),
-               const_cast<int32_t*>(d_lex_node), const_cast<int32_t*>(d_flags)};
-  cudaStream_t st = (cudaStream_t)stream;
-  // What must start at zero is cleared by k_prep itself on every call: both
-  // verdict bitmaps (its clearing blocks) and each row's queue, survivor and
-  // completion counters.  The other buffers are written before they are read
-  // within the call, so the previous call's contents do not matter.
-  const int zero_blocks = std::min(128, (int)(((size_t)B * words_ns / 4 + 1023) / 1024) + 1);
-  k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(t, c, ctx, rng, verd0,
-                                                                                               verd1, B, words_ns);
-  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c, ctx, A2, sel);
-  Tables tw = t;
-  tw.blob_bytes = 0;
-  k_filter<<<dim3((s->max_cd + 255) / 256 + (s->max_cd == 0), B, 2), 256, 0, st>>>(t, ctx, sel, surv, cap);
-  k_walk<<<s->walk_blocks, kWalkWarps * 32, 0, st>>>(tw, ctx, rng, d_stack, surv, cap, A2, verd0, verd1, vcbits,
-                                                     std::max(1, s->vcw), words_ns, B);
-  k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
-           st>>>(t, ctx, sel, vcbits, std::max(1, s->vcw), verd0, verd1, words_ns, d_mask, d_status, B);
-  GRID_CUDA(cudaGetLastError());
-  return GRID_OK;
+  const DevConfigs c{const_cast<uint16_t*>(d_stack), const_cast<int32_t*>(d_depth),
+                     const_cast<int32_t*>(d_dfa_state), const_cast<int32_t*>(d_lex_node),
+                     const_cast<int32_t*>(d_flags)};
+  // What must start at zero is cleared by k_prep itself on every call: the
+  // verdict bitmaps and verdict-class bits (its clearing blocks) and each
+  // row's queue, survivor and completion counters.  The other buffers are
+  // written before they are read within the call, so the previous call's
+  // contents do not matter.
+  return launch_masks(s, c, m, B, d_mask, d_status, (cudaStream_t)stream, nullptr);
 }
 
 extern "C" int grid_apply_mask(const uint32_t* d_mask, void* d_logits, int32_t dtype, int32_t B, int32_t V,
