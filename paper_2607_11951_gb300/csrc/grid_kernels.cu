@@ -1,28 +1,39 @@
 // libgrid device side for sm_103a: table upload, CI precompute, configurations
 // and the kernels of the cold full-vocabulary mask.
 //
-// Specialization (grid_specialize, Sec. 4.2 / cold-schema specialization):
-//   k_classify  per (precomputed lexer state, spelling): CI class id, or
-//               always/never viable, or CD (context-dependent)
-//   k_compact   per lexer state: the ascending list of its CD spellings
-//   k_permute   class tables re-indexed by token id (coalesced in k_pack)
+// Specialization (grid_specialize, Sec. 4.2 / cold-schema specialization), for
+// every precomputed lexer state (the start state and each state where no
+// lexicon category is live) and every distinct spelling:
+//   k_classify    the spelling's class: a CI class id (its verdict is a
+//                 function of the allowed set alone), always / never viable,
+//                 a verdict class (its stack-dependent events fit one record),
+//                 or byte-walked CD (more events than a record holds)
+//   k_events      the event records of the verdict-class spellings; the host
+//                 merges equal records (after rewriting class ids with equal
+//                 terminal sets to one id) into the table's verdict classes
+//   k_compact     per lexer state: the ascending list of its byte-walked spellings
+//   k_scatter_vc, k_permute   class codes and verdict-class indices re-indexed
+//                 by token id (coalesced in k_pack)
 //
 // Mask step (grid_masks, Def. 4):
 //   k_prep   one warp per row: A0 = A(sigma) by reduce-chain simulation; the
 //            forced emission of the pending lexeme (what every token whose first
 //            byte ends the lexeme must go through) -> sigma' and A1 = A(sigma');
-//            EOS gate (Sec. 3.2); class selections of both contexts; the
-//            first-byte ranges that continue the pending lexeme
+//            EOS gate (Sec. 3.2); the first bytes that end the lexeme; for rows
+//            without a table, the live first-byte ranges that continue it
 //   k_succ   per row, context and allowed terminal tau: the allowed set after
-//            shifting tau, so walks simulate nothing before their second shift
-//   k_filter per row and context: the CD spellings whose first stack-dependent
-//            emission can succeed (the others are rejected without a walk)
-//   k_walk   surviving CD spellings only: lanes walk token bytes through the DFA and the
-//            identifier trie, emissions pick the highest-priority parser-viable
-//            candidate on a copy-on-write overlay; a rejected prefix skips its
-//            whole trie subtree (Sec. 4.1)
-//   k_pack   per token id: CI class lookup | walked verdict | EOS gate, packed
-//            into the id-order mask (alias classes expand automatically)
+//            shifting tau (walks simulate nothing before their second shift);
+//            the class selections of both contexts
+//   k_filter per row and context: the byte-walked spellings and the verdict
+//            classes whose first stack-dependent emission can succeed
+//   k_walk   persistent; per row: each surviving verdict class evaluated once
+//            against the row's stack, and the byte walks: lanes walk token
+//            bytes through the DFA and the identifier trie, emissions pick the
+//            highest-priority parser-viable candidate on a copy-on-write
+//            overlay, a rejected prefix skips its whole trie subtree (Sec. 4.1)
+//   k_pack   per token id: CI class selection | verdict class | walked verdict
+//            | EOS gate, packed into the id-order mask (alias ids share a
+//            spelling and so a verdict)
 // Parser step (grid_advance):  k_advance.   Masked logits:  k_apply.
 //
 // Every loop is bounded; hitting a bound writes GRID_ST_BOUND.  No kernel traps.
