@@ -32,7 +32,7 @@ METRIC = "cold full-vocab masks/s (batch-32 mask step at V=151,936)"
 
 
 MASK_KERNELS = ["k_prep", "k_succ", "k_filter", "k_walk", "k_pack"]
-WALK_PROFILE = os.path.join(ROOT, "profiles", "k_walk_sql_select_only.md")
+PROFILE = os.path.join(ROOT, "profiles", "%s_sql_select_only.md")
 SMSP_PER_SM = 4  # warp schedulers per SM, each issuing at most one warp instruction per clock
 
 
@@ -60,12 +60,12 @@ def _source_sha():
     return h.hexdigest()[:16]
 
 
-def _walk_counters():
-    """Per-launch counters of the walk kernel from the committed ncu summary of
-    this workload, if they were taken on the current kernel sources."""
+def _counters(kernel):
+    """Per-launch ncu counters of `kernel` from the committed summary of this
+    workload, if they were taken on the current kernel sources."""
     try:
         kv = {}
-        with open(WALK_PROFILE) as f:
+        with open(PROFILE % kernel) as f:
             for line in f:
                 if line.startswith("- ") and ":" in line:
                     k, v = line[2:].split(":", 1)
@@ -139,79 +139,84 @@ def _dist():
     return ws, rank, local
 
 
+def _oracle_pool(wl):
+    import multiprocessing as mp
+    from tests.harness import _init_worker
+    cores = os.cpu_count() or 1
+    ctx = mp.get_context("spawn")
+    return ctx.Pool(cores, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])), cores
+
+
+def _oracle_throughput(pool, cores, wl, rows, jobs_per_row, ids_per_job, seed):
+    """Oracle mask throughput on the pool's workers: each job builds a
+    configuration from its prefix (not timed) and computes the mask bits of a
+    slice of token ids (timed inside the worker).  Returns (token checks per
+    second over all workers, checks, worker-seconds)."""
+    import numpy as np
+    from tests.harness import _oracle_rows_timed
+    V = len(wl["tokens"])
+    rng = np.random.default_rng(seed)
+    jobs = []
+    for r in rows:
+        ids = rng.choice(V, jobs_per_row * ids_per_job, replace=False)
+        for part in np.array_split(ids, jobs_per_row):
+            jobs.append((wl["prefixes"][r % len(wl["prefixes"])], wl["tokens"], wl["eos"], wl["specials"],
+                         [int(x) for x in part]))
+    checks, busy = 0, 0.0
+    for bits, sec in pool.map(_oracle_rows_timed, jobs, chunksize=1):
+        if bits is not None:
+            checks += len(bits)
+            busy += sec
+    return checks / (busy / cores), checks, busy
+
+
 def run_reference(args):
     """The CPU oracle as it stands, on the host cores: each step is a bounded
-    sample (one configuration of the workload, ``--ref-tokens`` token ids,
-    split over a spawn pool of all cores)."""
+    sample of the headline workload (``--ref-tokens`` token ids of one
+    configuration, split over a spawn pool of all cores), scaled to
+    full-vocabulary masks per second."""
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    import numpy as np
-    from tests.harness import _init_worker, _oracle_rows
     from workloads import configs
-    import multiprocessing as mp
     wl = configs.sql_select_only()
     V = len(wl["tokens"])
-    cores = os.cpu_count() or 1
-    S = args.ref_tokens
-    rng = np.random.default_rng(0)
-    ctx = mp.get_context("spawn")
-    times = []
-    with ctx.Pool(cores, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])) as pool:
-        def step(k):
-            row = k % len(wl["prefixes"])
-            ids = rng.choice(V, S, replace=False)
-            parts = np.array_split(ids, cores)
-            jobs = [(wl["prefixes"][row], wl["tokens"], wl["eos"], wl["specials"], list(p)) for p in parts]
-            t0 = time.perf_counter()
-            pool.map(_oracle_rows, jobs, chunksize=1)
-            return time.perf_counter() - t0
-        for k in range(args.warmup):
-            step(k)
-        for k in range(args.steps):
-            times.append(step(k))
+    pool, cores = _oracle_pool(wl)
+    per_job = max(1, args.ref_tokens // cores)
+    times, checks = [], 0
+    with pool:
+        for k in range(args.warmup + args.steps):
+            tps, n, _ = _oracle_throughput(pool, cores, wl, [k], cores, per_job, seed=k)
+            if k >= args.warmup:
+                times.append(n / tps)
+                checks += n
     tot = sum(times)
-    value = args.steps * S / V / tot
+    value = checks / V / tot
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "masks/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
             "data": "synthetic",
             "config": {"workload": "sql_select_only", "B": 32, "V": V},
             "cpu_baseline": {"value": value, "unit": "masks/s", "cores": cores, "kind": "oracle",
-                             "sample": "per step: %d random token ids of one configuration (rows rotate), "
-                                       "split over %d spawn workers" % (S, cores)},
+                             "sample": "per step: %d random token ids of one configuration (rows rotate), split "
+                                       "over %d spawn workers; worker time inside the mask only" %
+                                       (per_job * cores, cores)},
             "e2e": {"value": value, "unit": "masks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
-def cpu_baseline_sample(wl, seconds_target=15.0):
-    """Time the oracle on a bounded sample of the workload: whole rows split
-    across a spawn pool of all host cores; scaled to masks/s."""
-    import numpy as np
-    import multiprocessing as mp
-    from tests.harness import _init_worker, _oracle_rows
+def cpu_baseline_sample(wl):
+    """The oracle on a bounded sample of the workload: 4 configurations x
+    48,000 random token ids over a spawn pool of all host cores, scaled to
+    full-vocabulary masks per second."""
     V = len(wl["tokens"])
-    cores = os.cpu_count() or 1
-    ctx = mp.get_context("spawn")
-    rng = np.random.default_rng(1)
-    n_ids = 24000
-    done = 0
-    with ctx.Pool(cores, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])) as pool:
-        pool.map(_oracle_rows, [(wl["prefixes"][0], wl["tokens"], wl["eos"], wl["specials"], [0])] * cores)
-        t0 = time.perf_counter()
-        rows = 0
-        while time.perf_counter() - t0 < seconds_target / cores * 2 and rows < 8:
-            ids = rng.choice(V, n_ids, replace=False)
-            parts = np.array_split(ids, cores * 2)
-            jobs = [(wl["prefixes"][rows % len(wl["prefixes"])], wl["tokens"], wl["eos"], wl["specials"],
-                     list(p)) for p in parts]
-            pool.map(_oracle_rows, jobs, chunksize=1)
-            done += n_ids
-            rows += 1
-        dt = time.perf_counter() - t0
-    return {"value": done / V / dt, "unit": "masks/s", "cores": cores, "kind": "oracle",
-            "sample": "%d rows x %d random token ids of the headline workload (%.1f s wall on %d spawn "
-                      "workers), scaled to full-vocabulary masks" % (rows, n_ids, dt, cores)}
+    pool, cores = _oracle_pool(wl)
+    with pool:
+        tps, n, busy = _oracle_throughput(pool, cores, wl, range(4), 2 * cores, 48000 // (2 * cores), seed=1)
+    return {"value": tps / V, "unit": "masks/s", "cores": cores, "kind": "oracle",
+            "sample": "4 configurations x 48,000 random token ids of the headline workload (%d checks, %.1f "
+                      "worker-seconds inside the mask on %d spawn workers), scaled to full-vocabulary masks" %
+                      (n, busy, cores)}
 
 
 def main():
@@ -394,10 +399,11 @@ def main():
     # once + every logit written once (the reject fill touches every sector)
     hbm_peak, peak_kind = _peaks()
     apply_bytes = B * W * 4 + B * V * 4
+    ac = _counters("k_apply")
     roof_apply = {"kernel": "k_apply (grid_apply_mask)", "bound": "hbm",
                   "achieved": apply_bytes / (apply_us * 1e-6) / 1e9, "peak": hbm_peak,
-                  "peak_kind": peak_kind + " copy bandwidth", "unit": "GB/s", "traffic": None,
-                  "bytes_per_launch": apply_bytes}
+                  "peak_kind": peak_kind + " copy bandwidth", "unit": "GB/s",
+                  "traffic": ac["dram"] if ac else None, "bytes_per_launch": apply_bytes}
     roof_apply["frac"] = roof_apply["achieved"] / roof_apply["peak"]
     # walk: integer work without a memory stream (tables stay in L1/L2), so
     # its ceiling is the warp-instruction issue rate: SMs x 4 schedulers x
@@ -405,13 +411,13 @@ def main():
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     mhz = clocks.get("sm_mhz") or 2070.0
     issue_peak = sms * SMSP_PER_SM * mhz * 1e6 / 1e9
-    wc = _walk_counters()
+    wc = _counters("k_walk")
     walk_us = kern_us["k_walk"]
     roof_walk = {"kernel": "k_walk (grid_masks)", "bound": "alu", "unit": "G warp-inst/s",
                  "peak": issue_peak, "peak_kind": "derived: %d SMs x %d schedulers x %.0f MHz sampled" %
                  (sms, SMSP_PER_SM, mhz),
                  "achieved": None, "frac": None, "traffic": None,
-                 "counters": "ncu, " + os.path.relpath(WALK_PROFILE, ROOT) if wc else "stale or missing"}
+                 "counters": "ncu, " + os.path.relpath(PROFILE % "k_walk", ROOT) if wc else "stale or missing"}
     if wc:
         roof_walk["achieved"] = wc["inst"] / (walk_us * 1e-6) / 1e9
         roof_walk["frac"] = roof_walk["achieved"] / issue_peak

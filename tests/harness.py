@@ -86,6 +86,26 @@ def _oracle_rows(args):
     return og.mask(cfg, tokens, eos, specials, ids=ids)
 
 
+_CFG_CACHE = {}
+
+
+def _oracle_rows_timed(args):
+    """Like _oracle_rows, plus the seconds spent in the mask itself (building
+    the configuration from its prefix is not part of a mask step)."""
+    import time
+    prefix, tokens, eos, specials, ids = args
+    og = _OG
+    key = tuple(prefix)
+    if key not in _CFG_CACHE:
+        _CFG_CACHE[key] = og.config_from_ids(prefix, tokens, eos, specials)
+    cfg = _CFG_CACHE[key]
+    if cfg is None:
+        return None, 0.0
+    t0 = time.perf_counter()
+    bits = og.mask(cfg, tokens, eos, specials, ids=ids)
+    return bits, time.perf_counter() - t0
+
+
 def oracle_masks(wl, rows=None, ids_per_row=None, procs=None):
     """Oracle bits for the given rows (all by default) over all ids or the
     per-row id subsets ``ids_per_row``.  Returns a list of lists of bits."""
