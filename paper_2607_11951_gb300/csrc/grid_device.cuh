@@ -138,11 +138,43 @@ __device__ __forceinline__ bool bit4(const uint32_t* m, int t) { return (m[t >> 
 // Copy the staged block into shared memory and publish one block-wide copy of
 // the table descriptor, rebased onto it, in shared memory (`ts`).  Every thread
 // of the block must call this.
+// Copy the staged block into shared memory with one bulk asynchronous copy
+// (the block is 16-byte aligned and a multiple of 16 bytes), completion
+// tracked by an mbarrier.  The wait is bounded; if it gives up, the block is
+// copied again with plain loads (same bytes), so the result never depends on
+// the bulk copy finishing.
 __device__ __forceinline__ void stage_tables(const Tables& t, Tables& ts, uint8_t* smem) {
+  __shared__ __align__(8) uint64_t s_bar;
+  __shared__ int s_late;
   if (t.blob_bytes) {
-    const uint4* src = reinterpret_cast<const uint4*>(t.blob);
-    uint4* dst = reinterpret_cast<uint4*>(smem);
-    for (int i = threadIdx.x; i < (t.blob_bytes >> 4); i += blockDim.x) dst[i] = src[i];
+    const uint32_t bar = (uint32_t)__cvta_generic_to_shared(&s_bar);
+    if (threadIdx.x == 0) {
+      s_late = 0;
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(t.blob_bytes)
+                   : "memory");
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              (uint32_t)__cvta_generic_to_shared(smem)),
+          "l"(t.blob), "r"(t.blob_bytes), "r"(bar)
+          : "memory");
+    }
+    __syncthreads();
+    uint32_t done = 0;
+    for (int it = 0; it < (1 << 20) && !done; ++it)
+      asm volatile(
+          "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}"
+          : "=r"(done)
+          : "r"(bar)
+          : "memory");
+    if (!done) s_late = 1;
+    __syncthreads();
+    if (s_late) {
+      const uint4* src = reinterpret_cast<const uint4*>(t.blob);
+      uint4* dst = reinterpret_cast<uint4*>(smem);
+      for (int i = threadIdx.x; i < (t.blob_bytes >> 4); i += blockDim.x) dst[i] = src[i];
+    }
   }
   if (threadIdx.x == 0) {
     ts = t;
