@@ -193,6 +193,11 @@ __device__ __forceinline__ void stage_tables(const Tables& t, Tables& ts, uint8_
   __syncthreads();
 }
 
+// Programmatic dependent launch: the step's kernels are launched so that each
+// may start while its predecessor in the stream finishes; everything a kernel
+// does before this wait touches only the spec's read-only tables.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 constexpr uint32_t kHashEmpty = 0xFFFFFFFFu;
 
 // Child of identifier-trie node lx on byte b (-1 if none), with the child's

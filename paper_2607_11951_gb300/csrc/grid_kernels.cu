@@ -45,6 +45,7 @@
 #include <mutex>
 #include <string>
 #include <unordered_map>
+#include <utility>
 #include <vector>
 
 #include "grid_device.cuh"
@@ -285,6 +286,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
   if ((int)blockIdx.x >= row_blocks) {
     // clearing blocks: zero both verdict bitmaps and the verdict-class bits of every row
+    pdl_wait();
     const size_t n = (size_t)B * words_ns;
     const size_t n4 = n >> 2;
     const size_t stride = (size_t)(gridDim.x - row_blocks) * blockDim.x;
@@ -303,6 +305,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   }
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x * kPrepWarps + warp;
   if (b >= B) return;
@@ -463,9 +466,10 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   __shared__ uint16_t s_scr[kSuccWarps][kMaxOvl * 32];
   __shared__ int s_keep2[kSuccWarps], s_m2[kSuccWarps];
   const int b = blockIdx.x, cx = blockIdx.y;
+  stage_tables(t, ts, smem);
+  pdl_wait();
   const RowCtx& r = ctx[b];
   if (r.complete || (cx == 1 && !r.emit_ok) || (cx == 0 && r.q == kStart)) return;
-  stage_tables(t, ts, smem);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int depth = r.depth;
   const uint16_t* base = c.stack + (size_t)b * t.D;
@@ -538,6 +542,7 @@ __global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ c
                                                 int vcap, int cd_blocks) {
   __shared__ int s_warp[8];
   __shared__ int s_base;
+  pdl_wait();
   const int b = blockIdx.y, cx = blockIdx.z;
   RowCtx& r = ctx[b];
   const int q = r.q, tbl0 = r.tbl0;
@@ -644,6 +649,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   __shared__ int4 s_seg[kWalkRowsCached];
   __shared__ Tables ts;
   stage_tables(t, ts, smem);
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWalkWarps + warp;
   const int mc = max_chain_of(t);
@@ -845,6 +851,7 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   __shared__ int s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
   __shared__ uint32_t s_kill[kPackRows][8];
   __shared__ int s_last;
+  pdl_wait();
   const int id = blockIdx.x * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31;
   const int wi = id >> 5;
@@ -944,6 +951,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
   __shared__ Tables ts;
   __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
   stage_tables(t, ts, smem);
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x * kPrepWarps + warp;
   if (b >= B) return;
@@ -1045,6 +1053,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logits, int B,
                                                int V, int W, long long stride, int vec_ok) {
   constexpr int E = 32 / sizeof(T);  // elements per sector: 8 fp32 or 16 bf16
+  pdl_wait();
   const long long per_row = (V + E - 1) / E;
   const long long total = per_row * B;
   for (long long g = (long long)blockIdx.x * blockDim.x + threadIdx.x; g < total;
@@ -1090,6 +1099,25 @@ __global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask
       }
     }
   }
+}
+
+// Launch with programmatic stream serialization: the kernel may begin (stage
+// its tables) while the previous kernel in the stream drains; it waits for
+// that kernel's results with griddepcontrol.wait (pdl_wait).
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 // ---------------------------------------------------------------------------
@@ -1533,8 +1561,9 @@ extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_con
   if (!s || !in || !out || !d_tokens || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
     return set_error(GRID_E_INVALID_ARG, "grid_advance: bad arguments");
   const int B = in->B;
-  k_advance<<<(B + kPrepWarps - 1) / kPrepWarps, kPrepWarps * 32, s->t.blob_bytes, (cudaStream_t)stream>>>(
-      s->t, in->c, out->c, d_tokens, n_steps, d_status, B, in != out ? 1 : 0);
+  GRID_CUDA(launch_pdl(k_advance, dim3((B + kPrepWarps - 1) / kPrepWarps), dim3(kPrepWarps * 32), s->t.blob_bytes,
+                       (cudaStream_t)stream, s->t, in->c, out->c, d_tokens, n_steps, d_status, B,
+                       in != out ? 1 : 0));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
@@ -1559,22 +1588,26 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
   const size_t zero_words = (size_t)B * m.words_ns * 2 + n_vcbits;
   const int zero_blocks = std::min(128, (int)((zero_words / 8 + 1023) / 1024) + 1);
   if (ev) GRID_CUDA(cudaEventRecord(ev[0], st));
-  k_prep<<<(B + kPrepWarps - 1) / kPrepWarps + zero_blocks, kPrepWarps * 32, t.blob_bytes, st>>>(
-      t, c, m.ctx, m.rng, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns);
+  GRID_CUDA(launch_pdl(k_prep, dim3((B + kPrepWarps - 1) / kPrepWarps + zero_blocks), dim3(kPrepWarps * 32),
+                       t.blob_bytes, st, t, c, m.ctx, m.rng, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
-  k_succ<<<dim3(B, 2, kSuccSlots), kSuccWarps * 32, t.blob_bytes, st>>>(t, c, m.ctx, m.A2, m.sel);
+  GRID_CUDA(launch_pdl(k_succ, dim3(B, 2, kSuccSlots), dim3(kSuccWarps * 32), t.blob_bytes, st, t, c,
+                       (const RowCtx*)m.ctx, m.A2, m.sel));
   if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
   const int cd_blocks = (s->max_cd + 255) / 256;
   const int vc_blocks = (s->max_vc + 255) / 256;
-  k_filter<<<dim3(std::max(1, cd_blocks + vc_blocks), B, 2), 256, 0, st>>>(t, m.ctx, m.sel, m.surv, m.cap, m.vsurv,
-                                                                           m.vcap, cd_blocks);
+  GRID_CUDA(launch_pdl(k_filter, dim3(std::max(1, cd_blocks + vc_blocks), B, 2), dim3(256), 0, st, t, m.ctx,
+                       (const uint32_t*)m.sel, m.surv, m.cap, m.vsurv, m.vcap, cd_blocks));
   if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
-  k_walk<<<s->walk_blocks, kWalkWarps * 32, t.blob_bytes, st>>>(t, m.ctx, m.rng, c.stack, m.surv, m.cap, m.A2,
-                                                                m.verd0, m.verd1, m.vcbits, vcw, m.vsurv, m.vcap,
-                                                                m.words_ns, B);
+  GRID_CUDA(launch_pdl(k_walk, dim3(s->walk_blocks), dim3(kWalkWarps * 32), t.blob_bytes, st, t, m.ctx,
+                       (const RowRanges*)m.rng, (const uint16_t*)c.stack, (const int32_t*)m.surv, m.cap,
+                       (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
+                       m.words_ns, B));
   if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
-  k_pack<<<dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), 256, kPackRows * 2 * std::max(1, t.nselw) * 4,
-           st>>>(t, m.ctx, m.sel, m.vcbits, vcw, m.verd0, m.verd1, m.words_ns, d_mask, d_status, B);
+  GRID_CUDA(launch_pdl(k_pack, dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), dim3(256),
+                       (size_t)kPackRows * 2 * std::max(1, t.nselw) * 4, st, t, m.ctx, (const uint32_t*)m.sel,
+                       (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
+                       m.words_ns, d_mask, d_status, B));
   if (ev) GRID_CUDA(cudaEventRecord(ev[5], st));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
@@ -1730,9 +1763,11 @@ extern "C" int grid_apply_mask(const uint32_t* d_mask, void* d_logits, int32_t d
   long long blocks = (sectors + 255) / 256;
   blocks = std::min<long long>(blocks, (long long)sms * 8);
   if (dtype == GRID_DTYPE_F32)
-    k_apply<float><<<(int)blocks, 256, 0, st>>>(d_mask, (float*)d_logits, B, V, W, row_stride, vec_ok);
+    GRID_CUDA(launch_pdl(k_apply<float>, dim3((int)blocks), dim3(256), 0, st, d_mask, (float*)d_logits, B, V, W,
+                         (long long)row_stride, vec_ok));
   else
-    k_apply<uint16_t><<<(int)blocks, 256, 0, st>>>(d_mask, (uint16_t*)d_logits, B, V, W, row_stride, vec_ok);
+    GRID_CUDA(launch_pdl(k_apply<uint16_t>, dim3((int)blocks), dim3(256), 0, st, d_mask, (uint16_t*)d_logits, B, V,
+                         W, (long long)row_stride, vec_ok));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
