@@ -57,6 +57,7 @@ struct Bits4 {
     w |= i == 3 ? b : 0u;
   }
   __device__ __forceinline__ bool any() const { return (x | y | z | w) != 0u; }
+  __device__ __forceinline__ int count() const { return __popc(x) + __popc(y) + __popc(z) + __popc(w); }
   __device__ __forceinline__ Bits4 operator&(const Bits4& o) const { return Bits4{x & o.x, y & o.y, z & o.z, w & o.w}; }
   __device__ __forceinline__ Bits4 operator|(const Bits4& o) const { return Bits4{x | o.x, y | o.y, z | o.z, w | o.w}; }
   __device__ __forceinline__ Bits4 andnot(const Bits4& o) const {
@@ -94,6 +95,10 @@ struct Tables {
   const uint16_t* go;
   const uint8_t* plen;
   const uint16_t* plhs;
+  const uint32_t* shift_mask;  // S * 4: terminals whose action is SHIFT
+  const uint32_t* red_off;     // S + 1: reduce groups of state s are red_off[s] .. red_off[s+1]
+  const uint16_t* red_p;       // production of each reduce group
+  const uint32_t* red_mask;    // 4 per reduce group: its lookahead terminals
   // identifier trie
   const int32_t* lx_cstart;
   const uint8_t* lx_cbyte;
@@ -130,6 +135,8 @@ struct Tables {
   const uint16_t* vc_rec;     // kRecLen per verdict class
   const uint16_t* vc_first;   // class id of each verdict class's first event
   const uint32_t* vc_by_id;   // n_tbl * V: verdict class (within its table) of kClsVC spellings
+  const uint32_t* cls_sets;   // ncls * 4: terminal set of every class id
+  const uint32_t* cls_mask;   // T1 * nselw: bit c of row tau = tau is in class c's set
 };
 
 // Membership test in a 4-word set stored in memory.
@@ -188,6 +195,10 @@ __device__ __forceinline__ void stage_tables(const Tables& t, Tables& ts, uint8_
       ts.go = reinterpret_cast<const uint16_t*>(rebase(t.go));
       ts.plen = rebase(t.plen);
       ts.plhs = reinterpret_cast<const uint16_t*>(rebase(t.plhs));
+      ts.shift_mask = reinterpret_cast<const uint32_t*>(rebase(t.shift_mask));
+      ts.red_off = reinterpret_cast<const uint32_t*>(rebase(t.red_off));
+      ts.red_p = reinterpret_cast<const uint16_t*>(rebase(t.red_p));
+      ts.red_mask = reinterpret_cast<const uint32_t*>(rebase(t.red_mask));
     }
   }
   __syncthreads();
@@ -292,6 +303,82 @@ __device__ __forceinline__ int simulate(const Tables& t, const uint16_t* base, i
   return -1;
 }
 
+// The terminals of G whose reduce chains on the virtual stack reach SHIFT:
+// simulate() for a set of terminals at once.  Terminals travel together while
+// they take the same action; where the remaining ones reduce by different
+// productions, the group of the first production listed for the state goes
+// on and the others are simulated again from the start in a later round
+// (they follow the same path up to that state).  After kSetRounds rounds the
+// rest is simulated one terminal at a time.  `bound` is set on a bound.
+constexpr int kSetRounds = 8;
+
+template <typename OV>
+__device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* base, int keep, OV ovl, int m, Bits4 G,
+                                              LArr scr, int cap, int max_chain, bool& bound) {
+  Bits4 res = Bits4::zero();
+  Bits4 todo = G;
+  for (int round = 0; round < kSetRounds && todo.any(); ++round) {
+    Bits4 g = todo;
+    todo = Bits4::zero();
+    int k = keep, mm = m, ns = 0;
+    int it = 0;
+    for (; it < max_chain && g.any(); ++it) {
+      const int top = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
+      if (top >= t.S) break;
+      const Bits4 sh = Bits4::load(t.shift_mask + top * 4);
+      res = res | (g & sh);
+      g = g.andnot(sh);
+      if (!g.any()) break;
+      int p = -1;
+      Bits4 gp = Bits4::zero();
+      for (uint32_t e = t.red_off[top]; e < t.red_off[top + 1]; ++e) {
+        const Bits4 x = g & Bits4::load(t.red_mask + e * 4);
+        if (!x.any()) continue;
+        if (p < 0) {
+          p = t.red_p[e];
+          gp = x;
+        } else {
+          todo = todo | x;
+        }
+      }
+      if (p < 0) break;  // the rest is an error here
+      g = gp;
+      int n = t.plen[p];
+      int x = min(n, ns);
+      ns -= x;
+      n -= x;
+      x = min(n, mm);
+      mm -= x;
+      n -= x;
+      k -= n;
+      if (k < 1) break;
+      const int top2 = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
+      if (top2 >= t.S) break;
+      if (ns >= cap) {
+        bound = true;
+        return res;
+      }
+      scr[ns++] = t.go[top2 * t.NNT + t.plhs[p]];
+    }
+    if (it == max_chain && g.any()) {
+      bound = true;
+      return res;
+    }
+  }
+  while (todo.any()) {
+    const int tau = todo.lowest();
+    todo.clear_lowest();
+    int keep_o, m_o, ns;
+    const int a = simulate(t, base, keep, ovl, m, tau, scr, cap, keep_o, m_o, ns, max_chain);
+    if (a < 0) {
+      bound = true;
+      return res;
+    }
+    if (a > 0 && a != kAccept) res.set(tau);
+  }
+  return res;
+}
+
 // Per-lane walk state.  Acur is the allowed-terminal set of the current
 // virtual stack when it is known without simulation: the context's set before
 // any shift, and after the first shift of terminal tau the precomputed set
@@ -371,6 +458,26 @@ __device__ __forceinline__ int emit_set(const Tables& t, Walker& w, Bits4 K, int
       return 1;
     }
     if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
+    if (!w.Acur && K.count() > 0) {
+      // several candidates left: find the first that reaches SHIFT (or is
+      // ignored) with one set simulation, then simulate that one to shift it
+      bool bound = false;
+      Bits4 rest = K;
+      rest.set(tau);
+      const Bits4 ok = simulate_set(t, w.base, w.keep, w.ovl, w.m, rest.andnot(t.ign), w.scr, w.cap, max_chain, bound);
+      if (bound) return -1;
+      const int pick = (ok | (rest & t.ign)).lowest();
+      if (pick < 0) return 0;
+      if (t.ign.has(pick)) return 1;
+      K = Bits4::zero();
+      int keep_o, m_o, ns;
+      const int a = simulate(t, w.base, w.keep, w.ovl, w.m, pick, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+      if (a <= 0 || a == kAccept || !commit(w, keep_o, m_o, ns, a - 1)) return -1;
+      w.shifted = true;
+      w.Acur = (w.nshift == 0 && w.A2) ? w.A2 + pick * 4 : nullptr;
+      ++w.nshift;
+      return 1;
+    }
     int keep_o, m_o, ns;
     int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
     if (a < 0) return -1;
@@ -394,15 +501,16 @@ __device__ __forceinline__ int trailing_set(const Tables& t, Walker& w, Bits4 L,
   if ((L & t.ign).any()) return 1;
   if (const uint32_t* A = w.Acur) return (L & Bits4::load(A)).any() ? 1 : 0;
   if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
-  while (L.any()) {
-    const int tau = L.lowest();
-    L.clear_lowest();
+  if (L.count() == 1) {
     int keep_o, m_o, ns;
-    int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+    const int a = simulate(t, w.base, w.keep, w.ovl, w.m, L.lowest(), w.scr, w.cap, keep_o, m_o, ns, max_chain);
     if (a < 0) return -1;
-    if (a > 0 && a != kAccept) return 1;
+    return a > 0 && a != kAccept ? 1 : 0;
   }
-  return 0;
+  bool bound = false;
+  const Bits4 ok = simulate_set(t, w.base, w.keep, w.ovl, w.m, L, w.scr, w.cap, max_chain, bound);
+  if (bound) return -1;
+  return ok.any() ? 1 : 0;
 }
 
 __device__ __forceinline__ int trailing_live(const Tables& t, Walker& w, int max_chain) {
@@ -493,13 +601,16 @@ __device__ __forceinline__ int class_id(const Tables& t, int kind, int q, uint32
   return ((kind * t.Q + q) << t.n_cat) | (int)(cats & ((1u << t.n_cat) - 1u));
 }
 
-// Terminal set of a class id (for the per-row class selection).
-__device__ __forceinline__ Bits4 class_set(const Tables& t, int cls) {
+// Terminal set of a class id, computed from the lexer tables.
+__device__ __forceinline__ Bits4 class_terms(const Tables& t, int cls) {
   const int hi = cls >> t.n_cat;
   const uint32_t cats = (uint32_t)cls & ((1u << t.n_cat) - 1u);
   const int kind = hi / t.Q, q = hi - kind * t.Q;
   return lex_filter(t, kind ? t.acc : t.live, q, cats);
 }
+
+// The same, from the table of all class ids' sets built at specialization.
+__device__ __forceinline__ Bits4 class_set(const Tables& t, int cls) { return Bits4::load(t.cls_sets + cls * 4); }
 
 // Sec. 4.2 CI/CD classification of one spelling from lexer state (q, lx),
 // with the stack abstracted away.  Emissions whose first candidate is ignored

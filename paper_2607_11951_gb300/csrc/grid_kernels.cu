@@ -41,6 +41,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <array>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -60,8 +61,7 @@ constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared
 constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
-constexpr int kSuccWarps = 8;    // warps per k_succ block
-constexpr int kSuccSlots = 4;    // k_succ blocks per (row, context)
+constexpr int kSuccJobWarps = 4;  // k_succ: warps of lanes, one terminal each (covers 128 terminals)
 constexpr int kWalkRowsCached = 256;  // rows whose queue bounds k_walk keeps in shared memory
 constexpr int kLaneOvl = 32;     // overlay / scratch entries per walk lane (shared memory)
 constexpr int kMaxStage = 96 * 1024;
@@ -182,7 +182,7 @@ __global__ void k_events(Tables t, const uint16_t* __restrict__ cls_sp, const in
 __global__ void k_class_sets(Tables t, uint4* __restrict__ out) {
   const int cls = blockIdx.x * blockDim.x + threadIdx.x;
   if (cls >= t.ncls) return;
-  const Bits4 v = class_set(t, cls);
+  const Bits4 v = class_terms(t, cls);
   out[cls] = make_uint4(v.x, v.y, v.z, v.w);
 }
 
@@ -240,15 +240,19 @@ __global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const u
 }
 
 // ---------------- mask step ----------------
-// Class selection for allowed set A: bit c = set(c) meets A u I.
+// Class selection for allowed set A: bit c = set(c) meets A u I, the OR of
+// the class masks of the terminals in A u I (lanes take the words).
 __device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, int lane) {
   const Bits4 AI = A | t.ign;
-  for (int w0 = 0; w0 < t.nselw; ++w0) {
-    const int cls = w0 * 32 + lane;
-    bool v = false;
-    if (cls < t.ncls) v = (class_set(t, cls) & AI).any();
-    const uint32_t word = __ballot_sync(0xffffffffu, v);
-    if (lane == 0) out[w0] = word;
+  for (int w0 = lane; w0 < t.nselw; w0 += 32) {
+    uint32_t acc = 0u;
+    Bits4 r = AI;
+    while (r.any()) {
+      const int tau = r.lowest();
+      r.clear_lowest();
+      acc |= __ldg(&t.cls_mask[(size_t)tau * t.nselw + w0]);
+    }
+    out[w0] = acc;
   }
 }
 
@@ -450,21 +454,22 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
 }
 
 
-// grid = (B, 2, kSuccSlots): row b, context cx (0: sigma, 1: sigma' after the
-// forced emission).  Jobs j = 0..n_term of a (row, context) are spread over
-// its kSuccSlots * kSuccWarps warps.  Job tau < n_term, for tau allowed in the
-// context: the allowed set after tau's reduce chain and shift (A2), so that a
+// grid = (B, 2): row b, context cx (0: sigma, 1: sigma' after the forced
+// emission).  Warps 0..kSuccJobWarps-1: lane l of warp w takes terminal
+// tau = 32 w + l if tau is allowed in the context and computes the allowed set
+// after tau's reduce chain and shift (A2) with one set simulation, so that a
 // walk or verdict-class evaluation simulates nothing before its second shift.
-// Job n_term: the context's CI class selection.
-__global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c, const RowCtx* __restrict__ ctx,
-                                                          uint32_t* __restrict__ A2, uint32_t* __restrict__ sel) {
+// The last warp: the context's CI class selection.
+__global__ void __launch_bounds__((kSuccJobWarps + 1) * 32) k_succ(Tables t, DevConfigs c,
+                                                                    const RowCtx* __restrict__ ctx,
+                                                                    uint32_t* __restrict__ A2,
+                                                                    uint32_t* __restrict__ sel) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   __shared__ uint16_t s_win[kWalkWin];
   __shared__ uint16_t s_ovl1[kMaxOvl];
-  __shared__ uint16_t s_ovl2[kSuccWarps][kMaxOvl];
-  __shared__ uint16_t s_scr[kSuccWarps][kMaxOvl * 32];
-  __shared__ int s_keep2[kSuccWarps], s_m2[kSuccWarps];
+  __shared__ uint16_t s_ovl2[kSuccJobWarps][kMaxOvl * 32];
+  __shared__ uint16_t s_scr[kSuccJobWarps][kMaxOvl * 32];
   const int b = blockIdx.x, cx = blockIdx.y;
   stage_tables(t, ts, smem);
   pdl_wait();
@@ -482,46 +487,36 @@ __global__ void __launch_bounds__(kSuccWarps * 32) k_succ(Tables t, DevConfigs c
   __syncthreads();
   const int keep = cx ? r.keep1 : depth;
   const Bits4 A = Bits4::load(cx ? r.A1 : r.A0);
+  if (warp == kSuccJobWarps) {
+    if (t.ci_on && (cx == 1 || r.tbl0 >= 0)) select_classes(ts, A, sel + ((size_t)b * 2 + cx) * t.nselw, lane);
+    return;
+  }
   const int mc = max_chain_of(t);
-  uint32_t* out = A2 + ((size_t)b * 2 + cx) * t.T1 * 4;
+  const int tau = warp * 32 + lane;
   int status = GRID_ST_OK;
-  const int nw = kSuccSlots * kSuccWarps;
-  for (int j = blockIdx.z * kSuccWarps + warp; j <= t.n_term; j += nw) {
-    if (j == t.n_term) {
-      if (t.ci_on && (cx == 1 || r.tbl0 >= 0))
-        select_classes(ts, A, sel + ((size_t)b * 2 + cx) * t.nselw, lane);
-      continue;
-    }
-    const int tau = j;
-    if (!A.has(tau)) continue;
-    const LArr scr{s_scr[warp] + lane, 32};
-    if (lane == 0) {
-      int keep_o, m_o, ns;
-      const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
-      int m2 = -1;
-      if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
-        for (int i = 0; i < m_o; ++i) s_ovl2[warp][i] = s_ovl1[i];
-        for (int i = 0; i < ns; ++i) s_ovl2[warp][m_o + i] = scr[i];
-        s_ovl2[warp][m_o + ns] = (uint16_t)(a - 1);
-        m2 = m_o + ns + 1;
-      }
-      s_keep2[warp] = keep_o;
-      s_m2[warp] = m2;
-    }
-    __syncwarp();
-    const int m2 = s_m2[warp];
+  if (tau < t.n_term && A.has(tau)) {
+    const LArr scr{s_scr[warp] + lane, 32}, ovl2{s_ovl2[warp] + lane, 32};
+    int keep_o, m_o, ns;
+    const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
     Bits4 An = Bits4::zero();
-    if (m2 > 0)
-      An = allowed_set(ts, base, s_keep2[warp], s_ovl2[warp], m2, status, lane, scr);
-    else
+    if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
+      for (int i = 0; i < m_o; ++i) ovl2[i] = s_ovl1[i];
+      for (int i = 0; i < ns; ++i) ovl2[m_o + i] = scr[i];
+      ovl2[m_o + ns] = (uint16_t)(a - 1);
+      Bits4 G = Bits4::zero();
+      for (int k = 0; k < t.n_term; ++k) G.set(k);
+      G = G.andnot(ts.ign);
+      bool bound = false;
+      An = simulate_set(ts, base, keep_o, ovl2, m_o + ns + 1, G, scr, kMaxOvl, mc, bound);
+      if (bound) status = GRID_ST_BOUND;
+    } else {
       status = GRID_ST_BOUND;
-    if (lane == 0) {
-      out[tau * 4 + 0] = An.x;
-      out[tau * 4 + 1] = An.y;
-      out[tau * 4 + 2] = An.z;
-      out[tau * 4 + 3] = An.w;
     }
-    __syncwarp();
+    uint32_t* out = A2 + (((size_t)b * 2 + cx) * t.T1 + tau) * 4;
+    out[0] = An.x;
+    out[1] = An.y;
+    out[2] = An.z;
+    out[3] = An.w;
   }
   status = __reduce_max_sync(0xffffffffu, status);
   if (lane == 0 && status != GRID_ST_OK) atomicCAS(const_cast<int32_t*>(&ctx[b].status), GRID_ST_OK, status);
@@ -1236,25 +1231,52 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     delete s;
     return rc;
   };
-  // staged block: byte classes, DFA, acc/live, ACTION, GOTO, production tables
-  std::vector<size_t> off(9, 0);
-  const size_t sizes[8] = {256, h.next.size() * 2, h.acc.size() * 4, h.live.size() * 4, h.action.size() * 2,
-                           h.go.size() * 2, h.plen.size(), h.plhs.size() * 2};
-  for (int k = 0; k < 8; ++k) off[k + 1] = align16(off[k] + sizes[k]);
-  std::vector<uint8_t> blob(off[8], 0);
-  std::memcpy(blob.data() + off[0], h.byte_class, 256);
-  std::memcpy(blob.data() + off[1], h.next.data(), sizes[1]);
-  std::memcpy(blob.data() + off[2], h.acc.data(), sizes[2]);
-  std::memcpy(blob.data() + off[3], h.live.data(), sizes[3]);
-  std::memcpy(blob.data() + off[4], h.action.data(), sizes[4]);
-  std::memcpy(blob.data() + off[5], h.go.data(), sizes[5]);
-  std::memcpy(blob.data() + off[6], h.plen.data(), sizes[6]);
-  std::memcpy(blob.data() + off[7], h.plhs.data(), sizes[7]);
+  // per LALR state: the terminals that shift, and the terminals grouped by
+  // the production they reduce by (for simulating a set of terminals at once)
+  std::vector<uint32_t> shift_mask((size_t)h.S * 4, 0u), red_mask;
+  std::vector<uint32_t> red_off(h.S + 1, 0);
+  std::vector<uint16_t> red_p;
+  for (int st = 0; st < h.S; ++st) {
+    std::vector<std::pair<int, std::array<uint32_t, 4>>> groups;
+    for (int tau = 0; tau < h.T1; ++tau) {
+      const int a = h.action[(size_t)st * h.T1 + tau];
+      if (a > 0 && a != kAccept) {
+        shift_mask[(size_t)st * 4 + (tau >> 5)] |= 1u << (tau & 31);
+      } else if (a < 0) {
+        const int pr = -a - 1;
+        auto it = std::find_if(groups.begin(), groups.end(), [&](const auto& g) { return g.first == pr; });
+        if (it == groups.end()) {
+          groups.push_back({pr, {0u, 0u, 0u, 0u}});
+          it = groups.end() - 1;
+        }
+        it->second[tau >> 5] |= 1u << (tau & 31);
+      }
+    }
+    for (const auto& g : groups) {
+      red_p.push_back((uint16_t)g.first);
+      for (int w = 0; w < 4; ++w) red_mask.push_back(g.second[w]);
+    }
+    red_off[st + 1] = (uint32_t)red_p.size();
+  }
+  // staged block: byte classes, DFA, acc/live, ACTION, GOTO, production
+  // tables, shift masks and reduce groups
+  constexpr int kSec = 12;
+  std::vector<size_t> off(kSec + 1, 0);
+  const size_t sizes[kSec] = {256, h.next.size() * 2, h.acc.size() * 4, h.live.size() * 4, h.action.size() * 2,
+                              h.go.size() * 2, h.plen.size(), h.plhs.size() * 2, shift_mask.size() * 4,
+                              red_off.size() * 4, red_p.size() * 2, red_mask.size() * 4};
+  const void* srcs[kSec] = {h.byte_class, h.next.data(), h.acc.data(), h.live.data(), h.action.data(),
+                            h.go.data(), h.plen.data(), h.plhs.data(), shift_mask.data(), red_off.data(),
+                            red_p.data(), red_mask.data()};
+  for (int k = 0; k < kSec; ++k) off[k + 1] = align16(off[k] + sizes[k]);
+  std::vector<uint8_t> blob(off[kSec], 0);
+  for (int k = 0; k < kSec; ++k)
+    if (sizes[k]) std::memcpy(blob.data() + off[k], srcs[k], sizes[k]);
   const uint8_t* dblob = nullptr;
   int rc = s->mem.upload(blob, &dblob);
   if (rc) return fail(rc);
   t.blob = dblob;
-  t.blob_bytes = off[8] <= (size_t)kMaxStage ? (int)off[8] : 0;
+  t.blob_bytes = off[kSec] <= (size_t)kMaxStage ? (int)off[kSec] : 0;
   t.byte_class = dblob + off[0];
   t.next = reinterpret_cast<const uint16_t*>(dblob + off[1]);
   t.acc = reinterpret_cast<const uint32_t*>(dblob + off[2]);
@@ -1263,6 +1285,10 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   t.go = reinterpret_cast<const uint16_t*>(dblob + off[5]);
   t.plen = dblob + off[6];
   t.plhs = reinterpret_cast<const uint16_t*>(dblob + off[7]);
+  t.shift_mask = reinterpret_cast<const uint32_t*>(dblob + off[8]);
+  t.red_off = reinterpret_cast<const uint32_t*>(dblob + off[9]);
+  t.red_p = reinterpret_cast<const uint16_t*>(dblob + off[10]);
+  t.red_mask = reinterpret_cast<const uint32_t*>(dblob + off[11]);
   Arena& a = s->mem;
   {
     // identifier-trie edges -> open-addressing hash (load factor <= 1/2)
@@ -1399,13 +1425,23 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   // class ids with equal terminal sets are interchangeable in a record:
   // rewrite each to the smallest such id before deduplication
   std::vector<uint16_t> canon(std::max(1, t.ncls));
-  if (nslot > 0 && t.ncls > 0) {
+  if (t.ncls > 0) {
+    // terminal set of every class id, and per terminal the mask of the
+    // classes whose set holds it (the class selection ORs these)
     uint4* sets_d = nullptr;
-    if ((rc = tmp.alloc((size_t)t.ncls * 16, (void**)&sets_d))) return fail_tmp(rc);
+    if ((rc = a.alloc((size_t)t.ncls * 16, (void**)&sets_d))) return fail_tmp(rc);
     k_class_sets<<<(t.ncls + 255) / 256, 256, 0, st>>>(t, sets_d);
     std::vector<uint4> sets(t.ncls);
     GRID_CUDA(cudaMemcpyAsync(sets.data(), sets_d, (size_t)t.ncls * 16, cudaMemcpyDeviceToHost, st));
     GRID_CUDA(cudaStreamSynchronize(st));
+    t.cls_sets = reinterpret_cast<const uint32_t*>(sets_d);
+    std::vector<uint32_t> cmask((size_t)t.T1 * t.nselw, 0u);
+    for (int c = 0; c < t.ncls; ++c) {
+      const uint32_t wv[4] = {sets[c].x, sets[c].y, sets[c].z, sets[c].w};
+      for (int tau = 0; tau < t.T1; ++tau)
+        if ((wv[tau >> 5] >> (tau & 31)) & 1u) cmask[(size_t)tau * t.nselw + (c >> 5)] |= 1u << (c & 31);
+    }
+    if ((rc = a.upload(cmask, &t.cls_mask))) return fail_tmp(rc);
     std::unordered_map<std::string, uint16_t> first;
     for (int c = 0; c < t.ncls; ++c) {
       std::string key(reinterpret_cast<const char*>(&sets[c]), 16);
@@ -1591,7 +1627,7 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
   GRID_CUDA(launch_pdl(k_prep, dim3((B + kPrepWarps - 1) / kPrepWarps + zero_blocks), dim3(kPrepWarps * 32),
                        t.blob_bytes, st, t, c, m.ctx, m.rng, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
-  GRID_CUDA(launch_pdl(k_succ, dim3(B, 2, kSuccSlots), dim3(kSuccWarps * 32), t.blob_bytes, st, t, c,
+  GRID_CUDA(launch_pdl(k_succ, dim3(B, 2), dim3((kSuccJobWarps + 1) * 32), t.blob_bytes, st, t, c,
                        (const RowCtx*)m.ctx, m.A2, m.sel));
   if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
   const int cd_blocks = (s->max_cd + 255) / 256;
