@@ -219,6 +219,131 @@ def cpu_baseline_sample(wl):
                       (n, busy, cores)}
 
 
+def _time_steps(fn, steps, warmup, stream):
+    """Per-step device times (us) of fn(k) over `steps` steps after `warmup`."""
+    import torch
+    for k in range(warmup):
+        fn(k)
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for k in range(steps):
+        evs[k][0].record(stream)
+        fn(warmup + k)
+        evs[k][1].record(stream)
+    torch.cuda.synchronize()
+    return sorted(a.elapsed_time(b) * 1e3 for a, b in evs)
+
+
+def run_sweep(args):
+    """Flatness of the per-step cost (the paper's requirement R): grid_masks on
+    B=32 configurations per cell, n in {100, 1k, 4k, 16k} prefix tokens x
+    nesting depth in {1, 8, 32, 64}; p50 per cell and, per depth, the OLS slope
+    of step time vs n."""
+    import numpy as np
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    from workloads import configs
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream()
+    ns, depths = [100, 1000, 4000, 16000], [1, 8, 32, 64]
+    first = configs.sql_sweep_cell(ns[0], depths[0])
+    grammar = G.Grammar(first["grammar"], first["role"], first["lexicons"])
+    vocab = G.Vocab(first["tokens"], first["eos"], first["specials"])
+    spec = G.Spec(grammar, vocab)
+    B, V = first["B"], len(first["tokens"])
+    W = (V + 31) // 32
+    mask = torch.zeros((B, W), dtype=torch.int32, device=dev)
+    status = torch.zeros(B, dtype=torch.int32, device=dev)
+    cells = {}
+    for d in depths:
+        for n in ns:
+            wl = configs.sql_sweep_cell(n, d)
+            c = G.Configs(spec, B)
+            tt = np.full((B, n), -1, dtype=np.int32)
+            for i, p in enumerate(wl["prefixes"]):
+                tt[i, :len(p)] = p
+            G.grid_advance(spec.h, c.h, c.h, torch.from_numpy(tt).to(dev), status)
+            torch.cuda.synchronize()
+            assert (status.cpu().numpy() == 0).all(), (n, d, status)
+            t = _time_steps(lambda k: G.grid_masks(spec.h, c.h, mask, status, stream), args.steps, args.warmup,
+                            stream)
+            assert (status.cpu().numpy() == 0).all(), (n, d, status)
+            cells["%d,%d" % (n, d)] = {"p50_us": t[len(t) // 2], "p99_us": t[min(len(t) - 1, int(0.99 * len(t)))]}
+    slopes = {}
+    for d in depths:
+        x = np.array(ns, dtype=np.float64)
+        y = np.array([cells["%d,%d" % (n, d)]["p50_us"] for n in ns])
+        slope = float(np.polyfit(x, y, 1)[0]) * 1000.0
+        slopes[str(d)] = {"us_per_1k_tokens": slope, "p50_at_100": y[0], "p50_at_16k": y[-1]}
+    print(json.dumps({"metric": "grid_masks p50 us per batch-32 step vs prefix length (flatness)",
+                      "unit": "us", "higher_is_better": False, "steps": args.steps, "warmup": args.warmup,
+                      "config": {"workload": "sql_sweep_cell", "B": B, "V": V, "grammar": "SQL admin",
+                                 "schema": "200 x 30", "n": ns, "depth": depths},
+                      "cells": cells, "ols_slope_by_depth": slopes}), flush=True)
+
+
+def run_cold(args):
+    """Cold-schema specialization: grid_specialize (CI classes of every
+    precomputed lexer state over V=151,936) for a fresh 1,000 x 50 schema,
+    then B=256 steps (advance + masks + bf16 apply) on its configurations."""
+    import numpy as np
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    from workloads import configs
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream()
+    wl = configs.sql_cold_schema()
+    B, V = wl["B"], len(wl["tokens"])
+    W = (V + 31) // 32
+    t0 = time.perf_counter()
+    grammar = G.Grammar(wl["grammar"], wl["role"], wl["lexicons"])
+    t1 = time.perf_counter()
+    vocab = G.Vocab(wl["tokens"], wl["eos"], wl["specials"])
+    t2 = time.perf_counter()
+    spec_ms = []
+    specs = []
+    for k in range(4):  # the first includes one-time CUDA module set-up
+        torch.cuda.synchronize()
+        a = time.perf_counter()
+        specs.append(G.Spec(grammar, vocab))
+        torch.cuda.synchronize()
+        spec_ms.append((time.perf_counter() - a) * 1e3)
+    spec = specs[-1]
+    status = torch.zeros(B, dtype=torch.int32, device=dev)
+    mask = torch.zeros((B, W), dtype=torch.int32, device=dev)
+    c = G.Configs(spec, B)
+    n = max(len(p) for p in wl["prefixes"])
+    tt = np.full((B, n), -1, dtype=np.int32)
+    for i, p in enumerate(wl["prefixes"]):
+        tt[i, :len(p)] = p
+    G.grid_advance(spec.h, c.h, c.h, torch.from_numpy(tt).to(dev), status)
+    G.grid_masks(spec.h, c.h, mask, status)
+    torch.cuda.synchronize()
+    assert (status.cpu().numpy() == 0).all(), status
+    from tests.harness import unpack
+    bits = unpack(mask.cpu().numpy().view(np.uint32), V)
+    rng = np.random.default_rng(7)
+    tok = torch.from_numpy(np.array([rng.choice(np.nonzero(bits[i])[0]) for i in range(B)], np.int32)).to(dev)
+    scratch = G.Configs(spec, B)
+    logits = [torch.from_numpy(configs.logits(200 + k, B, V)).to(dev).to(torch.bfloat16) for k in range(2)]
+
+    def step(k):
+        G.grid_advance(spec.h, c.h, scratch.h, tok, status, stream)
+        G.grid_masks(spec.h, scratch.h, mask, status, stream)
+        G.grid_apply_mask(mask, logits[k % 2], stream)
+
+    t = _time_steps(step, args.steps, args.warmup, stream)
+    p50 = t[len(t) // 2]
+    print(json.dumps({"metric": "cold-schema specialization ms and B=256 masks/s", "unit": "ms | masks/s",
+                      "grid_specialize_ms": sorted(spec_ms[1:])[1], "grid_specialize_ms_first": spec_ms[0],
+                      "grid_compile_ms": (t1 - t0) * 1e3, "grid_load_vocab_ms": (t2 - t1) * 1e3,
+                      "spec": spec.info(), "step_p50_us": p50, "masks_per_s": B / (p50 * 1e-6),
+                      "steps": args.steps, "warmup": args.warmup,
+                      "config": {"workload": "sql_cold_schema", "B": B, "V": V, "schema": "1,000 x 50",
+                                 "logits": "bf16 N(0,3), 2 rotating batches = 156 MB > L2",
+                                 "step": "grid_advance + grid_masks + grid_apply_mask"}}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -228,9 +353,17 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=8192)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--workload", default="headline", choices=["headline", "sweep", "cold"],
+                    help="headline: the driver's line; sweep: per-step cost vs prefix length and nesting "
+                         "(n in {100,1k,4k,16k} x depth in {1,8,32,64}); cold: specialization of a fresh "
+                         "1,000 x 50 schema, then B=256 steps with bf16 logits")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "sweep":
+        return run_sweep(args)
+    if args.workload == "cold":
+        return run_cold(args)
     args.warmup = max(3, args.warmup)
 
     import numpy as np

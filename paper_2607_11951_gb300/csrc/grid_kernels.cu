@@ -256,24 +256,27 @@ __device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, in
   }
 }
 
-// A(sigma) for the virtual stack base[0:keep] ++ ovl[0:m]: lane l simulates
-// terminals l, l+32, ...; `scr` is the lane's scratch (kMaxOvl entries).
+// A(sigma) for the virtual stack base[0:keep] ++ ovl[0:m], by one set
+// simulation on lane 0 (`scr`: its scratch, kMaxOvl entries), broadcast to
+// the warp.
 __device__ Bits4 allowed_set(const Tables& t, const uint16_t* base, int keep, const uint16_t* ovl, int m,
                              int& status, int lane, LArr scr) {
   const int mc = max_chain_of(t);
-  uint32_t wds[4];
-#pragma unroll
-  for (int wd = 0; wd < 4; ++wd) {
-    const int tau = wd * 32 + lane;
-    bool ok = false;
-    if (tau < t.n_term && !t.ign.has(tau)) {
-      int keep_o, m_o, ns;
-      int a = simulate(t, base, keep, ovl, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
-      ok = a > 0 && a != kAccept;
-      if (a < 0) status = GRID_ST_BOUND;
-    }
-    wds[wd] = __ballot_sync(0xffffffffu, ok);
+  uint32_t wds[4] = {0u, 0u, 0u, 0u};
+  if (lane == 0) {
+    Bits4 G = Bits4::zero();
+    for (int k = 0; k < t.n_term; ++k) G.set(k);
+    G = G.andnot(t.ign);
+    bool bound = false;
+    const Bits4 A = simulate_set(t, base, keep, ovl, m, G, scr, kMaxOvl, mc, bound);
+    if (bound) status = GRID_ST_BOUND;
+    wds[0] = A.x;
+    wds[1] = A.y;
+    wds[2] = A.z;
+    wds[3] = A.w;
   }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) wds[k] = __shfl_sync(0xffffffffu, wds[k], 0);
   return Bits4{wds[0], wds[1], wds[2], wds[3]};
 }
 
@@ -287,6 +290,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   __shared__ uint16_t s_scr[kPrepWarps][kMaxOvl * 32];
   __shared__ uint32_t s_A0[kPrepWarps][4];
   __shared__ int s_km[kPrepWarps][3];
+  __shared__ uint32_t s_keep[kPrepWarps][8];
   const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
   if ((int)blockIdx.x >= row_blocks) {
     // clearing blocks: zero both verdict bitmaps and the verdict-class bits of every row
@@ -380,38 +384,64 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
   // every spelling it starts: liveness only shrinks along the lexeme, and any
   // later emission picks among its live terminals.
   int total0 = 0, nrng = 0;
-  if (!complete && q != kStart) {
-    if (tbl0 < 0) {
-      RowRanges& R = rng[b];
-      const Bits4 AI = A0 | ts.ign;
-      for (int b0 = 0; b0 < 256; b0 += 32) {
-        const int by = b0 + lane;
-        const int lo = t.first_of_byte[by], hi = t.first_of_byte[by + 1];
-        const int q2 = ts.next[q * ts.C + ts.byte_class[by]];
-        bool cont = hi > lo && q2 != kDead;
-        if (cont) {
-          uint32_t pc2 = 0u, wc2 = 0u;
-          if (lx >= 0) lex_step(ts, lx, by, pc2, wc2);
-          cont = (live_prime(ts, q2, pc2) & AI).any();
-        }
-        const int chunks = cont ? (hi - lo + kRangeSpan - 1) / kRangeSpan : 0;
-        const uint32_t bal = __ballot_sync(0xffffffffu, cont);
-        int incl = chunks;
-        for (int d = 1; d < 32; d <<= 1) {
-          int v = __shfl_up_sync(0xffffffffu, incl, d);
-          if (lane >= d) incl += v;
-        }
-        if (cont) {
-          const int k = nrng + __popc(bal & ((1u << lane) - 1u));
-          R.lo[k] = lo;
-          R.hi[k] = hi;
-          R.cpre[k] = total0 + incl - chunks;
-        }
-        total0 += __shfl_sync(0xffffffffu, incl, 31);
-        nrng += __popc(bal);
-      }
-      if (lane == 0) R.cpre[nrng] = total0;
+  if (!complete && q != kStart && tbl0 < 0) {
+    RowRanges& R = rng[b];
+    const Bits4 AI = A0 | ts.ign;
+    int lo_r[8], hi_r[8];
+    uint32_t cw[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      lo_r[j] = t.first_of_byte[j * 32 + lane];
+      hi_r[j] = t.first_of_byte[j * 32 + lane + 1];
     }
+    int nc = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int by = j * 32 + lane;
+      cw[j] = __ballot_sync(0xffffffffu, hi_r[j] > lo_r[j] && ts.next[q * ts.C + ts.byte_class[by]] != kDead);
+      nc += __popc(cw[j]);
+    }
+    // the live test of the continuing bytes, one byte per lane
+    if (lane < 8) s_keep[warp][lane] = 0u;
+    __syncwarp();
+    for (int i0 = 0; i0 < nc; i0 += 32) {
+      int idx = i0 + lane, by = -1;
+      if (idx < nc) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int cnt = __popc(cw[j]);
+          if (by < 0 && idx < cnt) by = j * 32 + (int)__fns(cw[j], 0u, idx + 1);
+          if (by < 0) idx -= cnt;
+        }
+      }
+      if (by >= 0) {
+        uint32_t pc2 = 0u, wc2 = 0u;
+        if (lx >= 0) lex_step(ts, lx, by, pc2, wc2);
+        const int q2 = ts.next[q * ts.C + ts.byte_class[by]];
+        if ((live_prime(ts, q2, pc2) & AI).any()) atomicOr(&s_keep[warp][by >> 5], 1u << (by & 31));
+      }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const bool cont = (s_keep[warp][j] >> lane) & 1u;
+      const int chunks = cont ? (hi_r[j] - lo_r[j] + kRangeSpan - 1) / kRangeSpan : 0;
+      const uint32_t bal = __ballot_sync(0xffffffffu, cont);
+      int incl = chunks;
+      for (int d = 1; d < 32; d <<= 1) {
+        int v = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += v;
+      }
+      if (cont) {
+        const int k = nrng + __popc(bal & ((1u << lane) - 1u));
+        R.lo[k] = lo_r[j];
+        R.hi[k] = hi_r[j];
+        R.cpre[k] = total0 + incl - chunks;
+      }
+      total0 += __shfl_sync(0xffffffffu, incl, 31);
+      nrng += __popc(bal);
+    }
+    if (lane == 0) R.cpre[nrng] = total0;
   }
   // first bytes that end the pending lexeme (every byte when it is empty)
   for (int b0 = 0; b0 < 256; b0 += 32) {
