@@ -132,6 +132,25 @@ def _gpu_index(local):
     return local
 
 
+def max_over_ranks(ms, ws, device):
+    """The slowest rank's time: every rank runs its own replica of the step
+    (rows are independent; no collective on the data path), so the job takes
+    as long as the slowest one.  A barrier follows so no rank runs ahead."""
+    if ws <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    tt = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    dist.barrier()
+    return float(tt.item())
+
+
+def replica_value(ws, B, steps, ms):
+    """Whole-job masks/s: every rank's B rows per step, over the slowest time."""
+    return ws * B * steps / (ms / 1e3)
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -472,11 +491,7 @@ def main():
     torch.cuda.synchronize()
     G.grid_configs_set_events(scratch.h, [])
     clocks = clk.stop()
-    if ws > 1:
-        tt = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(tt.item())
-        torch.distributed.barrier()
+    total_ms = max_over_ranks(total_ms, ws, dev)
     per_step = [e[0].elapsed_time(e[3]) * 1e3 for e in ev_b]
     adv_us = statistics.mean(e[0].elapsed_time(e[1]) * 1e3 for e in ev_b)
     masks_us = statistics.mean(e[1].elapsed_time(e[2]) * 1e3 for e in ev_b)
@@ -487,7 +502,7 @@ def main():
     per_step.sort()
     p50 = per_step[len(per_step) // 2]
     p99 = per_step[min(len(per_step) - 1, int(math.ceil(0.99 * len(per_step))) - 1)]
-    value = ws * B * args.steps / (total_ms / 1e3)
+    value = replica_value(ws, B, args.steps, total_ms)
 
     # ---- end to end through the public API with host buffers ----
     e2e = None
@@ -520,11 +535,8 @@ def main():
         b.record()
         torch.cuda.synchronize()
         e_ms = a.elapsed_time(b)
-        if ws > 1:
-            tt = torch.tensor([e_ms], device=dev)
-            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-            e_ms = float(tt.item())
-        e2e = {"value": ws * B * args.steps / (e_ms / 1e3), "unit": "masks/s",
+        e_ms = max_over_ranks(e_ms, ws, dev)
+        e2e = {"value": replica_value(ws, B, args.steps, e_ms), "unit": "masks/s",
                "h2d_bytes_per_step": B * 4 + B * V * 4, "d2h_bytes_per_step": B * W * 4 + B * 4}
 
     # ---- rooflines ----
