@@ -81,6 +81,7 @@ struct Bits4 {
 struct Tables {
   int n_term, T1, S, NNT, P, Q, C, n_cat, LN;
   int NS, V, eos, W, D;
+  int Vp;     // V rounded up to a multiple of 4: the row length of the id-indexed tables
   Bits4 ign;  // ignored terminals (the set I)
   Bits4 cm;   // category terminals
   int cat_term[32];

@@ -62,6 +62,10 @@ constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
 constexpr int kSuccJobWarps = 4;  // k_succ: warps of lanes, one terminal each (covers 128 terminals)
+// Class codes as k_pack reads them: CI class ids 0..ncls-1, then these five
+// (so that one bit test of the row's class selection covers CI, always and
+// never, and only verdict-class and walked tokens need a second lookup).
+constexpr int kPackCodes = 5;  // ncls + 0 always, +1 never, +2 n/a, +3 verdict class, +4 walked
 constexpr int kWalkRowsCached = 256;  // rows whose queue bounds k_walk keeps in shared memory
 constexpr int kLaneOvl = 32;     // overlay / scratch entries per walk lane (shared memory)
 constexpr int kMaxStage = 96 * 1024;
@@ -229,13 +233,16 @@ __global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const u
                           uint16_t* __restrict__ cls_by_id, uint32_t* __restrict__ vc_by_id,
                           uint8_t* __restrict__ fb_by_id) {
   const int id = blockIdx.x * blockDim.x + threadIdx.x;
-  if (id >= t.V) return;
-  const int s = t.spell_of_id[id];
+  if (id >= t.Vp) return;
+  const int s = t.spell_of_id[id];  // -1 for EOS, specials and the padding ids
   fb_by_id[id] = s >= 0 ? t.spell_bytes[t.spell_off[s]] : 0;
   for (int k = 0; k < t.n_tbl; ++k) {
     const uint16_t c = s >= 0 ? cls_sp[(size_t)k * t.NS + s] : kClsNA;
-    cls_by_id[(size_t)k * t.V + id] = c;
-    vc_by_id[(size_t)k * t.V + id] = c == kClsVC ? vc_sp[(size_t)k * t.NS + s] : 0xFFFFFFFFu;
+    uint16_t code = c;  // the k_pack code of c
+    if (c >= kClsFirstCode)
+      code = (uint16_t)(t.ncls + (c == kClsAcc ? 0 : c == kClsRej ? 1 : c == kClsNA ? 2 : c == kClsVC ? 3 : 4));
+    cls_by_id[(size_t)k * t.Vp + id] = code;
+    vc_by_id[(size_t)k * t.Vp + id] = c == kClsVC ? vc_sp[(size_t)k * t.NS + s] : 0xFFFFFFFFu;
   }
 }
 
@@ -252,6 +259,7 @@ __device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, in
       r.clear_lowest();
       acc |= __ldg(&t.cls_mask[(size_t)tau * t.nselw + w0]);
     }
+    if (w0 == (t.ncls >> 5)) acc |= 1u << (t.ncls & 31);  // the code "always"
     out[w0] = acc;
   }
 }
@@ -862,11 +870,15 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
 }
 
-// grid = (ceil(V/256), ceil(B/kPackRows)), 256 threads: one token id per
-// thread and kPackRows rows per block.  The per-id data (spelling, first byte,
-// start-state class) is loaded once; each warp writes one mask word per row.
-// The last block to finish writes every row's status (EMPTY_MASK for a viable
-// row with no bit set).
+// grid = (ceil(Vp/1024), ceil(B/kPackRows)), 256 threads: four consecutive
+// token ids per thread (vector loads of the id tables) and kPackRows rows per
+// block, whose context (flags, kill bits, class selections) is staged in
+// shared memory.  Per row, a token's code indexes the context's class
+// selection (CI, always, never in one bit test) and only verdict-class and
+// walked codes look further; the eight lanes that hold a mask word's 32 ids
+// combine their 4-bit pieces with shuffles and one of them stores it.  The
+// last block to finish writes every row's status (EMPTY_MASK for a viable row
+// with no bit set).
 __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
                                               const uint32_t* __restrict__ vcbits, int vcw,
                                               const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
@@ -877,12 +889,12 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   __shared__ uint32_t s_kill[kPackRows][8];
   __shared__ int s_last;
   pdl_wait();
-  const int id = blockIdx.x * blockDim.x + threadIdx.x;
-  const int lane = threadIdx.x & 31;
-  const int wi = id >> 5;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int base = blockIdx.x * 1024 + warp * 128 + lane * 4;  // this thread's ids base .. base+3
   const int r0 = blockIdx.y * kPackRows;
   const int nr = min(kPackRows, B - r0);
   const int nw = t.nselw;
+  const int code_vc = t.ncls + 3, code_walk = t.ncls + 4, code_never = t.ncls + 1;
   for (int i = threadIdx.x; i < nr; i += blockDim.x) {
     const RowCtx& rc = ctx[r0 + i];
     s_tbl[i] = rc.tbl0;
@@ -890,63 +902,68 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
     s_any[i] = 0;
   }
   for (int i = threadIdx.x; i < nr * 8; i += blockDim.x) s_kill[i >> 3][i & 7] = ctx[r0 + (i >> 3)].kill[i & 7];
-  for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) s_sel[i] = sel[(size_t)r0 * 2 * nw + i];
-  int s = -1, b0 = 0;
-  uint16_t cl_start = kClsNA;
-  uint32_t vc_start = 0u;
-  if (id < t.V && id != t.eos) {
-    s = t.spell_of_id[id];
-    if (s >= 0) {
-      b0 = t.first_byte_by_id[id];
-      cl_start = t.cls_by_id[id];
-      if (cl_start == kClsVC) vc_start = t.vc_by_id[id];
-    }
+  __syncthreads();
+  // class selections; a context that k_succ did not select for (a completed
+  // row, sigma' without a forced emission, sigma without a table) reads zeros
+  for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) {
+    const int k = i / (2 * nw), cx = (i / nw) & 1;
+    const int fl = s_fl[k];
+    const bool valid = t.ci_on && !(fl & 4) && (cx ? (fl & 1) : s_tbl[k] >= 0);
+    s_sel[i] = valid ? sel[(size_t)r0 * 2 * nw + i] : 0u;
   }
+  // per-id data of the four ids (the tables are padded to Vp ids)
+  int sp[4] = {-1, -1, -1, -1}, b0[4] = {0, 0, 0, 0}, cs[4] = {code_never, code_never, code_never, code_never};
+  uint32_t vs[4] = {0u, 0u, 0u, 0u};
+  const bool have = base < t.Vp;
+  if (have) {
+    const int4 s4 = *reinterpret_cast<const int4*>(t.spell_of_id + base);
+    const uchar4 f4 = *reinterpret_cast<const uchar4*>(t.first_byte_by_id + base);
+    const ushort4 c4 = *reinterpret_cast<const ushort4*>(t.cls_by_id + base);
+    sp[0] = s4.x, sp[1] = s4.y, sp[2] = s4.z, sp[3] = s4.w;
+    b0[0] = f4.x, b0[1] = f4.y, b0[2] = f4.z, b0[3] = f4.w;
+    cs[0] = c4.x, cs[1] = c4.y, cs[2] = c4.z, cs[3] = c4.w;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (cs[j] == code_vc) vs[j] = t.vc_by_id[base + j];
+  }
+  const int eos_j = t.eos - base;  // the EOS id's slot in this thread, if 0..3
+  if (eos_j >= 0 && eos_j < 4) sp[eos_j] = -1;  // EOS takes only the gate's bit
   __syncthreads();
   for (int k = 0; k < nr; ++k) {
     const int b = r0 + k;
     const int fl = s_fl[k];
-    bool bit = false;
-    if (id < t.V && !(fl & 4)) {
-      if (id == t.eos) {
-        bit = fl & 2;
-      } else if (s >= 0) {
-        if ((s_kill[k][b0 >> 5] >> (b0 & 31)) & 1u) {
-          if (fl & 1) {
-            const uint16_t cl = cl_start;
-            if (cl < kClsFirstCode)
-              bit = (s_sel[(2 * k + 1) * nw + (cl >> 5)] >> (cl & 31)) & 1u;
-            else if (cl == kClsAcc)
-              bit = true;
-            else if (cl == kClsCD)
-              bit = (verd1[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-            else if (cl == kClsVC)
-              bit = (vcbits[((size_t)b * 2 + 1) * vcw + (vc_start >> 5)] >> (vc_start & 31)) & 1u;
-          }
-        } else {
-          const int tbl0 = s_tbl[k];
-          if (tbl0 >= 0) {
-            const uint16_t cl = t.cls_by_id[(size_t)tbl0 * t.V + id];
-            if (cl < kClsFirstCode)
-              bit = (s_sel[2 * k * nw + (cl >> 5)] >> (cl & 31)) & 1u;
-            else if (cl == kClsAcc)
-              bit = true;
-            else if (cl == kClsCD)
-              bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
-            else if (cl == kClsVC) {
-              const uint32_t v = t.vc_by_id[(size_t)tbl0 * t.V + id];
-              bit = (vcbits[(size_t)b * 2 * vcw + (v >> 5)] >> (v & 31)) & 1u;
-            }
+    const int tb = s_tbl[k];
+    uint32_t nib = 0u;
+    if (have && !(fl & 4)) {
+      ushort4 ct = make_ushort4(code_walk, code_walk, code_walk, code_walk);
+      if (tb >= 0) ct = *reinterpret_cast<const ushort4*>(t.cls_by_id + (size_t)tb * t.Vp + base);
+      const int ctv[4] = {ct.x, ct.y, ct.z, ct.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (sp[j] < 0) continue;
+        const int cx = (s_kill[k][b0[j] >> 5] >> (b0[j] & 31)) & 1u;
+        const int code = cx ? cs[j] : ctv[j];
+        uint32_t bit = (s_sel[(2 * k + cx) * nw + (code >> 5)] >> (code & 31)) & 1u;
+        if (code >= code_vc && (!cx || (fl & 1))) {
+          if (code == code_vc) {
+            const uint32_t v = cx ? vs[j] : t.vc_by_id[(size_t)tb * t.Vp + base + j];
+            bit = (vcbits[((size_t)b * 2 + cx) * vcw + (v >> 5)] >> (v & 31)) & 1u;
           } else {
-            bit = (verd0[(size_t)b * words_ns + (s >> 5)] >> (s & 31)) & 1u;
+            bit = ((cx ? verd1 : verd0)[(size_t)b * words_ns + (sp[j] >> 5)] >> (sp[j] & 31)) & 1u;
           }
         }
+        nib |= bit << j;
       }
+      if (eos_j >= 0 && eos_j < 4 && (fl & 2)) nib |= 1u << eos_j;
     }
-    const uint32_t word = __ballot_sync(0xffffffffu, bit);
-    if (lane == 0 && wi < t.W) {
-      mask[(size_t)b * t.W + wi] = word;
-      if (word) s_any[k] = 1;
+    uint32_t v = nib << (4 * (lane & 7));
+    v |= __shfl_xor_sync(0xffffffffu, v, 1);
+    v |= __shfl_xor_sync(0xffffffffu, v, 2);
+    v |= __shfl_xor_sync(0xffffffffu, v, 4);
+    const int wi = (blockIdx.x * 1024 + warp * 128) / 32 + (lane >> 3);
+    if ((lane & 7) == 0 && wi < t.W) {
+      mask[(size_t)b * t.W + wi] = v;
+      if (v) s_any[k] = 1;
     }
   }
   __syncthreads();
@@ -1218,9 +1235,9 @@ static int set_smem_limits() {
   GRID_CUDA(cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_events, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   // k_pack: the class selections of kPackRows rows, two contexts, at most
-  // kClsFirstCode class ids
+  // kClsFirstCode + kPackCodes codes
   GRID_CUDA(cudaFuncSetAttribute(k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kPackRows * 2 * ((kClsFirstCode + 31) / 32) * 4));
+                                 kPackRows * 2 * ((kClsFirstCode + kPackCodes + 31) / 32) * 4));
   GRID_CUDA(cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_succ, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
@@ -1347,11 +1364,15 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     t.root_pc = h.LN > 0 ? h.lx_pcats[0] : 0u;
     t.root_wc = h.LN > 0 ? h.lx_wcats[0] : 0u;
   }
+  // id-indexed tables are padded to Vp ids (a multiple of 4) for 4-id vector loads
+  t.Vp = (hv.V + 3) & ~3;
+  std::vector<int32_t> spell_of_id_p(hv.spell_of_id);
+  spell_of_id_p.resize(t.Vp, -1);
   if ((rc = a.upload(h.lx_cstart, &t.lx_cstart)) || (rc = a.upload(h.lx_cbyte, &t.lx_cbyte)) ||
       (rc = a.upload(h.lx_cnode, &t.lx_cnode)) || (rc = a.upload(h.lx_pcats, &t.lx_pcats)) ||
       (rc = a.upload(h.lx_wcats, &t.lx_wcats)) || (rc = a.upload(hv.spell_off, &t.spell_off)) ||
       (rc = a.upload(hv.spell_bytes, &t.spell_bytes)) || (rc = a.upload(hv.skip, &t.skip)) ||
-      (rc = a.upload(hv.spell_of_id, &t.spell_of_id)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
+      (rc = a.upload(spell_of_id_p, &t.spell_of_id)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
     return fail(rc);
   {
     std::vector<uint32_t> s16((size_t)hv.NS * 4, 0u);
@@ -1383,7 +1404,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   }
   t.n_tbl = (int)tq.size();
   t.ncls = t.ci_on ? (int)ncls : 0;
-  t.nselw = (t.ncls + 31) / 32;
+  t.nselw = (t.ncls + kPackCodes + 31) / 32;
   if ((rc = a.upload(tq, &t.tbl_q)) || (rc = a.upload(tbl_of_q, &t.tbl_of_q))) return fail(rc);
   if ((rc = set_smem_limits())) return fail(rc);
   int dev = 0;
@@ -1405,8 +1426,8 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   if ((rc = tmp.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&cls_sp)) ||
       (rc = tmp.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&key_sp)) ||
       (rc = tmp.alloc((size_t)t.n_tbl * 8, (void**)&counts_d)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.V * 2, (void**)&cls_by_id)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.V * 4, (void**)&vc_by_id)) || (rc = a.alloc((size_t)t.V, (void**)&fb)))
+      (rc = a.alloc((size_t)t.n_tbl * t.Vp * 2, (void**)&cls_by_id)) ||
+      (rc = a.alloc((size_t)t.n_tbl * t.Vp * 4, (void**)&vc_by_id)) || (rc = a.alloc((size_t)t.Vp, (void**)&fb)))
     return fail_tmp(rc);
   t.cls_by_id = cls_by_id;
   t.vc_by_id = vc_by_id;
@@ -1537,7 +1558,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     return fail_tmp(rc);
   if (nslot > 0)
     k_scatter_vc<<<(nslot + 255) / 256, 256, 0, st>>>(slot_tbl, slot_sp, slot_vc_c, nslot, t.NS, vc_sp);
-  k_permute<<<(t.V + 255) / 256, 256, 0, st>>>(t, cls_sp, vc_sp, cls_by_id, vc_by_id, fb);
+  k_permute<<<(t.Vp + 255) / 256, 256, 0, st>>>(t, cls_sp, vc_sp, cls_by_id, vc_by_id, fb);
   GRID_CUDA(cudaGetLastError());
   GRID_CUDA(cudaStreamSynchronize(st));
   tmp.release();
@@ -1670,7 +1691,7 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
                        (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
                        m.words_ns, B));
   if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
-  GRID_CUDA(launch_pdl(k_pack, dim3((t.V + 255) / 256, (B + kPackRows - 1) / kPackRows), dim3(256),
+  GRID_CUDA(launch_pdl(k_pack, dim3((t.Vp + 1023) / 1024, (B + kPackRows - 1) / kPackRows), dim3(256),
                        (size_t)kPackRows * 2 * std::max(1, t.nselw) * 4, st, t, m.ctx, (const uint32_t*)m.sel,
                        (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
                        m.words_ns, d_mask, d_status, B));
