@@ -31,7 +31,7 @@ N_BATCHES = 16
 METRIC = "cold full-vocab masks/s (batch-32 mask step at V=151,936)"
 
 
-MASK_KERNELS = ["k_prep", "k_succ", "k_filter", "k_walk", "k_pack"]
+MASK_KERNELS = ["k_row", "k_filter", "k_walk", "k_pack"]
 PROFILE = os.path.join(ROOT, "profiles", "%s_sql_select_only.md")
 SMSP_PER_SM = 4  # warp schedulers per SM, each issuing at most one warp instruction per clock
 
@@ -460,7 +460,7 @@ def main():
     #   C  events recorded by the library around each kernel of grid_masks
     # Events cost the GPU a little time each, so A carries none between steps.
     ev_b = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
-    ev_c = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    ev_c = [[torch.cuda.Event(enable_timing=True) for _ in range(len(MASK_KERNELS) + 1)] for _ in range(args.steps)]
     for ev in ev_b + ev_c:  # create each event by a first record, before the library sees its handle
         for e in ev:
             e.record(stream)

@@ -203,12 +203,12 @@ int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
 int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
                void* stream);
 
-/* Measurement hook: with n_events == 6, every later grid_masks on `c` records
- * events[0..5] (cudaEvent_t, created by the caller) on its stream before its
- * first kernel and after each of its five kernels (allowed sets and EOS gate;
- * allowed sets after the first shift and class selections; byte-walk
- * candidate filter; walk and verdict classes; id-order packing), so that
- * cudaEventElapsedTime between neighbours gives each kernel's duration.
+/* Measurement hook: with n_events == 5, every later grid_masks on `c` records
+ * events[0..4] (cudaEvent_t, created by the caller) on its stream before its
+ * first kernel and after each of its four kernels (per-row allowed sets, EOS
+ * gate, allowed sets after one shift and class selections; filtering of
+ * what the walk evaluates; walk and verdict classes; id-order packing), so
+ * that cudaEventElapsedTime between neighbours gives each kernel's duration.
  * n_events == 0 stops the recording.  The caller keeps the events alive while
  * they are set. */
 int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events);

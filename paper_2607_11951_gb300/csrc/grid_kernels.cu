@@ -16,14 +16,15 @@
 //                 by token id (coalesced in k_pack)
 //
 // Mask step (grid_masks, Def. 4):
-//   k_prep   one warp per row: A0 = A(sigma) by reduce-chain simulation; the
-//            forced emission of the pending lexeme (what every token whose first
-//            byte ends the lexeme must go through) -> sigma' and A1 = A(sigma');
-//            EOS gate (Sec. 3.2); the first bytes that end the lexeme; for rows
-//            without a table, the live first-byte ranges that continue it
-//   k_succ   per row, context and allowed terminal tau: the allowed set after
-//            shifting tau (walks simulate nothing before their second shift);
-//            the class selections of both contexts
+//   k_row    one block per row: A0 = A(sigma) by a set simulation of the reduce
+//            chains; in parallel the forced emission of the pending lexeme
+//            (what every token whose first byte ends the lexeme must go
+//            through) -> sigma' and A1 = A(sigma'), and the EOS gate (Sec. 3.2);
+//            the first bytes that end the lexeme; for rows without a table,
+//            the live first-byte ranges that continue it; then per context and
+//            allowed terminal tau the allowed set after shifting tau (walks
+//            simulate nothing before their second shift) and the class
+//            selections
 //   k_filter per row and context: the byte-walked spellings and the verdict
 //            classes whose first stack-dependent emission can succeed
 //   k_walk   persistent; per row: each surviving verdict class evaluated once
@@ -56,12 +57,13 @@ namespace {
 
 constexpr int kWalkWarps = 8;    // warps per k_walk block
 constexpr int kSpan = 32;        // CD list entries per walk item (one warp batch)
-constexpr int kPrepWarps = 4;    // rows per k_prep block
-constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_prep/k_advance
+constexpr int kPrepWarps = 4;    // rows per k_advance block
+constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_row/k_advance
 constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
-constexpr int kSuccJobWarps = 4;  // k_succ: warps of lanes, one terminal each (covers 128 terminals)
+constexpr int kRowWarps = 6;     // k_row: warps per row block
+constexpr int kRowJobWarps = 4;  // k_row: warps 2 .. 5 compute the allowed sets after one shift
 // Class codes as k_pack reads them: CI class ids 0..ncls-1, then these five
 // (so that one bit test of the row's class selection covers CI, always and
 // never, and only verdict-class and walked tokens need a second lookup).
@@ -288,25 +290,40 @@ __device__ Bits4 allowed_set(const Tables& t, const uint16_t* base, int keep, co
   return Bits4{wds[0], wds[1], wds[2], wds[3]};
 }
 
-__global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
-                                                          RowRanges* __restrict__ rng, uint32_t* __restrict__ verd0,
-                                                          uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
-                                                          int n_vcbits, int B, int words_ns) {
+// One block per row (kRowWarps warps), plus clearing blocks after the rows.
+// Phase 1, three warps at once: warp 0 computes A0 = A(sigma) and then the
+// live first-byte ranges that continue the pending lexeme (rows without a CI
+// table); warp 1 makes the forced emission of the pending lexeme (sigma ->
+// sigma', what every token whose first byte ends the lexeme must go through),
+// the EOS gate (Sec. 3.2) and A1 = A(sigma'); warp 2 finds the first bytes
+// that end the lexeme.  Phase 2: for both contexts, lanes of the job warps
+// take one allowed terminal tau each and compute the allowed set after tau's
+// reduce chain and shift (A2: walks and verdict classes simulate nothing
+// before their second shift); warps 0 and 1 select the contexts' CI classes.
+// Clearing blocks zero both verdict bitmaps and the verdict-class bits.
+__global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
+                                                        RowRanges* __restrict__ rng, uint32_t* __restrict__ A2,
+                                                        uint32_t* __restrict__ sel, uint32_t* __restrict__ verd0,
+                                                        uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
+                                                        int n_vcbits, int B, int words_ns) {
   extern __shared__ __align__(16) uint8_t smem[];
-  __shared__ uint16_t s_ovl[kPrepWarps][kMaxOvl];
-  __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
-  __shared__ uint16_t s_scr[kPrepWarps][kMaxOvl * 32];
-  __shared__ uint32_t s_A0[kPrepWarps][4];
-  __shared__ int s_km[kPrepWarps][3];
-  __shared__ uint32_t s_keep[kPrepWarps][8];
-  const int row_blocks = (B + kPrepWarps - 1) / kPrepWarps;
-  if ((int)blockIdx.x >= row_blocks) {
+  __shared__ Tables ts;
+  __shared__ uint16_t s_stk[kStackWin];
+  __shared__ uint16_t s_ovl1[kMaxOvl];
+  __shared__ uint16_t s_ovl2[kRowJobWarps][kMaxOvl * 32];
+  __shared__ uint16_t s_scr[kRowJobWarps][kMaxOvl * 32];
+  __shared__ uint16_t s_scr01[2][kMaxOvl];
+  __shared__ uint32_t s_A0[4], s_A1[4], s_keep[8], s_kill[8];
+  __shared__ int s_row[8];  // complete, depth, q, lx, emit_ok, keep1, m1, eos_ok | sigma'==sigma << 1
+  __shared__ uint32_t s_pc[2];
+  __shared__ int s_status, s_total0, s_nrng;
+  if ((int)blockIdx.x >= B) {
     // clearing blocks: zero both verdict bitmaps and the verdict-class bits of every row
     pdl_wait();
     const size_t n = (size_t)B * words_ns;
     const size_t n4 = n >> 2;
-    const size_t stride = (size_t)(gridDim.x - row_blocks) * blockDim.x;
-    const size_t first = (size_t)(blockIdx.x - row_blocks) * blockDim.x + threadIdx.x;
+    const size_t stride = (size_t)(gridDim.x - B) * blockDim.x;
+    const size_t first = (size_t)(blockIdx.x - B) * blockDim.x + threadIdx.x;
     const uint4 z = make_uint4(0u, 0u, 0u, 0u);
     for (size_t i = first; i < n4; i += stride) {
       reinterpret_cast<uint4*>(verd0)[i] = z;
@@ -319,154 +336,168 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     for (size_t i = first; i < (size_t)n_vcbits; i += stride) vcbits[i] = 0u;
     return;
   }
-  __shared__ Tables ts;
   stage_tables(t, ts, smem);
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int b = blockIdx.x * kPrepWarps + warp;
-  if (b >= B) return;
+  const int b = blockIdx.x;
   RowCtx& r = ctx[b];
-  const int complete = c.flags[b] & 1;
-  const uint16_t* gbase = c.stack + (size_t)b * t.D;
-  const int depth = c.depth[b], q = c.q[b], lx = c.lx[b];
-  const uint32_t pc0 = lx >= 0 ? t.lx_pcats[lx] : 0u, wc0 = lx >= 0 ? t.lx_wcats[lx] : 0u;
-  const uint16_t* base = gbase;
+  if (threadIdx.x == 0) {
+    const int lx = c.lx[b];
+    s_row[0] = c.flags[b] & 1;
+    s_row[1] = c.depth[b];
+    s_row[2] = c.q[b];
+    s_row[3] = lx;
+    s_pc[0] = lx >= 0 ? t.lx_pcats[lx] : 0u;
+    s_pc[1] = lx >= 0 ? t.lx_wcats[lx] : 0u;
+    s_status = GRID_ST_OK;
+    s_total0 = 0;
+    s_nrng = 0;
+  }
+  __syncthreads();
+  const int complete = s_row[0], depth = s_row[1], q = s_row[2], lx = s_row[3];
+  const uint32_t pc0 = s_pc[0], wc0 = s_pc[1];
+  const uint16_t* base = c.stack + (size_t)b * t.D;
   if (depth <= kStackWin) {  // the reduce chains below read the stack top repeatedly
-    for (int i = lane; i < depth; i += 32) s_stk[warp][i] = gbase[i];
-    __syncwarp();
-    base = s_stk[warp];
+    for (int i = threadIdx.x; i < depth; i += blockDim.x) s_stk[i] = base[i];
+    base = s_stk;
   }
+  __syncthreads();
   const int mc = max_chain_of(t);
-  int status = complete ? GRID_ST_COMPLETE : GRID_ST_OK;
-  Bits4 A0 = Bits4::zero(), A1 = Bits4::zero();
-  const LArr scr{s_scr[warp] + lane, 32};
-  if (!complete) A0 = allowed_set(ts, base, depth, nullptr, 0, status, lane, scr);
-  if (lane == 0) {
-    s_A0[warp][0] = A0.x;
-    s_A0[warp][1] = A0.y;
-    s_A0[warp][2] = A0.z;
-    s_A0[warp][3] = A0.w;
-  }
-  __syncwarp();
-  // forced emission of the pending lexeme + EOS gate (lane 0)
-  if (lane == 0) {
+  const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
+  int status = GRID_ST_OK;
+  // ---- phase 1
+  if (warp == 0) {
+    Bits4 A0 = Bits4::zero();
+    if (!complete) A0 = allowed_set(ts, base, depth, nullptr, 0, status, lane, LArr{s_scr01[0], 1});
+    if (lane < 4) s_A0[lane] = A0.word(lane);
+    // continuing first-byte ranges (rows without a CI table for q).  A first
+    // byte whose lexeme has no live terminal in A0 u I (category terminals
+    // counted only while the lexeme is a prefix of one of their words)
+    // rejects every spelling it starts: liveness only shrinks along the
+    // lexeme, and any later emission picks among its live terminals.
+    if (!complete && q != kStart && tbl0 < 0) {
+      int total0 = 0, nrng = 0;
+      RowRanges& R = rng[b];
+      const Bits4 AI = A0 | ts.ign;
+      int lo_r[8], hi_r[8];
+      uint32_t cw[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        lo_r[j] = t.first_of_byte[j * 32 + lane];
+        hi_r[j] = t.first_of_byte[j * 32 + lane + 1];
+      }
+      int nc = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int by = j * 32 + lane;
+        cw[j] = __ballot_sync(0xffffffffu, hi_r[j] > lo_r[j] && ts.next[q * ts.C + ts.byte_class[by]] != kDead);
+        nc += __popc(cw[j]);
+      }
+      if (lane < 8) s_keep[lane] = 0u;
+      __syncwarp();
+      for (int i0 = 0; i0 < nc; i0 += 32) {  // the live test of the continuing bytes, one per lane
+        int idx = i0 + lane, by = -1;
+        if (idx < nc) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int cnt = __popc(cw[j]);
+            if (by < 0 && idx < cnt) by = j * 32 + (int)__fns(cw[j], 0u, idx + 1);
+            if (by < 0) idx -= cnt;
+          }
+        }
+        if (by >= 0) {
+          uint32_t pc2 = 0u, wc2 = 0u;
+          if (lx >= 0) lex_step(ts, lx, by, pc2, wc2);
+          const int q2 = ts.next[q * ts.C + ts.byte_class[by]];
+          if ((live_prime(ts, q2, pc2) & AI).any()) atomicOr(&s_keep[by >> 5], 1u << (by & 31));
+        }
+      }
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const bool cont = (s_keep[j] >> lane) & 1u;
+        const int chunks = cont ? (hi_r[j] - lo_r[j] + kRangeSpan - 1) / kRangeSpan : 0;
+        const uint32_t bal = __ballot_sync(0xffffffffu, cont);
+        int incl = chunks;
+        for (int d = 1; d < 32; d <<= 1) {
+          int v = __shfl_up_sync(0xffffffffu, incl, d);
+          if (lane >= d) incl += v;
+        }
+        if (cont) {
+          const int k = nrng + __popc(bal & ((1u << lane) - 1u));
+          R.lo[k] = lo_r[j];
+          R.hi[k] = hi_r[j];
+          R.cpre[k] = total0 + incl - chunks;
+        }
+        total0 += __shfl_sync(0xffffffffu, incl, 31);
+        nrng += __popc(bal);
+      }
+      if (lane == 0) {
+        R.cpre[nrng] = total0;
+        s_total0 = total0;
+        s_nrng = nrng;
+      }
+    }
+  } else if (warp == 1) {
+    // forced emission of the pending lexeme, EOS gate, A1
     int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
-    if (!complete) {
+    if (lane == 0 && !complete) {
       Walker w;
       uint16_t lo[kMaxOvl], ls[kMaxOvl];
-      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, s_A0[warp], nullptr);
+      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, nullptr, nullptr);
       if (q == kStart) {
         emit_ok = 1;
       } else {
-        int e = emit(ts, w, mc);
+        const int e = emit(ts, w, mc);
         if (e < 0) status = GRID_ST_BOUND;
         emit_ok = e > 0;
         keep1 = w.keep;
         m1 = w.m;
-        for (int i = 0; i < m1; ++i) s_ovl[warp][i] = w.ovl[i];
+        for (int i = 0; i < m1; ++i) s_ovl1[i] = w.ovl[i];
       }
       Walker w2;
-      walker_init(w2, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, s_A0[warp], nullptr);
-      int g = eos_gate(ts, w2, mc);
+      walker_init(w2, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, nullptr, nullptr);
+      const int g = eos_gate(ts, w2, mc);
       if (g < 0) status = GRID_ST_BOUND;
       eos = g > 0;
     }
-    s_km[warp][0] = emit_ok;
-    s_km[warp][1] = keep1;
-    s_km[warp][2] = m1;
-    r.eos_ok = eos;
-  }
-  __syncwarp();
-  const int emit_ok = s_km[warp][0], keep1 = s_km[warp][1], m1 = s_km[warp][2];
-  if (!complete && emit_ok) {
-    if (keep1 == depth && m1 == 0)
-      A1 = A0;
-    else
-      A1 = allowed_set(ts, base, keep1, s_ovl[warp], m1, status, lane, scr);
+    emit_ok = __shfl_sync(0xffffffffu, emit_ok, 0);
+    keep1 = __shfl_sync(0xffffffffu, keep1, 0);
+    m1 = __shfl_sync(0xffffffffu, m1, 0);
+    __syncwarp();
+    Bits4 A1 = Bits4::zero();
+    const bool same = keep1 == depth && m1 == 0;  // sigma' = sigma: A1 = A0, taken after the barrier
+    if (!complete && emit_ok && !same) A1 = allowed_set(ts, base, keep1, s_ovl1, m1, status, lane, LArr{s_scr01[1], 1});
+    if (lane < 4) s_A1[lane] = A1.word(lane);
+    if (lane == 0) {
+      s_row[4] = emit_ok;
+      s_row[5] = keep1;
+      s_row[6] = m1;
+      s_row[7] = eos | (same ? 2 : 0);
+    }
+  } else if (warp == 2) {
+    // first bytes that end the pending lexeme (every byte when it is empty)
+    for (int b0 = 0; b0 < 256; b0 += 32) {
+      const int by = b0 + lane;
+      const bool kill = q == kStart || ts.next[q * ts.C + ts.byte_class[by]] == kDead;
+      const uint32_t word = __ballot_sync(0xffffffffu, kill);
+      if (lane == 0) s_kill[b0 >> 5] = word;
+    }
   }
   status = __reduce_max_sync(0xffffffffu, status);
-  const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
-  // continuing first-byte ranges (rows without a CI table for q).  A first
-  // byte whose lexeme has no live terminal in A0 u I (category terminals
-  // counted only while the lexeme is a prefix of one of their words) rejects
-  // every spelling it starts: liveness only shrinks along the lexeme, and any
-  // later emission picks among its live terminals.
-  int total0 = 0, nrng = 0;
-  if (!complete && q != kStart && tbl0 < 0) {
-    RowRanges& R = rng[b];
-    const Bits4 AI = A0 | ts.ign;
-    int lo_r[8], hi_r[8];
-    uint32_t cw[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      lo_r[j] = t.first_of_byte[j * 32 + lane];
-      hi_r[j] = t.first_of_byte[j * 32 + lane + 1];
+  if (lane == 0 && status != GRID_ST_OK) atomicMax(&s_status, status);
+  __syncthreads();
+  const int emit_ok = s_row[4], keep1 = s_row[5], m1 = s_row[6];
+  if (threadIdx.x < 4 && (s_row[7] & 2) && emit_ok && !complete) s_A1[threadIdx.x] = s_A0[threadIdx.x];
+  __syncthreads();
+  const Bits4 A0 = Bits4::load(s_A0), A1 = Bits4::load(s_A1);
+  // ---- the row's context for the later kernels
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < 4; ++k) {
+      r.A0[k] = s_A0[k];
+      r.A1[k] = s_A1[k];
     }
-    int nc = 0;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int by = j * 32 + lane;
-      cw[j] = __ballot_sync(0xffffffffu, hi_r[j] > lo_r[j] && ts.next[q * ts.C + ts.byte_class[by]] != kDead);
-      nc += __popc(cw[j]);
-    }
-    // the live test of the continuing bytes, one byte per lane
-    if (lane < 8) s_keep[warp][lane] = 0u;
-    __syncwarp();
-    for (int i0 = 0; i0 < nc; i0 += 32) {
-      int idx = i0 + lane, by = -1;
-      if (idx < nc) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int cnt = __popc(cw[j]);
-          if (by < 0 && idx < cnt) by = j * 32 + (int)__fns(cw[j], 0u, idx + 1);
-          if (by < 0) idx -= cnt;
-        }
-      }
-      if (by >= 0) {
-        uint32_t pc2 = 0u, wc2 = 0u;
-        if (lx >= 0) lex_step(ts, lx, by, pc2, wc2);
-        const int q2 = ts.next[q * ts.C + ts.byte_class[by]];
-        if ((live_prime(ts, q2, pc2) & AI).any()) atomicOr(&s_keep[warp][by >> 5], 1u << (by & 31));
-      }
-    }
-    __syncwarp();
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const bool cont = (s_keep[warp][j] >> lane) & 1u;
-      const int chunks = cont ? (hi_r[j] - lo_r[j] + kRangeSpan - 1) / kRangeSpan : 0;
-      const uint32_t bal = __ballot_sync(0xffffffffu, cont);
-      int incl = chunks;
-      for (int d = 1; d < 32; d <<= 1) {
-        int v = __shfl_up_sync(0xffffffffu, incl, d);
-        if (lane >= d) incl += v;
-      }
-      if (cont) {
-        const int k = nrng + __popc(bal & ((1u << lane) - 1u));
-        R.lo[k] = lo_r[j];
-        R.hi[k] = hi_r[j];
-        R.cpre[k] = total0 + incl - chunks;
-      }
-      total0 += __shfl_sync(0xffffffffu, incl, 31);
-      nrng += __popc(bal);
-    }
-    if (lane == 0) R.cpre[nrng] = total0;
-  }
-  // first bytes that end the pending lexeme (every byte when it is empty)
-  for (int b0 = 0; b0 < 256; b0 += 32) {
-    const int by = b0 + lane;
-    const bool kill = q == kStart || ts.next[q * ts.C + ts.byte_class[by]] == kDead;
-    const uint32_t word = __ballot_sync(0xffffffffu, kill);
-    if (lane == 0) r.kill[b0 >> 5] = word;
-  }
-  if (lane == 0) {
-    r.A0[0] = A0.x;
-    r.A0[1] = A0.y;
-    r.A0[2] = A0.z;
-    r.A0[3] = A0.w;
-    r.A1[0] = A1.x;
-    r.A1[1] = A1.y;
-    r.A1[2] = A1.z;
-    r.A1[3] = A1.w;
+    for (int k = 0; k < 8; ++k) r.kill[k] = s_kill[k];
     r.q = q;
     r.lx = lx;
     r.pc0 = pc0;
@@ -474,91 +505,71 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_prep(Tables t, DevConfigs c
     r.depth = depth;
     r.tbl0 = tbl0;
     r.emit_ok = emit_ok;
-    r.status = status;
+    r.eos_ok = s_row[7] & 1;
     r.complete = complete;
     r.nonempty = 0;
     r.done_blocks = 0;
     r.keep1 = keep1;
     r.m1 = m1;
     r.work0 = 0;
-    r.nrange = total0;
+    r.nrange = s_total0;
     r.nsurv[0] = 0;
     r.nsurv[1] = 0;
     r.nvs[0] = 0;
     r.nvs[1] = 0;
-    r.nrng = nrng;
+    r.nrng = s_nrng;
   }
-  for (int i = lane; i < m1; i += 32) r.ovl1[i] = s_ovl[warp][i];
-}
-
-
-// grid = (B, 2): row b, context cx (0: sigma, 1: sigma' after the forced
-// emission).  Warps 0..kSuccJobWarps-1: lane l of warp w takes terminal
-// tau = 32 w + l if tau is allowed in the context and computes the allowed set
-// after tau's reduce chain and shift (A2) with one set simulation, so that a
-// walk or verdict-class evaluation simulates nothing before its second shift.
-// The last warp: the context's CI class selection.
-__global__ void __launch_bounds__((kSuccJobWarps + 1) * 32) k_succ(Tables t, DevConfigs c,
-                                                                    const RowCtx* __restrict__ ctx,
-                                                                    uint32_t* __restrict__ A2,
-                                                                    uint32_t* __restrict__ sel) {
-  extern __shared__ __align__(16) uint8_t smem[];
-  __shared__ Tables ts;
-  __shared__ uint16_t s_win[kWalkWin];
-  __shared__ uint16_t s_ovl1[kMaxOvl];
-  __shared__ uint16_t s_ovl2[kSuccJobWarps][kMaxOvl * 32];
-  __shared__ uint16_t s_scr[kSuccJobWarps][kMaxOvl * 32];
-  const int b = blockIdx.x, cx = blockIdx.y;
-  stage_tables(t, ts, smem);
-  pdl_wait();
-  const RowCtx& r = ctx[b];
-  if (r.complete || (cx == 1 && !r.emit_ok) || (cx == 0 && r.q == kStart)) return;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int depth = r.depth;
-  const uint16_t* base = c.stack + (size_t)b * t.D;
-  const int m = cx ? r.m1 : 0;
-  for (int i = threadIdx.x; i < m; i += blockDim.x) s_ovl1[i] = r.ovl1[i];
-  if (depth <= kWalkWin) {
-    for (int i = threadIdx.x; i < depth; i += blockDim.x) s_win[i] = base[i];
-    base = s_win;
-  }
-  __syncthreads();
-  const int keep = cx ? r.keep1 : depth;
-  const Bits4 A = Bits4::load(cx ? r.A1 : r.A0);
-  if (warp == kSuccJobWarps) {
-    if (t.ci_on && (cx == 1 || r.tbl0 >= 0)) select_classes(ts, A, sel + ((size_t)b * 2 + cx) * t.nselw, lane);
-    return;
-  }
-  const int mc = max_chain_of(t);
-  const int tau = warp * 32 + lane;
-  int status = GRID_ST_OK;
-  if (tau < t.n_term && A.has(tau)) {
-    const LArr scr{s_scr[warp] + lane, 32}, ovl2{s_ovl2[warp] + lane, 32};
-    int keep_o, m_o, ns;
-    const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
-    Bits4 An = Bits4::zero();
-    if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
-      for (int i = 0; i < m_o; ++i) ovl2[i] = s_ovl1[i];
-      for (int i = 0; i < ns; ++i) ovl2[m_o + i] = scr[i];
-      ovl2[m_o + ns] = (uint16_t)(a - 1);
+  for (int i = threadIdx.x; i < m1; i += blockDim.x) r.ovl1[i] = s_ovl1[i];
+  // ---- phase 2
+  status = GRID_ST_OK;
+  if (!complete) {
+    if (warp >= 2) {
+      // A2 of the allowed terminals: the first half of the job warps for
+      // sigma, the second half for sigma'
+      const int half = kRowJobWarps / 2;
+      const int cx = warp - 2 >= half ? 1 : 0;
+      const int jw = warp - 2 - cx * half;
+      const bool has_ctx = cx ? (emit_ok != 0) : (q != kStart);
+      const Bits4 A = cx ? A1 : A0;
+      const int keep = cx ? keep1 : depth, m = cx ? m1 : 0;
+      const LArr scr{s_scr[warp - 2] + lane, 32}, ovl2{s_ovl2[warp - 2] + lane, 32};
       Bits4 G = Bits4::zero();
       for (int k = 0; k < t.n_term; ++k) G.set(k);
       G = G.andnot(ts.ign);
-      bool bound = false;
-      An = simulate_set(ts, base, keep_o, ovl2, m_o + ns + 1, G, scr, kMaxOvl, mc, bound);
-      if (bound) status = GRID_ST_BOUND;
-    } else {
-      status = GRID_ST_BOUND;
+      for (int tau = jw * 32 + lane; has_ctx && tau < t.n_term; tau += 32 * half) {
+        if (!A.has(tau)) continue;
+        int keep_o, m_o, ns;
+        const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
+        Bits4 An = Bits4::zero();
+        if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
+          for (int i = 0; i < m_o; ++i) ovl2[i] = s_ovl1[i];
+          for (int i = 0; i < ns; ++i) ovl2[m_o + i] = scr[i];
+          ovl2[m_o + ns] = (uint16_t)(a - 1);
+          bool bound = false;
+          An = simulate_set(ts, base, keep_o, ovl2, m_o + ns + 1, G, scr, kMaxOvl, mc, bound);
+          if (bound) status = GRID_ST_BOUND;
+        } else {
+          status = GRID_ST_BOUND;
+        }
+        uint32_t* out = A2 + (((size_t)b * 2 + cx) * t.T1 + tau) * 4;
+        out[0] = An.x;
+        out[1] = An.y;
+        out[2] = An.z;
+        out[3] = An.w;
+      }
+    } else if (t.ci_on) {
+      // class selections: warp 0 for sigma (rows with a table), warp 1 for sigma'
+      if (warp == 0 && tbl0 >= 0) select_classes(ts, A0, sel + ((size_t)b * 2) * t.nselw, lane);
+      if (warp == 1 && emit_ok) select_classes(ts, A1, sel + ((size_t)b * 2 + 1) * t.nselw, lane);
     }
-    uint32_t* out = A2 + (((size_t)b * 2 + cx) * t.T1 + tau) * 4;
-    out[0] = An.x;
-    out[1] = An.y;
-    out[2] = An.z;
-    out[3] = An.w;
   }
   status = __reduce_max_sync(0xffffffffu, status);
-  if (lane == 0 && status != GRID_ST_OK) atomicCAS(const_cast<int32_t*>(&ctx[b].status), GRID_ST_OK, status);
+  if (lane == 0 && status != GRID_ST_OK) atomicMax(&s_status, status);
+  __syncthreads();
+  if (threadIdx.x == 0) r.status = complete ? GRID_ST_COMPLETE : s_status;
 }
+
+
 
 // grid = (cd_blocks + vc_blocks, B, 2), 256 threads: compact, per row and
 // context, what the walk has to evaluate.
@@ -656,7 +667,7 @@ __device__ __forceinline__ int4 row_queue(const Tables& t, const RowCtx& x) {
 //
 // Verdict-class items: 32 of the records that k_filter kept for the row and
 // context, one per lane, each evaluated once against the row's stack; an
-// accepted record sets its bit in vcbits (cleared by k_prep), which k_pack
+// accepted record sets its bit in vcbits (cleared by k_row), which k_pack
 // reads back per token id.
 // List items (kSpan CD spellings): a spelling is walked only if the class of
 // its first stack-dependent emission is selected for the context's allowed
@@ -903,7 +914,7 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   }
   for (int i = threadIdx.x; i < nr * 8; i += blockDim.x) s_kill[i >> 3][i & 7] = ctx[r0 + (i >> 3)].kill[i & 7];
   __syncthreads();
-  // class selections; a context that k_succ did not select for (a completed
+  // class selections; a context that k_row did not select for (a completed
   // row, sigma' without a forced emission, sigma without a table) reads zeros
   for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) {
     const int k = i / (2 * nw), cx = (i / nw) & 1;
@@ -1208,7 +1219,7 @@ struct grid_spec {
   int max_vc = 0;       // verdict classes of the largest table
 };
 
-constexpr int kMaskKernels = 5;  // k_prep, k_succ, k_filter, k_walk, k_pack
+constexpr int kMaskKernels = 4;  // k_row, k_filter, k_walk, k_pack
 
 struct grid_configs {
   int B = 0, D = 0, words_ns = 0;
@@ -1238,9 +1249,8 @@ static int set_smem_limits() {
   // kClsFirstCode + kPackCodes codes
   GRID_CUDA(cudaFuncSetAttribute(k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kPackRows * 2 * ((kClsFirstCode + kPackCodes + 31) / 32) * 4));
-  GRID_CUDA(cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
-  GRID_CUDA(cudaFuncSetAttribute(k_succ, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   return GRID_OK;
 }
@@ -1673,29 +1683,26 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
   const int vcw = std::max(1, s->vcw);
   const int n_vcbits = B * 2 * vcw;
   const size_t zero_words = (size_t)B * m.words_ns * 2 + n_vcbits;
-  const int zero_blocks = std::min(128, (int)((zero_words / 8 + 1023) / 1024) + 1);
+  const int zero_blocks = std::min(128, (int)((zero_words / 8 + kRowWarps * 32 * 4 - 1) / (kRowWarps * 32 * 4)) + 1);
   if (ev) GRID_CUDA(cudaEventRecord(ev[0], st));
-  GRID_CUDA(launch_pdl(k_prep, dim3((B + kPrepWarps - 1) / kPrepWarps + zero_blocks), dim3(kPrepWarps * 32),
-                       t.blob_bytes, st, t, c, m.ctx, m.rng, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns));
+  GRID_CUDA(launch_pdl(k_row, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx, m.rng,
+                       m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
-  GRID_CUDA(launch_pdl(k_succ, dim3(B, 2), dim3((kSuccJobWarps + 1) * 32), t.blob_bytes, st, t, c,
-                       (const RowCtx*)m.ctx, m.A2, m.sel));
-  if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
   const int cd_blocks = (s->max_cd + 255) / 256;
   const int vc_blocks = (s->max_vc + 255) / 256;
   GRID_CUDA(launch_pdl(k_filter, dim3(std::max(1, cd_blocks + vc_blocks), B, 2), dim3(256), 0, st, t, m.ctx,
                        (const uint32_t*)m.sel, m.surv, m.cap, m.vsurv, m.vcap, cd_blocks));
-  if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
+  if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
   GRID_CUDA(launch_pdl(k_walk, dim3(s->walk_blocks), dim3(kWalkWarps * 32), t.blob_bytes, st, t, m.ctx,
                        (const RowRanges*)m.rng, (const uint16_t*)c.stack, (const int32_t*)m.surv, m.cap,
                        (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
                        m.words_ns, B));
-  if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
+  if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
   GRID_CUDA(launch_pdl(k_pack, dim3((t.Vp + 1023) / 1024, (B + kPackRows - 1) / kPackRows), dim3(256),
                        (size_t)kPackRows * 2 * std::max(1, t.nselw) * 4, st, t, m.ctx, (const uint32_t*)m.sel,
                        (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
                        m.words_ns, d_mask, d_status, B));
-  if (ev) GRID_CUDA(cudaEventRecord(ev[5], st));
+  if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
@@ -1710,7 +1717,7 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
 
 extern "C" int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events) {
   if (!c || (n_events != 0 && n_events != kMaskKernels + 1) || (n_events && !events))
-    return set_error(GRID_E_INVALID_ARG, "grid_configs_set_events: pass 0 or 6 events");
+    return set_error(GRID_E_INVALID_ARG, "grid_configs_set_events: pass 0 or 5 events");
   for (int i = 0; i <= kMaskKernels; ++i) {
     c->ev[i] = n_events ? static_cast<cudaEvent_t>(events[i]) : nullptr;
     if (n_events && !c->ev[i]) {
@@ -1826,7 +1833,7 @@ extern "C" int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, co
   const DevConfigs c{const_cast<uint16_t*>(d_stack), const_cast<int32_t*>(d_depth),
                      const_cast<int32_t*>(d_dfa_state), const_cast<int32_t*>(d_lex_node),
                      const_cast<int32_t*>(d_flags)};
-  // What must start at zero is cleared by k_prep itself on every call: the
+  // What must start at zero is cleared by k_row itself on every call: the
   // verdict bitmaps and verdict-class bits (its clearing blocks) and each
   // row's queue, survivor and completion counters.  The other buffers are
   // written before they are read within the call, so the previous call's

@@ -213,7 +213,7 @@ def grid_masks(spec, cfg, mask, status, stream=None):
 
 
 def grid_configs_set_events(cfg, events):
-    """events: 6 torch.cuda.Event(enable_timing=True) recorded around the five
+    """events: 5 torch.cuda.Event(enable_timing=True) recorded around the four
     kernels of every later grid_masks on cfg; an empty list stops it."""
     arr = (ctypes.c_void_p * max(1, len(events)))(*[e.cuda_event for e in events])
     _check(lib().grid_configs_set_events(cfg, ctypes.cast(arr, ctypes.c_void_p), len(events)))
