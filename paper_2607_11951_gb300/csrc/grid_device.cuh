@@ -98,7 +98,7 @@ struct Tables {
   const uint16_t* plhs;
   const uint32_t* shift_mask;  // S * 4: terminals whose action is SHIFT
   const uint32_t* red_off;     // S + 1: reduce groups of state s are red_off[s] .. red_off[s+1]
-  const uint16_t* red_p;       // production of each reduce group
+  const uint16_t* red_p;       // each reduce group's production as plen << 10 | lhs
   const uint32_t* red_mask;    // 4 per reduce group: its lookahead terminals
   // identifier trie
   const int32_t* lx_cstart;
@@ -276,18 +276,18 @@ __device__ __forceinline__ int simulate(const Tables& t, const uint16_t* base, i
                                         LArr scr, int cap, int& keep_o, int& m_o, int& ns, int max_chain) {
   int k = keep, mm = m;
   ns = 0;
+  int top = mm ? ovl[mm - 1] : base[k - 1];
   for (int it = 0; it < max_chain; ++it) {
-    int top = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
     if (top >= t.S) return 0;
-    int a = t.action[top * t.T1 + tau];
+    const int a = t.action[top * t.T1 + tau];
     if (a == 0) return 0;
     if (a > 0) {
       keep_o = k;
       m_o = mm;
       return a;
     }
-    int p = -a - 1;
-    int n = t.plen[p];
+    const int code = -a - 1;  // plen << 10 | lhs
+    int n = code >> 10;
     int x = min(n, ns);
     ns -= x;
     n -= x;
@@ -296,10 +296,11 @@ __device__ __forceinline__ int simulate(const Tables& t, const uint16_t* base, i
     n -= x;
     k -= n;
     if (k < 1) return 0;
-    int top2 = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
+    const int top2 = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
     if (top2 >= t.S) return 0;
     if (ns >= cap) return -1;
-    scr[ns++] = t.go[top2 * t.NNT + t.plhs[p]];
+    top = t.go[top2 * t.NNT + (code & 1023)];
+    scr[ns++] = (uint16_t)top;
   }
   return -1;
 }
@@ -323,8 +324,8 @@ __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* b
     todo = Bits4::zero();
     int k = keep, mm = m, ns = 0;
     int it = 0;
+    int top = mm ? ovl[mm - 1] : base[k - 1];
     for (; it < max_chain && g.any(); ++it) {
-      const int top = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
       if (top >= t.S) break;
       const Bits4 sh = Bits4::load(t.shift_mask + top * 4);
       res = res | (g & sh);
@@ -344,7 +345,7 @@ __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* b
       }
       if (p < 0) break;  // the rest is an error here
       g = gp;
-      int n = t.plen[p];
+      int n = p >> 10;  // p: plen << 10 | lhs
       int x = min(n, ns);
       ns -= x;
       n -= x;
@@ -359,7 +360,8 @@ __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* b
         bound = true;
         return res;
       }
-      scr[ns++] = t.go[top2 * t.NNT + t.plhs[p]];
+      top = t.go[top2 * t.NNT + (p & 1023)];
+      scr[ns++] = (uint16_t)top;
     }
     if (it == max_chain && g.any()) {
       bound = true;

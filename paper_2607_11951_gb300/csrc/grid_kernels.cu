@@ -1291,6 +1291,18 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   // per LALR state: the terminals that shift, and the terminals grouped by
   // the production they reduce by (for simulating a set of terminals at once)
   std::vector<uint32_t> shift_mask((size_t)h.S * 4, 0u), red_mask;
+  // reduce actions carry their production's length and left-hand side
+  // (-(1 + (plen << 10 | lhs))), so that a reduce step needs no second lookup
+  int max_plen = 0;
+  for (int pr = 0; pr < h.P; ++pr) max_plen = std::max(max_plen, (int)h.plen[pr]);
+  if (h.NNT >= 1024 || max_plen >= 32)
+    return fail(set_error(GRID_E_TOO_LARGE, "grammar exceeds the packed reduce encoding (1024 nonterminals, "
+                                            "right-hand sides of 31 symbols)"));
+  std::vector<int16_t> action16(h.action.size());
+  for (size_t i = 0; i < h.action.size(); ++i) {
+    const int a = h.action[i];
+    action16[i] = a >= 0 ? (int16_t)a : (int16_t)(-(1 + ((h.plen[-a - 1] << 10) | h.plhs[-a - 1])));
+  }
   std::vector<uint32_t> red_off(h.S + 1, 0);
   std::vector<uint16_t> red_p;
   for (int st = 0; st < h.S; ++st) {
@@ -1310,7 +1322,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
       }
     }
     for (const auto& g : groups) {
-      red_p.push_back((uint16_t)g.first);
+      red_p.push_back((uint16_t)((h.plen[g.first] << 10) | h.plhs[g.first]));
       for (int w = 0; w < 4; ++w) red_mask.push_back(g.second[w]);
     }
     red_off[st + 1] = (uint32_t)red_p.size();
@@ -1322,7 +1334,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   const size_t sizes[kSec] = {256, h.next.size() * 2, h.acc.size() * 4, h.live.size() * 4, h.action.size() * 2,
                               h.go.size() * 2, h.plen.size(), h.plhs.size() * 2, shift_mask.size() * 4,
                               red_off.size() * 4, red_p.size() * 2, red_mask.size() * 4};
-  const void* srcs[kSec] = {h.byte_class, h.next.data(), h.acc.data(), h.live.data(), h.action.data(),
+  const void* srcs[kSec] = {h.byte_class, h.next.data(), h.acc.data(), h.live.data(), action16.data(),
                             h.go.data(), h.plen.data(), h.plhs.data(), shift_mask.data(), red_off.data(),
                             red_p.data(), red_mask.data()};
   for (int k = 0; k < kSec; ++k) off[k + 1] = align16(off[k] + sizes[k]);
