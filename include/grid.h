@@ -248,8 +248,8 @@ int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, const int32_t
 /* Sec. 2 masked decoding: for b < B, t < V, set d_logits[b*row_stride + t] to
  * -inf (fp32 0xFF800000 / bf16 0xFF80) where mask bit t of row b is 0; accepted
  * values are left bit-identical.  d_logits is device memory of `dtype`
- * (GRID_DTYPE_F32 or GRID_DTYPE_BF16); row_stride >= V elements.  In place,
- * enqueue only. */
+ * (GRID_DTYPE_F32 or GRID_DTYPE_BF16); row_stride >= V elements; B <= 65535
+ * (GRID_E_TOO_LARGE above).  In place, enqueue only. */
 int grid_apply_mask(const uint32_t* d_mask, void* d_logits, int32_t dtype, int32_t B, int32_t V,
                     int64_t row_stride, void* stream);
 

@@ -1099,51 +1099,56 @@ __global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfig
   d_status[b] = status;
 }
 
-// In-place -inf fill: one thread per 32-byte sector of logits.  A sector whose
+// In-place -inf fill, grid = (blocks per row, B): threads stride over a row's
+// 32-byte sectors of logits (8 fp32 or 16 bf16), one 256-bit access per
+// sector, so that every store writes a whole sector and a warp's store covers
+// 1 KB of contiguous bytes (few, long-lived blocks: block scheduling, not
+// memory, bounds a grid of one short block per 256 sectors).  A sector whose
 // tokens are all rejected is written without being read; a mixed sector is
-// read, blended and written; a fully accepted sector is not touched.
+// read, blended and written; a fully accepted sector is not touched.  Rows
+// whose sectors are not 32-byte aligned, and the ragged end of a row, are
+// done element by element.
 template <typename T>
 __global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logits, int B,
                                                int V, int W, long long stride, int vec_ok) {
-  constexpr int E = 32 / sizeof(T);  // elements per sector: 8 fp32 or 16 bf16
+  constexpr int E = 32 / sizeof(T);  // elements per sector
+  constexpr uint32_t sfull = E == 32 ? 0xFFFFFFFFu : (1u << E) - 1u;
   pdl_wait();
-  const long long per_row = (V + E - 1) / E;
-  const long long total = per_row * B;
-  for (long long g = (long long)blockIdx.x * blockDim.x + threadIdx.x; g < total;
-       g += (long long)gridDim.x * blockDim.x) {
-    const int b = (int)(g / per_row);
-    const int e0 = (int)(g - (long long)b * per_row) * E;
+  const int b = blockIdx.y;
+  for (int sc = blockIdx.x * blockDim.x + threadIdx.x; sc * E < V; sc += gridDim.x * blockDim.x) {
+    const int e0 = sc * E;
     const uint32_t word = mask[(size_t)b * W + (e0 >> 5)];
-    const uint32_t full = (1u << E) - 1u;
-    const uint32_t bits = (word >> (e0 & 31)) & full;
+    const uint32_t sb = (word >> (e0 & 31)) & sfull;
     T* p = logits + (size_t)b * stride + e0;
     const int n = min(E, V - e0);
     if (vec_ok && n == E) {
-      uint4* p4 = reinterpret_cast<uint4*>(p);
-      if (bits == 0u) {
-        const uint4 v = sizeof(T) == 4 ? make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u)
-                                       : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
-        p4[0] = v;
-        p4[1] = v;
-      } else if (bits != full) {
-        uint4 v[2] = {p4[0], p4[1]};
+      if (sb == 0u) {
+        const uint32_t f = sizeof(T) == 4 ? 0xFF800000u : 0xFF80FF80u;
+        asm volatile("st.global.v8.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1};" ::"l"(p), "r"(f) : "memory");
+      } else if (sb != sfull) {
+        uint32_t u[8];
+        asm volatile("ld.global.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                     : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]), "=r"(u[7])
+                     : "l"(p)
+                     : "memory");
         if (sizeof(T) == 4) {
-          uint32_t* u = reinterpret_cast<uint32_t*>(v);
 #pragma unroll
           for (int k = 0; k < 8; ++k)
-            if (!((bits >> k) & 1u)) u[k] = 0xFF800000u;
+            if (!((sb >> k) & 1u)) u[k] = 0xFF800000u;
         } else {
-          uint16_t* u = reinterpret_cast<uint16_t*>(v);
 #pragma unroll
-          for (int k = 0; k < 16; ++k)
-            if (!((bits >> k) & 1u)) u[k] = 0xFF80u;
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t lo = (sb >> (2 * k)) & 1u, hi = (sb >> (2 * k + 1)) & 1u;
+            u[k] = (lo ? (u[k] & 0xFFFFu) : 0xFF80u) | (hi ? (u[k] & 0xFFFF0000u) : 0xFF800000u);
+          }
         }
-        p4[0] = v[0];
-        p4[1] = v[1];
+        asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(u[0]), "r"(u[1]), "r"(u[2]),
+                     "r"(u[3]), "r"(u[4]), "r"(u[5]), "r"(u[6]), "r"(u[7])
+                     : "memory");
       }
     } else {
       for (int k = 0; k < n; ++k) {
-        if (!((bits >> k) & 1u)) {
+        if (!((sb >> k) & 1u)) {
           if (sizeof(T) == 4)
             reinterpret_cast<uint32_t*>(p)[k] = 0xFF800000u;
           else
@@ -1203,6 +1208,8 @@ size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 }  // namespace grid
 
 using namespace grid;
+
+static int g_sms = 152;  // SM count of the current device, set by grid_specialize
 
 struct grid_spec {
   const grid_grammar* g = nullptr;
@@ -1433,6 +1440,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   cudaGetDevice(&dev);
   s->device = dev;
   cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
+  g_sms = s->sms;
   // CI classification on the device (temporaries live in `tmp`)
   Arena tmp;
   auto fail_tmp = [&](int code) {
@@ -1861,19 +1869,17 @@ extern "C" int grid_apply_mask(const uint32_t* d_mask, void* d_logits, int32_t d
   cudaStream_t st = (cudaStream_t)stream;
   const int W = (V + 31) / 32;
   const int esz = dtype == GRID_DTYPE_F32 ? 4 : 2;
-  const int vec_ok = ((uintptr_t)d_logits % 16 == 0) && ((row_stride * esz) % 16 == 0);
-  const long long sectors = (long long)B * ((V * esz + 31) / 32);
-  int dev = 0, sms = 152;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  long long blocks = (sectors + 255) / 256;
-  blocks = std::min<long long>(blocks, (long long)sms * 8);
+  const int vec_ok = ((uintptr_t)d_logits % 32 == 0) && ((row_stride * esz) % 32 == 0);  // 256-bit sectors
+  if (B > 65535) return set_error(GRID_E_TOO_LARGE, "grid_apply_mask: more than 65535 rows in one call");
+  const int sectors = (V * esz + 31) / 32;  // 32-byte sectors per row
+  const int per_row = std::max(1, std::min((sectors + 255) / 256, (g_sms * 4 + B - 1) / B));
+  const dim3 grid(per_row, B);
   if (dtype == GRID_DTYPE_F32)
-    GRID_CUDA(launch_pdl(k_apply<float>, dim3((int)blocks), dim3(256), 0, st, d_mask, (float*)d_logits, B, V, W,
+    GRID_CUDA(launch_pdl(k_apply<float>, grid, dim3(256), 0, st, d_mask, (float*)d_logits, B, V, W,
                          (long long)row_stride, vec_ok));
   else
-    GRID_CUDA(launch_pdl(k_apply<uint16_t>, dim3((int)blocks), dim3(256), 0, st, d_mask, (uint16_t*)d_logits, B, V,
-                         W, (long long)row_stride, vec_ok));
+    GRID_CUDA(launch_pdl(k_apply<uint16_t>, grid, dim3(256), 0, st, d_mask, (uint16_t*)d_logits, B, V, W,
+                         (long long)row_stride, vec_ok));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }

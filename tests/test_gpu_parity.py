@@ -114,7 +114,7 @@ def test_masked_logits_bit_exact(dtype):
     lg = torch.from_numpy(configs.logits(7, run.B, run.V))
     lg[0, :7] = float("nan")
     tdt = torch.float32 if dtype == "f32" else torch.bfloat16
-    for stride in (run.V, run.V + 8):
+    for stride in (run.V, run.V + 4, run.V + 8):  # 32-byte aligned rows and not
         buf = torch.zeros(run.B, stride, dtype=tdt)
         buf[:, :run.V] = lg.to(tdt)
         ref = buf.clone()
