@@ -455,11 +455,15 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
         m1 = w.m;
         for (int i = 0; i < m1; ++i) s_ovl1[i] = w.ovl[i];
       }
-      Walker w2;
-      walker_init(w2, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, nullptr, nullptr);
-      const int g = eos_gate(ts, w2, mc);
-      if (g < 0) status = GRID_ST_BOUND;
-      eos = g > 0;
+      // EOS gate (Sec. 3.2) on the stack after the same forced emission:
+      // $end's reduce chain must reach ACCEPT
+      if (emit_ok) {
+        int keep_o, m_o, ns;
+        const int a = simulate(ts, base, keep1, (const uint16_t*)s_ovl1, m1, t.n_term, LArr{ls, 1}, kMaxOvl, keep_o, m_o,
+                               ns, mc);
+        if (a < 0) status = GRID_ST_BOUND;
+        eos = a == kAccept;
+      }
     }
     emit_ok = __shfl_sync(0xffffffffu, emit_ok, 0);
     keep1 = __shfl_sync(0xffffffffu, keep1, 0);
