@@ -57,7 +57,7 @@ namespace {
 
 constexpr int kWalkWarps = 8;    // warps per k_walk block
 constexpr int kSpan = 32;        // CD list entries per walk item (one warp batch)
-constexpr int kPrepWarps = 4;    // rows per k_advance block
+constexpr int kAdvWarps = 4;     // rows per k_advance block
 constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_row/k_advance
 constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of this many spellings
@@ -712,7 +712,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   }
   __syncthreads();
   int row = gw % B;
-  int bound = 0, bound_row = -1;
+  int bound_row = -1;  // first row whose walk hit a bound (its status becomes BOUND)
   int cur = -1;  // row whose context is cached below
   int tbl0 = -1, depth = 0, q = 0, lx = 0, keep1 = 0, m1 = 0, nrng = 0;
   uint32_t pc0 = 0, wc0 = 0;
@@ -790,7 +790,6 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     const bool c1 = cidx >= ed && cidx < eb;
     const bool is_vc = (cidx >= ed && cidx < ea) || cidx >= eb;
     if (c1 && m1 > kLaneOvl) {  // sigma' overlay larger than a walk lane holds: flag the row
-      bound = 1;
       bound_row = bound_row < 0 ? row : bound_row;
       continue;
     }
@@ -811,7 +810,6 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
         res = eval_record(ts, w, ts.vc_rec + (size_t)(t.vc_off[tb] + v) * kRecLen, mc);
         if (res < 0 && bound_row < 0) bound_row = row;
-        if (res < 0) bound = 1;
       }
       if (res > 0) atomicOr(&vcbits[((size_t)row * 2 + cxi) * vcw + (v >> 5)], 1u << (v & 31));
       continue;
@@ -860,7 +858,6 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
         res = walk_bytes(ts, w, sp, mc, rej);
         if (res < 0) {
-          bound = 1;
           rej = -1;
           if (bound_row < 0) bound_row = row;
         }
@@ -1001,16 +998,16 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
 }
 
 // One warp per row; lane 0 feeds the tokens, all lanes copy for out-of-place.
-__global__ void __launch_bounds__(kPrepWarps * 32) k_advance(Tables t, DevConfigs cin, DevConfigs cout,
+__global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs cin, DevConfigs cout,
                                                              const int32_t* __restrict__ tokens, int n_steps,
                                                              int32_t* __restrict__ d_status, int B, int copy) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
-  __shared__ uint16_t s_stk[kPrepWarps][kStackWin];
+  __shared__ uint16_t s_stk[kAdvWarps][kStackWin];
   stage_tables(t, ts, smem);
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int b = blockIdx.x * kPrepWarps + warp;
+  const int b = blockIdx.x * kAdvWarps + warp;
   if (b >= B) return;
   if (copy) {
     const int d = cin.depth[b];
@@ -1682,7 +1679,7 @@ extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_con
   if (!s || !in || !out || !d_tokens || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
     return set_error(GRID_E_INVALID_ARG, "grid_advance: bad arguments");
   const int B = in->B;
-  GRID_CUDA(launch_pdl(k_advance, dim3((B + kPrepWarps - 1) / kPrepWarps), dim3(kPrepWarps * 32), s->t.blob_bytes,
+  GRID_CUDA(launch_pdl(k_advance, dim3((B + kAdvWarps - 1) / kAdvWarps), dim3(kAdvWarps * 32), s->t.blob_bytes,
                        (cudaStream_t)stream, s->t, in->c, out->c, d_tokens, n_steps, d_status, B,
                        in != out ? 1 : 0));
   GRID_CUDA(cudaGetLastError());
