@@ -505,57 +505,74 @@ def main():
     value = replica_value(ws, B, args.steps, total_ms)
 
     # ---- end to end through the public API with host buffers ----
-    # Every step copies its logits and token ids from pinned host memory and
-    # reads its mask and status back.  The logits copy of step k+1 runs on a
-    # copy stream into the second of two device buffers while step k
-    # computes; the copy stream waits for the timed region to start, and the
-    # compute stream for each step's copy before its apply.
+    # Every step copies its token ids and logits from pinned host memory and
+    # reads its mask and status back.  Three streams: a host-to-device stream
+    # brings step k+1's inputs into the second of two device buffers while
+    # step k computes, the compute stream waits for them before using them,
+    # and a device-to-host stream reads each step's mask and status (double
+    # buffered) while the next step computes.  The timed region starts before
+    # the first copy and ends after the last read.
     e2e = None
     if not args.no_e2e:
         h_logits = [torch.from_numpy(configs.logits(100 + k, B, V)).pin_memory() for k in range(4)]
         h_toks = [t.cpu().pin_memory() for t in toks]
-        h_mask = torch.empty((B, W), dtype=torch.int32).pin_memory()
-        h_status = torch.empty(B, dtype=torch.int32).pin_memory()
-        d_tok = torch.empty(B, dtype=torch.int32, device=dev)
+        h_mask = [torch.empty((B, W), dtype=torch.int32).pin_memory() for _ in range(2)]
+        h_status = [torch.empty(B, dtype=torch.int32).pin_memory() for _ in range(2)]
+        d_tok = [torch.empty(B, dtype=torch.int32, device=dev) for _ in range(2)]
         d_logits = [torch.empty((B, V), dtype=torch.float32, device=dev) for _ in range(2)]
-        cs = torch.cuda.Stream(device=dev)
-        ev_copied = [torch.cuda.Event() for _ in range(2)]
-        ev_free = [torch.cuda.Event() for _ in range(2)]
+        d_mask = [torch.empty((B, W), dtype=torch.int32, device=dev) for _ in range(2)]
+        d_status = [torch.empty(B, dtype=torch.int32, device=dev) for _ in range(2)]
+        h2d, d2h = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+        ev_in = [torch.cuda.Event() for _ in range(2)]    # step's inputs on the device
+        ev_used = [torch.cuda.Event() for _ in range(2)]  # step's apply done: its input buffers are free
+        ev_out = [torch.cuda.Event() for _ in range(2)]   # step's mask and status read back
 
-        def e2e_step(k):
-            i, j = k % N_BATCHES, k % 2
-            cs.wait_event(ev_free[j])
-            with torch.cuda.stream(cs):
+        def copy_in(k):
+            j = k % 2
+            h2d.wait_event(ev_used[j])
+            with torch.cuda.stream(h2d):
+                d_tok[j].copy_(h_toks[k % N_BATCHES], non_blocking=True)
                 d_logits[j].copy_(h_logits[k % 4], non_blocking=True)
-            ev_copied[j].record(cs)
-            d_tok.copy_(h_toks[i], non_blocking=True)
-            G.grid_advance(spec.h, cfgs[i].h, scratch.h, d_tok, status, stream)
-            G.grid_masks(spec.h, scratch.h, mask, status, stream)
-            stream.wait_event(ev_copied[j])
-            G.grid_apply_mask(mask, d_logits[j], stream)
-            ev_free[j].record(stream)
-            h_mask.copy_(mask, non_blocking=True)
-            h_status.copy_(status, non_blocking=True)
+            ev_in[j].record(h2d)
 
-        for e in ev_free:
-            e.record(stream)
-        for k in range(args.warmup):
-            e2e_step(k)
+        def e2e_step(k, last):
+            i, j = k % N_BATCHES, k % 2
+            if not last:
+                copy_in(k + 1)
+            stream.wait_event(ev_in[j])
+            stream.wait_event(ev_out[j])  # mask/status buffers of step k-2 read back
+            G.grid_advance(spec.h, cfgs[i].h, scratch.h, d_tok[j], d_status[j], stream)
+            G.grid_masks(spec.h, scratch.h, d_mask[j], d_status[j], stream)
+            G.grid_apply_mask(d_mask[j], d_logits[j], stream)
+            ev_used[j].record(stream)
+            d2h.wait_event(ev_used[j])
+            with torch.cuda.stream(d2h):
+                h_mask[j].copy_(d_mask[j], non_blocking=True)
+                h_status[j].copy_(d_status[j], non_blocking=True)
+            ev_out[j].record(d2h)
+
+        def run(n):
+            for e in ev_used + ev_out:
+                e.record(stream)
+            copy_in(0)
+            for k in range(n):
+                e2e_step(k, k == n - 1)
+            stream.wait_event(ev_out[(n - 1) % 2])
+
+        run(args.warmup)
         torch.cuda.synchronize()
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        for e in ev_free:  # no copy of the timed steps starts before the timed region
-            e.record(stream)
-        for k in range(args.steps):
-            e2e_step(k)
+        run(args.steps)
         b.record(stream)
         torch.cuda.synchronize()
         e_ms = a.elapsed_time(b)
         e_ms = max_over_ranks(e_ms, ws, dev)
         e2e = {"value": replica_value(ws, B, args.steps, e_ms), "unit": "masks/s",
                "h2d_bytes_per_step": B * 4 + B * V * 4, "d2h_bytes_per_step": B * W * 4 + B * 4,
-               "overlap": "logits copy of step k+1 on a copy stream during step k (two device buffers)"}
+               "overlap": "inputs of step k+1 copied in and outputs of step k read back on two copy streams "
+                          "while step k computes (double-buffered)"}
 
     # ---- rooflines ----
     # mask apply: HBM-bound, write-mostly; algorithmic bytes = the mask read
