@@ -116,7 +116,6 @@ struct Tables {
   const int32_t* spell_off;
   const uint8_t* spell_bytes;
   const uint4* spell16;  // first 16 bytes of each spelling, zero padded (one load per walk)
-  const int32_t* skip;
   const int32_t* spell_of_id;
   const int32_t* first_of_byte;
   const uint8_t* first_byte_by_id;
@@ -545,46 +544,31 @@ __device__ __forceinline__ Spell load_spell(const Tables& t, int s) {
 }
 
 // Walk one token's bytes (Sec. 4.1).  1 = the output stays a viable prefix,
-// 0 = rejected (every spelling sharing bytes[0..rej] is rejected too:
-// rejection is monotone under extension), -1 = bound.
-__device__ __forceinline__ int walk_bytes(const Tables& t, Walker& w, const Spell& sp, int max_chain, int& rej) {
+// 0 = rejected, -1 = bound.
+__device__ __forceinline__ int walk_bytes(const Tables& t, Walker& w, const Spell& sp, int max_chain) {
   const int len = sp.len;
   for (int i = 0; i < len; ++i) {
     const int b = sp.at(i);
     const int c = t.byte_class[b];
     int nq = t.next[w.q * t.C + c];
     if (nq == kDead) {
-      if (w.q == kStart) {
-        rej = i;
-        return 0;
-      }
-      int e = emit(t, w, max_chain);
-      if (e <= 0) {
-        rej = i;
-        return e;
-      }
+      if (w.q == kStart) return 0;
+      const int e = emit(t, w, max_chain);
+      if (e <= 0) return e;
       w.q = kStart;
       w.lx = 0;
       w.pc = t.root_pc;
       w.wc = t.root_wc;
       nq = t.next[kStart * t.C + c];
-      if (nq == kDead) {
-        rej = i;
-        return 0;
-      }
+      if (nq == kDead) return 0;
     }
     w.q = nq;
     w.lx = lex_step(t, w.lx, b, w.pc, w.wc);
     const Bits4 L = live_prime(t, w.q, w.pc);
     const bool any = w.Acur ? (L & (Bits4::load(w.Acur) | t.ign)).any() : L.any();
-    if (!any) {
-      rej = i;
-      return 0;
-    }
+    if (!any) return 0;
   }
-  int r = trailing_live(t, w, max_chain);
-  if (r == 0) rej = len - 1;
-  return r;
+  return trailing_live(t, w, max_chain);
 }
 
 // EOS gate (Sec. 3.2).  1 / 0 / -1.

@@ -1066,17 +1066,6 @@ extern "C" int grid_load_vocab(const uint8_t* bytes, const int64_t* offsets, int
     h.spell_of_id[sp[i].second] = (int32_t)h.spell_off.size() - 2;
   }
   h.NS = (int)h.spell_off.size() - 1;
-  // subtree ends: skip(s, d) = s+1 if s+1 does not share d+1 bytes, else skip(s+1, d)
-  h.skip.assign(h.spell_bytes.size(), 0);
-  for (int s = h.NS - 1; s >= 0; --s) {
-    int a = h.spell_off[s], la = h.spell_off[s + 1] - a;
-    int lcp = 0;
-    if (s + 1 < h.NS) {
-      int b = h.spell_off[s + 1], lb = h.spell_off[s + 2] - b;
-      while (lcp < la && lcp < lb && h.spell_bytes[a + lcp] == h.spell_bytes[b + lcp]) ++lcp;
-    }
-    for (int d = 0; d < la; ++d) h.skip[a + d] = (lcp >= d + 1) ? h.skip[h.spell_off[s + 1] + d] : s + 1;
-  }
   h.first_of_byte.assign(257, h.NS);
   for (int s = h.NS - 1; s >= 0; --s) h.first_of_byte[h.spell_bytes[h.spell_off[s]]] = s;
   for (int b = 255; b >= 0; --b)

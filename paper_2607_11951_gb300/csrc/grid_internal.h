@@ -55,16 +55,14 @@ struct HostGrammar {
 };
 
 // Byte trie of the vocabulary (Def. 3), stored as the lexicographically sorted
-// distinct spellings (= DFS order of the trie) plus, for every spelling s and
-// depth d < len(s), skip[off(s)+d] = the first spelling index after s that does
-// not share s's first d+1 bytes (the end of the subtree of that trie node).
+// distinct spellings (= DFS order of the trie): the spellings that start with
+// one byte, and so one subtree of the root, are contiguous.
 struct HostVocab {
   int V = 0;
   int eos = -1;
   int NS = 0;
   std::vector<int32_t> spell_off;   // NS+1
   std::vector<uint8_t> spell_bytes;
-  std::vector<int32_t> skip;        // parallel to spell_bytes
   std::vector<int32_t> spell_of_id; // V, -1 for EOS/special
   std::vector<int32_t> first_of_byte;  // 257: spellings with first byte b are [f[b], f[b+1])
   bool byte_complete = false;

@@ -31,7 +31,8 @@
 //            against the row's stack, and the byte walks: lanes walk token
 //            bytes through the DFA and the identifier trie, emissions pick the
 //            highest-priority parser-viable candidate on a copy-on-write
-//            overlay, a rejected prefix skips its whole trie subtree (Sec. 4.1)
+//            overlay (Sec. 4.1); first-byte subtrees of the trie in which no
+//            spelling can survive are never entered
 //   k_pack   per token id: CI class selection | verdict class | walked verdict
 //            | EOS gate, packed into the id-order mask (alias ids share a
 //            spelling and so a verdict)
@@ -60,7 +61,7 @@ constexpr int kSpan = 32;        // CD list entries per walk item (one warp batc
 constexpr int kAdvWarps = 4;     // rows per k_advance block
 constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_row/k_advance
 constexpr int kPackRows = 8;     // rows per k_pack block
-constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of this many spellings
+constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of (up to) this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
 constexpr int kRowWarps = 6;     // k_row: warps per row block
 constexpr int kRowJobWarps = 4;  // k_row: warps 2 .. 5 compute the allowed sets after one shift
@@ -677,10 +678,11 @@ __device__ __forceinline__ int4 row_queue(const Tables& t, const RowCtx& x) {
 // its first stack-dependent emission is selected for the context's allowed
 // set (otherwise that emission, and so the spelling, fails) and, for sigma',
 // if its first byte ends the pending lexeme; survivors are compacted onto the
-// low lanes.  Range items (kRangeSpan spellings of one first-byte range):
-// lanes walk consecutive spellings; when the last lane's spelling is rejected,
-// every spelling sharing its rejected prefix is skipped (a trie subtree,
-// contiguous in DFS order).  Both kinds share one call of walk_bytes.
+// low lanes.  Range items (up to kRangeSpan spellings of one live first-byte
+// range; k_row already dropped the first-byte subtrees in which no spelling
+// can survive): the range's items interleave, lane j of item i walking
+// spelling lo + i + j * (items of the range).  Both kinds share one call of
+// walk_bytes, one spelling per lane.
 __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* __restrict__ ctx,
                                                              const RowRanges* __restrict__ rng, const uint16_t* stacks,
                                                              const int32_t* __restrict__ surv, int cap,
@@ -816,7 +818,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     }
     uint32_t* vb = (c1 ? verd1 : verd0) + (size_t)row * words_ns;
     const int32_t* list = nullptr;
-    int p0, p1;
+    int p0, p1, step = 1;
     if (c1 || tbl0 >= 0) {  // survivors of k_filter
       const int n = c1 ? r.nsurv[1] : r.nsurv[0];
       list = surv + ((size_t)row * 2 + (c1 ? 1 : 0)) * cap;
@@ -833,49 +835,33 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
         else
           z = mid;
       }
-      p0 = R.lo[a] + (c0 - R.cpre[a]) * kRangeSpan;
-      p1 = min(R.hi[a], p0 + kRangeSpan);
+      // the range's items interleave: item i takes spellings lo + i,
+      // lo + i + n, lo + i + 2n, ... (n items), so that runs of costly
+      // neighbours (long multi-word continuations of one prefix) spread
+      // over many warps instead of lengthening one
+      step = R.cpre[a + 1] - R.cpre[a];
+      p0 = R.lo[a] + (c0 - R.cpre[a]);
+      p1 = R.hi[a];
     }
-    // ---- one or more warp batches, one walk call site
-    int pos = p0;
-    for (bool first = true;; first = false) {
-      int s = -1;
+    // ---- one spelling per lane, one walk call site
+    {
+      int sp_i = -1;
       bool go = false;
       if (list) {
-        if (!first) break;
         const int i = p0 + lane;
         go = i < p1;
-        if (go) s = list[i];
+        if (go) sp_i = list[i];
       } else {
-        if (pos >= p1) break;
-        s = pos + lane;
-        go = s < p1;
+        sp_i = p0 + lane * step;
+        go = sp_i < p1;
       }
-      int res = 0, rej = -1;
       if (go) {
-        const Spell sp = load_spell(ts, s);
+        const Spell sp = load_spell(ts, sp_i);
         Walker w;
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
-        res = walk_bytes(ts, w, sp, mc, rej);
-        if (res < 0) {
-          rej = -1;
-          if (bound_row < 0) bound_row = row;
-        }
-      }
-      if (list) {
-        if (res > 0) atomicOr(&vb[s >> 5], 1u << (s & 31));
-      } else {
-        const uint32_t m = __ballot_sync(0xffffffffu, res > 0);
-        if (lane == 0 && m) {
-          const int sh = pos & 31;
-          atomicOr(&vb[pos >> 5], m << sh);
-          if (sh && (m >> (32 - sh))) atomicOr(&vb[(pos >> 5) + 1], m >> (32 - sh));
-        }
-        int nxt = pos + 32;
-        const int last = min(31, p1 - 1 - pos);
-        const int lrej = __shfl_sync(0xffffffffu, rej, last);
-        if (lrej >= 0) nxt = max(nxt, ts.skip[ts.spell_off[pos + last] + lrej]);
-        pos = nxt;
+        const int res = walk_bytes(ts, w, sp, mc);
+        if (res < 0 && bound_row < 0) bound_row = row;
+        if (res > 0) atomicOr(&vb[sp_i >> 5], 1u << (sp_i & 31));
       }
     }
   }
@@ -1067,8 +1053,7 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
       status = GRID_ST_TOKEN_NOT_ALLOWED;
       break;
     }
-    int rej;
-    const int r = walk_bytes(ts, w, load_spell(t, s), mc, rej);
+    const int r = walk_bytes(ts, w, load_spell(t, s), mc);
     if (r < 0) {
       status = GRID_ST_BOUND;
       break;
@@ -1401,7 +1386,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   if ((rc = a.upload(h.lx_cstart, &t.lx_cstart)) || (rc = a.upload(h.lx_cbyte, &t.lx_cbyte)) ||
       (rc = a.upload(h.lx_cnode, &t.lx_cnode)) || (rc = a.upload(h.lx_pcats, &t.lx_pcats)) ||
       (rc = a.upload(h.lx_wcats, &t.lx_wcats)) || (rc = a.upload(hv.spell_off, &t.spell_off)) ||
-      (rc = a.upload(hv.spell_bytes, &t.spell_bytes)) || (rc = a.upload(hv.skip, &t.skip)) ||
+      (rc = a.upload(hv.spell_bytes, &t.spell_bytes)) ||
       (rc = a.upload(spell_of_id_p, &t.spell_of_id)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
     return fail(rc);
   {
