@@ -267,40 +267,18 @@ __device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, in
   }
 }
 
-// A(sigma) for the virtual stack base[0:keep] ++ ovl[0:m], by one set
-// simulation on lane 0 (`scr`: its scratch, kMaxOvl entries), broadcast to
-// the warp.
-__device__ Bits4 allowed_set(const Tables& t, const uint16_t* base, int keep, const uint16_t* ovl, int m,
-                             int& status, int lane, LArr scr) {
-  const int mc = max_chain_of(t);
-  uint32_t wds[4] = {0u, 0u, 0u, 0u};
-  if (lane == 0) {
-    Bits4 G = Bits4::zero();
-    for (int k = 0; k < t.n_term; ++k) G.set(k);
-    G = G.andnot(t.ign);
-    bool bound = false;
-    const Bits4 A = simulate_set(t, base, keep, ovl, m, G, scr, kMaxOvl, mc, bound);
-    if (bound) status = GRID_ST_BOUND;
-    wds[0] = A.x;
-    wds[1] = A.y;
-    wds[2] = A.z;
-    wds[3] = A.w;
-  }
-#pragma unroll
-  for (int k = 0; k < 4; ++k) wds[k] = __shfl_sync(0xffffffffu, wds[k], 0);
-  return Bits4{wds[0], wds[1], wds[2], wds[3]};
-}
-
 // One block per row (kRowWarps warps), plus clearing blocks after the rows.
-// Phase 1, three warps at once: warp 0 computes A0 = A(sigma) and then the
-// live first-byte ranges that continue the pending lexeme (rows without a CI
-// table); warp 1 makes the forced emission of the pending lexeme (sigma ->
-// sigma', what every token whose first byte ends the lexeme must go through),
-// the EOS gate (Sec. 3.2) and A1 = A(sigma'); warp 2 finds the first bytes
-// that end the lexeme.  Phase 2: for both contexts, lanes of the job warps
-// take one allowed terminal tau each and compute the allowed set after tau's
-// reduce chain and shift (A2: walks and verdict classes simulate nothing
-// before their second shift); warps 0 and 1 select the contexts' CI classes.
+// Phase 1, every warp at once: warp 0 finds the first bytes that end the
+// pending lexeme; warp 1 makes the forced emission of the pending lexeme
+// (sigma -> sigma', what every token whose first byte ends the lexeme must go
+// through) and the EOS gate (Sec. 3.2) on the stack it leaves; lanes of the
+// job warps take one terminal tau each, in sigma (first half) or sigma'
+// (second half, each lane making the same forced emission itself): tau is
+// allowed iff its reduce chain reaches SHIFT (A0 and A1 are the warps'
+// ballots), and then the allowed set after that shift is A2 (walks and verdict
+// classes simulate nothing before their second shift).  Phase 2: warp 0 lays
+// out the live first-byte ranges that continue the lexeme (rows without a CI
+// table; they need A0), warps 1 and 2 select the contexts' CI classes.
 // Clearing blocks zero both verdict bitmaps and the verdict-class bits.
 __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
                                                         RowRanges* __restrict__ rng, uint32_t* __restrict__ A2,
@@ -313,9 +291,8 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   __shared__ uint16_t s_ovl1[kMaxOvl];
   __shared__ uint16_t s_ovl2[kRowJobWarps][kMaxOvl * 32];
   __shared__ uint16_t s_scr[kRowJobWarps][kMaxOvl * 32];
-  __shared__ uint16_t s_scr01[2][kMaxOvl];
   __shared__ uint32_t s_A0[4], s_A1[4], s_keep[8], s_kill[8];
-  __shared__ int s_row[8];  // complete, depth, q, lx, emit_ok, keep1, m1, eos_ok | sigma'==sigma << 1
+  __shared__ int s_row[8];  // complete, depth, q, lx, emit_ok, keep1, m1, eos_ok
   __shared__ uint32_t s_pc[2];
   __shared__ int s_status, s_total0, s_nrng;
   if ((int)blockIdx.x >= B) {
@@ -366,17 +343,125 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   const int mc = max_chain_of(t);
   const int tbl0 = (q != kStart && t.ci_on) ? t.tbl_of_q[q] : -1;
   int status = GRID_ST_OK;
-  // ---- phase 1
+  // ---- phase 1: all at once
+  if (threadIdx.x < 8) s_keep[threadIdx.x] = 0u;
+  if (threadIdx.x < 4) {
+    s_A0[threadIdx.x] = 0u;
+    s_A1[threadIdx.x] = 0u;
+  }
+  __syncthreads();
   if (warp == 0) {
-    Bits4 A0 = Bits4::zero();
-    if (!complete) A0 = allowed_set(ts, base, depth, nullptr, 0, status, lane, LArr{s_scr01[0], 1});
-    if (lane < 4) s_A0[lane] = A0.word(lane);
-    // continuing first-byte ranges (rows without a CI table for q).  A first
-    // byte whose lexeme has no live terminal in A0 u I (category terminals
-    // counted only while the lexeme is a prefix of one of their words)
-    // rejects every spelling it starts: liveness only shrinks along the
-    // lexeme, and any later emission picks among its live terminals.
-    if (!complete && q != kStart && tbl0 < 0) {
+    // first bytes that end the pending lexeme (every byte when it is empty)
+    for (int b0 = 0; b0 < 256; b0 += 32) {
+      const int by = b0 + lane;
+      const bool kill = q == kStart || ts.next[q * ts.C + ts.byte_class[by]] == kDead;
+      const uint32_t word = __ballot_sync(0xffffffffu, kill);
+      if (lane == 0) s_kill[b0 >> 5] = word;
+    }
+  } else if (warp == 1) {
+    // the forced emission of the pending lexeme (sigma -> sigma'), and the
+    // EOS gate (Sec. 3.2) on the stack it leaves
+    int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
+    if (lane == 0 && !complete) {
+      Walker w;
+      uint16_t lo[kMaxOvl], ls[kMaxOvl];
+      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, nullptr, nullptr);
+      if (q == kStart) {
+        emit_ok = 1;
+      } else {
+        const int e = emit(ts, w, mc);
+        if (e < 0) status = GRID_ST_BOUND;
+        emit_ok = e > 0;
+        keep1 = w.keep;
+        m1 = w.m;
+        for (int i = 0; i < m1; ++i) s_ovl1[i] = w.ovl[i];
+      }
+      if (emit_ok) {
+        int keep_o, m_o, ns;
+        const int a = simulate(ts, base, keep1, (const uint16_t*)s_ovl1, m1, t.n_term, LArr{ls, 1}, kMaxOvl, keep_o, m_o,
+                               ns, mc);
+        if (a < 0) status = GRID_ST_BOUND;
+        eos = a == kAccept;
+      }
+      s_row[4] = emit_ok;
+      s_row[5] = keep1;
+      s_row[6] = m1;
+      s_row[7] = eos;
+    }
+  } else if (!complete) {
+    // job warps: lane l of job warp jw takes terminal tau = 32 jw + l (and
+    // tau + 32 * half, ...) in one context: tau is allowed iff its reduce
+    // chain reaches SHIFT (A0 / A1 are the ballots), and then the allowed set
+    // after that shift (A2) comes from one set simulation.  sigma' lanes make
+    // the forced emission themselves (the same pick as warp 1), so that both
+    // contexts start at once.
+    const int half = kRowJobWarps / 2;
+    const int cx = warp - 2 >= half ? 1 : 0;
+    const int jw = warp - 2 - cx * half;
+    const LArr scr{s_scr[warp - 2] + lane, 32}, ovl{s_ovl2[warp - 2] + lane, 32};
+    int keep = depth, m = 0;
+    bool has_ctx = cx == 0 ? q != kStart : true;
+    if (cx == 1 && q != kStart) {
+      Walker w;
+      walker_init(w, ovl, scr, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, nullptr, nullptr);
+      const int e = emit(ts, w, mc);
+      if (e < 0) status = GRID_ST_BOUND;
+      has_ctx = e > 0;
+      keep = w.keep;
+      m = w.m;  // sigma' is base[0:keep] ++ ovl[0:m]
+    }
+    Bits4 G = Bits4::zero();
+    for (int k = 0; k < t.n_term; ++k) G.set(k);
+    G = G.andnot(ts.ign);
+    for (int tau0 = jw * 32; has_ctx && tau0 < t.n_term; tau0 += 32 * half) {
+      const int tau = tau0 + lane;
+      bool allowed = false;
+      Bits4 An = Bits4::zero();
+      if (tau < t.n_term && !ts.ign.has(tau)) {
+        int keep_o, m_o, ns;
+        const int a = simulate(ts, base, keep, ovl, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
+        if (a < 0) status = GRID_ST_BOUND;
+        allowed = a > 0 && a != kAccept;
+        if (allowed) {
+          if (m_o + ns + 1 <= kMaxOvl) {
+            // the stack after the shift, built in place: base[0:keep_o] ++
+            // ovl[0:m_o] ++ scr[0:ns] ++ (a-1); sigma' itself is rebuilt for
+            // the next terminal of this lane
+            uint16_t saved[kMaxOvl];
+            for (int i = 0; i < m; ++i) saved[i] = ovl[i];
+            for (int i = 0; i < ns; ++i) ovl[m_o + i] = scr[i];
+            ovl[m_o + ns] = (uint16_t)(a - 1);
+            bool bound = false;
+            An = simulate_set(ts, base, keep_o, ovl, m_o + ns + 1, G, scr, kMaxOvl, mc, bound);
+            if (bound) status = GRID_ST_BOUND;
+            for (int i = 0; i < m; ++i) ovl[i] = saved[i];
+          } else {
+            status = GRID_ST_BOUND;
+          }
+          uint32_t* out = A2 + (((size_t)b * 2 + cx) * t.T1 + tau) * 4;
+          out[0] = An.x;
+          out[1] = An.y;
+          out[2] = An.z;
+          out[3] = An.w;
+        }
+      }
+      const uint32_t word = __ballot_sync(0xffffffffu, allowed);
+      if (lane == 0 && word) atomicOr(cx ? &s_A1[tau0 >> 5] : &s_A0[tau0 >> 5], word);
+    }
+  }
+  status = __reduce_max_sync(0xffffffffu, status);
+  if (lane == 0 && status != GRID_ST_OK) atomicMax(&s_status, status);
+  __syncthreads();
+  const int emit_ok = complete ? 0 : s_row[4], keep1 = complete ? depth : s_row[5], m1 = complete ? 0 : s_row[6];
+  const Bits4 A0 = Bits4::load(s_A0), A1 = Bits4::load(s_A1);
+  // ---- phase 2: ranges (warp 0), class selections (warps 1, 2)
+  if (!complete) {
+    if (warp == 0 && q != kStart && tbl0 < 0) {
+      // continuing first-byte ranges (rows without a CI table for q).  A first
+      // byte whose lexeme has no live terminal in A0 u I (category terminals
+      // counted only while the lexeme is a prefix of one of their words)
+      // rejects every spelling it starts: liveness only shrinks along the
+      // lexeme, and any later emission picks among its live terminals.
       int total0 = 0, nrng = 0;
       RowRanges& R = rng[b];
       const Bits4 AI = A0 | ts.ign;
@@ -394,8 +479,6 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
         cw[j] = __ballot_sync(0xffffffffu, hi_r[j] > lo_r[j] && ts.next[q * ts.C + ts.byte_class[by]] != kDead);
         nc += __popc(cw[j]);
       }
-      if (lane < 8) s_keep[lane] = 0u;
-      __syncwarp();
       for (int i0 = 0; i0 < nc; i0 += 32) {  // the live test of the continuing bytes, one per lane
         int idx = i0 + lane, by = -1;
         if (idx < nc) {
@@ -438,69 +521,18 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
         s_total0 = total0;
         s_nrng = nrng;
       }
-    }
-  } else if (warp == 1) {
-    // forced emission of the pending lexeme, EOS gate, A1
-    int emit_ok = 0, keep1 = depth, m1 = 0, eos = 0;
-    if (lane == 0 && !complete) {
-      Walker w;
-      uint16_t lo[kMaxOvl], ls[kMaxOvl];
-      walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, base, depth, nullptr, 0, q, lx, pc0, wc0, nullptr, nullptr);
-      if (q == kStart) {
-        emit_ok = 1;
-      } else {
-        const int e = emit(ts, w, mc);
-        if (e < 0) status = GRID_ST_BOUND;
-        emit_ok = e > 0;
-        keep1 = w.keep;
-        m1 = w.m;
-        for (int i = 0; i < m1; ++i) s_ovl1[i] = w.ovl[i];
-      }
-      // EOS gate (Sec. 3.2) on the stack after the same forced emission:
-      // $end's reduce chain must reach ACCEPT
-      if (emit_ok) {
-        int keep_o, m_o, ns;
-        const int a = simulate(ts, base, keep1, (const uint16_t*)s_ovl1, m1, t.n_term, LArr{ls, 1}, kMaxOvl, keep_o, m_o,
-                               ns, mc);
-        if (a < 0) status = GRID_ST_BOUND;
-        eos = a == kAccept;
-      }
-    }
-    emit_ok = __shfl_sync(0xffffffffu, emit_ok, 0);
-    keep1 = __shfl_sync(0xffffffffu, keep1, 0);
-    m1 = __shfl_sync(0xffffffffu, m1, 0);
-    __syncwarp();
-    Bits4 A1 = Bits4::zero();
-    const bool same = keep1 == depth && m1 == 0;  // sigma' = sigma: A1 = A0, taken after the barrier
-    if (!complete && emit_ok && !same) A1 = allowed_set(ts, base, keep1, s_ovl1, m1, status, lane, LArr{s_scr01[1], 1});
-    if (lane < 4) s_A1[lane] = A1.word(lane);
-    if (lane == 0) {
-      s_row[4] = emit_ok;
-      s_row[5] = keep1;
-      s_row[6] = m1;
-      s_row[7] = eos | (same ? 2 : 0);
-    }
-  } else if (warp == 2) {
-    // first bytes that end the pending lexeme (every byte when it is empty)
-    for (int b0 = 0; b0 < 256; b0 += 32) {
-      const int by = b0 + lane;
-      const bool kill = q == kStart || ts.next[q * ts.C + ts.byte_class[by]] == kDead;
-      const uint32_t word = __ballot_sync(0xffffffffu, kill);
-      if (lane == 0) s_kill[b0 >> 5] = word;
+    } else if (warp == 1 && t.ci_on && tbl0 >= 0) {
+      select_classes(ts, A0, sel + ((size_t)b * 2) * t.nselw, lane);
+    } else if (warp == 2 && t.ci_on && emit_ok) {
+      select_classes(ts, A1, sel + ((size_t)b * 2 + 1) * t.nselw, lane);
     }
   }
-  status = __reduce_max_sync(0xffffffffu, status);
-  if (lane == 0 && status != GRID_ST_OK) atomicMax(&s_status, status);
   __syncthreads();
-  const int emit_ok = s_row[4], keep1 = s_row[5], m1 = s_row[6];
-  if (threadIdx.x < 4 && (s_row[7] & 2) && emit_ok && !complete) s_A1[threadIdx.x] = s_A0[threadIdx.x];
-  __syncthreads();
-  const Bits4 A0 = Bits4::load(s_A0), A1 = Bits4::load(s_A1);
   // ---- the row's context for the later kernels
   if (threadIdx.x == 0) {
     for (int k = 0; k < 4; ++k) {
       r.A0[k] = s_A0[k];
-      r.A1[k] = s_A1[k];
+      r.A1[k] = emit_ok ? s_A1[k] : 0u;
     }
     for (int k = 0; k < 8; ++k) r.kill[k] = s_kill[k];
     r.q = q;
@@ -510,7 +542,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
     r.depth = depth;
     r.tbl0 = tbl0;
     r.emit_ok = emit_ok;
-    r.eos_ok = s_row[7] & 1;
+    r.eos_ok = complete ? 0 : s_row[7];
     r.complete = complete;
     r.nonempty = 0;
     r.done_blocks = 0;
@@ -525,52 +557,6 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
     r.nrng = s_nrng;
   }
   for (int i = threadIdx.x; i < m1; i += blockDim.x) r.ovl1[i] = s_ovl1[i];
-  // ---- phase 2
-  status = GRID_ST_OK;
-  if (!complete) {
-    if (warp >= 2) {
-      // A2 of the allowed terminals: the first half of the job warps for
-      // sigma, the second half for sigma'
-      const int half = kRowJobWarps / 2;
-      const int cx = warp - 2 >= half ? 1 : 0;
-      const int jw = warp - 2 - cx * half;
-      const bool has_ctx = cx ? (emit_ok != 0) : (q != kStart);
-      const Bits4 A = cx ? A1 : A0;
-      const int keep = cx ? keep1 : depth, m = cx ? m1 : 0;
-      const LArr scr{s_scr[warp - 2] + lane, 32}, ovl2{s_ovl2[warp - 2] + lane, 32};
-      Bits4 G = Bits4::zero();
-      for (int k = 0; k < t.n_term; ++k) G.set(k);
-      G = G.andnot(ts.ign);
-      for (int tau = jw * 32 + lane; has_ctx && tau < t.n_term; tau += 32 * half) {
-        if (!A.has(tau)) continue;
-        int keep_o, m_o, ns;
-        const int a = simulate(ts, base, keep, (const uint16_t*)s_ovl1, m, tau, scr, kMaxOvl, keep_o, m_o, ns, mc);
-        Bits4 An = Bits4::zero();
-        if (a > 0 && a != kAccept && m_o + ns + 1 <= kMaxOvl) {
-          for (int i = 0; i < m_o; ++i) ovl2[i] = s_ovl1[i];
-          for (int i = 0; i < ns; ++i) ovl2[m_o + i] = scr[i];
-          ovl2[m_o + ns] = (uint16_t)(a - 1);
-          bool bound = false;
-          An = simulate_set(ts, base, keep_o, ovl2, m_o + ns + 1, G, scr, kMaxOvl, mc, bound);
-          if (bound) status = GRID_ST_BOUND;
-        } else {
-          status = GRID_ST_BOUND;
-        }
-        uint32_t* out = A2 + (((size_t)b * 2 + cx) * t.T1 + tau) * 4;
-        out[0] = An.x;
-        out[1] = An.y;
-        out[2] = An.z;
-        out[3] = An.w;
-      }
-    } else if (t.ci_on) {
-      // class selections: warp 0 for sigma (rows with a table), warp 1 for sigma'
-      if (warp == 0 && tbl0 >= 0) select_classes(ts, A0, sel + ((size_t)b * 2) * t.nselw, lane);
-      if (warp == 1 && emit_ok) select_classes(ts, A1, sel + ((size_t)b * 2 + 1) * t.nselw, lane);
-    }
-  }
-  status = __reduce_max_sync(0xffffffffu, status);
-  if (lane == 0 && status != GRID_ST_OK) atomicMax(&s_status, status);
-  __syncthreads();
   if (threadIdx.x == 0) r.status = complete ? GRID_ST_COMPLETE : s_status;
 }
 
