@@ -117,6 +117,8 @@ struct Tables {
   const uint8_t* spell_bytes;
   const uint4* spell16;  // first 16 bytes of each spelling, zero padded (one load per walk)
   const int32_t* spell_of_id;
+  const int32_t* id_of_spell;  // NS: the smallest id with each spelling
+  const int32_t* next_alias;   // Vp: the next larger id with the same spelling, -1 after the last
   const int32_t* first_of_byte;
   const uint8_t* first_byte_by_id;
   // CI tables (one per lexer state in the precomputed set; table 0 = start state)

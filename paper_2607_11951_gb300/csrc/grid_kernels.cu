@@ -32,10 +32,11 @@
 //            bytes through the DFA and the identifier trie, emissions pick the
 //            highest-priority parser-viable candidate on a copy-on-write
 //            overlay (Sec. 4.1); first-byte subtrees of the trie in which no
-//            spelling can survive are never entered
+//            spelling can survive are never entered; a walked spelling's
+//            verdict is set for each of its ids (alias ids share a spelling
+//            and so a verdict) in an id-indexed bitmap with the mask's layout
 //   k_pack   per token id: CI class selection | verdict class | walked verdict
-//            | EOS gate, packed into the id-order mask (alias ids share a
-//            spelling and so a verdict)
+//            | EOS gate, packed into the id-order mask
 // Parser step (grid_advance):  k_advance.   Masked logits:  k_apply.
 //
 // Every loop is bounded; hitting a bound writes GRID_ST_BOUND.  No kernel traps.
@@ -87,7 +88,7 @@ struct RowCtx {
   int32_t q, lx, depth, tbl0;
   uint32_t pc0, wc0;  // category bits of the pending lexeme's trie node
   int32_t emit_ok, eos_ok, status, complete;
-  uint32_t nonempty, done_blocks;
+  unsigned long long pack_done;  // k_pack blocks done with the row (low half) and with a set bit (high half)
   int32_t keep1, m1;
   int32_t work0;          // next item of the row's walk queue
   int32_t nrange;         // items over the continuing first-byte ranges (rows without a CI table)
@@ -284,7 +285,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
                                                         RowRanges* __restrict__ rng, uint32_t* __restrict__ A2,
                                                         uint32_t* __restrict__ sel, uint32_t* __restrict__ verd0,
                                                         uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
-                                                        int n_vcbits, int B, int words_ns) {
+                                                        int n_vcbits, int B, int words_v) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   __shared__ uint16_t s_stk[kStackWin];
@@ -298,7 +299,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   if ((int)blockIdx.x >= B) {
     // clearing blocks: zero both verdict bitmaps and the verdict-class bits of every row
     pdl_wait();
-    const size_t n = (size_t)B * words_ns;
+    const size_t n = (size_t)B * words_v;
     const size_t n4 = n >> 2;
     const size_t stride = (size_t)(gridDim.x - B) * blockDim.x;
     const size_t first = (size_t)(blockIdx.x - B) * blockDim.x + threadIdx.x;
@@ -544,8 +545,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
     r.emit_ok = emit_ok;
     r.eos_ok = complete ? 0 : s_row[7];
     r.complete = complete;
-    r.nonempty = 0;
-    r.done_blocks = 0;
+    r.pack_done = 0ull;
     r.keep1 = keep1;
     r.m1 = m1;
     r.work0 = 0;
@@ -676,7 +676,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
                                                              uint32_t* __restrict__ verd0,
                                                              uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
                                                              int vcw, const int32_t* __restrict__ vsurv, int vcap,
-                                                             int words_ns, int B) {
+                                                             int words_v, int B) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
   __shared__ uint16_t s_win[kWalkWarps][kWalkWin];
@@ -802,7 +802,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
       if (res > 0) atomicOr(&vcbits[((size_t)row * 2 + cxi) * vcw + (v >> 5)], 1u << (v & 31));
       continue;
     }
-    uint32_t* vb = (c1 ? verd1 : verd0) + (size_t)row * words_ns;
+    uint32_t* vb = (c1 ? verd1 : verd0) + (size_t)row * words_v;
     const int32_t* list = nullptr;
     int p0, p1, step = 1;
     if (c1 || tbl0 >= 0) {  // survivors of k_filter
@@ -847,7 +847,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
         const int res = walk_bytes(ts, w, sp, mc);
         if (res < 0 && bound_row < 0) bound_row = row;
-        if (res > 0) atomicOr(&vb[sp_i >> 5], 1u << (sp_i & 31));
+        if (res > 0)  // the verdict of every id with this spelling, in the mask's layout
+          for (int id = t.id_of_spell[sp_i]; id >= 0; id = t.next_alias[id]) atomicOr(&vb[id >> 5], 1u << (id & 31));
       }
     }
   }
@@ -866,12 +867,11 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
 __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
                                               const uint32_t* __restrict__ vcbits, int vcw,
                                               const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
-                                              int words_ns, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
+                                              int words_v, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
                                               int B) {
   extern __shared__ __align__(16) uint32_t s_sel[];  // kPackRows * 2 * nselw
   __shared__ int s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
   __shared__ uint32_t s_kill[kPackRows][8];
-  __shared__ int s_last;
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int base = blockIdx.x * 1024 + warp * 128 + lane * 4;  // this thread's ids base .. base+3
@@ -913,12 +913,16 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   const int eos_j = t.eos - base;  // the EOS id's slot in this thread, if 0..3
   if (eos_j >= 0 && eos_j < 4) sp[eos_j] = -1;  // EOS takes only the gate's bit
   __syncthreads();
+  const int wi = (blockIdx.x * 1024 + warp * 128) / 32 + (lane >> 3);
   for (int k = 0; k < nr; ++k) {
     const int b = r0 + k;
     const int fl = s_fl[k];
     const int tb = s_tbl[k];
     uint32_t nib = 0u;
     if (have && !(fl & 4)) {
+      // the walks' verdicts of this word's ids, both contexts (one coalesced load each)
+      const uint32_t wv[2] = {verd0[(size_t)b * words_v + wi] >> (base & 31),
+                              (fl & 1) ? verd1[(size_t)b * words_v + wi] >> (base & 31) : 0u};
       ushort4 ct = make_ushort4(code_walk, code_walk, code_walk, code_walk);
       if (tb >= 0) ct = *reinterpret_cast<const ushort4*>(t.cls_by_id + (size_t)tb * t.Vp + base);
       const int ctv[4] = {ct.x, ct.y, ct.z, ct.w};
@@ -933,7 +937,7 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
             const uint32_t v = cx ? vs[j] : t.vc_by_id[(size_t)tb * t.Vp + base + j];
             bit = (vcbits[((size_t)b * 2 + cx) * vcw + (v >> 5)] >> (v & 31)) & 1u;
           } else {
-            bit = ((cx ? verd1 : verd0)[(size_t)b * words_ns + (sp[j] >> 5)] >> (sp[j] & 31)) & 1u;
+            bit = (wv[cx] >> j) & 1u;
           }
         }
         nib |= bit << j;
@@ -944,26 +948,21 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
     v |= __shfl_xor_sync(0xffffffffu, v, 1);
     v |= __shfl_xor_sync(0xffffffffu, v, 2);
     v |= __shfl_xor_sync(0xffffffffu, v, 4);
-    const int wi = (blockIdx.x * 1024 + warp * 128) / 32 + (lane >> 3);
     if ((lane & 7) == 0 && wi < t.W) {
       mask[(size_t)b * t.W + wi] = v;
       if (v) s_any[k] = 1;
     }
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < nr; i += blockDim.x)
-    if (s_any[i]) atomicOr(&ctx[r0 + i].nonempty, 1u);
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    s_last = atomicAdd(&ctx[0].done_blocks, 1u) == gridDim.x * gridDim.y - 1;
-  }
-  __syncthreads();
-  if (s_last) {
-    __threadfence();
-    for (int b = threadIdx.x; b < B; b += blockDim.x) {
+  // one atomic per row counts the block and carries whether it set a bit; the
+  // row's last block writes its status
+  if (threadIdx.x < nr) {
+    const int b = r0 + threadIdx.x;
+    const unsigned long long old =
+        atomicAdd(&ctx[b].pack_done, 1ull + (s_any[threadIdx.x] ? (1ull << 32) : 0ull));
+    if ((uint32_t)old == gridDim.x - 1) {
       int st = atomicAdd(&ctx[b].status, 0);
-      if (st == GRID_ST_OK && atomicAdd(&ctx[b].nonempty, 0u) == 0u) st = GRID_ST_EMPTY_MASK;
+      if (st == GRID_ST_OK && (old >> 32) == 0ull && !s_any[threadIdx.x]) st = GRID_ST_EMPTY_MASK;
       d_status[b] = st;
     }
   }
@@ -1201,7 +1200,7 @@ struct grid_spec {
 constexpr int kMaskKernels = 4;  // k_row, k_filter, k_walk, k_pack
 
 struct grid_configs {
-  int B = 0, D = 0, words_ns = 0;
+  int B = 0, D = 0, words_v = 0;
   DevConfigs c;
   RowCtx* ctx = nullptr;
   RowRanges* rng = nullptr;
@@ -1369,11 +1368,20 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   t.Vp = (hv.V + 3) & ~3;
   std::vector<int32_t> spell_of_id_p(hv.spell_of_id);
   spell_of_id_p.resize(t.Vp, -1);
+  // the ids of each spelling (aliases), for the walks' id-indexed verdicts
+  std::vector<int32_t> id_of_spell(std::max(1, t.NS), -1), next_alias(t.Vp, -1);
+  for (int id = t.Vp - 1; id >= 0; --id) {
+    const int sp = spell_of_id_p[id];
+    if (sp < 0) continue;
+    next_alias[id] = id_of_spell[sp];
+    id_of_spell[sp] = id;
+  }
   if ((rc = a.upload(h.lx_cstart, &t.lx_cstart)) || (rc = a.upload(h.lx_cbyte, &t.lx_cbyte)) ||
       (rc = a.upload(h.lx_cnode, &t.lx_cnode)) || (rc = a.upload(h.lx_pcats, &t.lx_pcats)) ||
       (rc = a.upload(h.lx_wcats, &t.lx_wcats)) || (rc = a.upload(hv.spell_off, &t.spell_off)) ||
       (rc = a.upload(hv.spell_bytes, &t.spell_bytes)) ||
-      (rc = a.upload(spell_of_id_p, &t.spell_of_id)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
+      (rc = a.upload(spell_of_id_p, &t.spell_of_id)) || (rc = a.upload(id_of_spell, &t.id_of_spell)) ||
+      (rc = a.upload(next_alias, &t.next_alias)) || (rc = a.upload(hv.first_of_byte, &t.first_of_byte)))
     return fail(rc);
   {
     std::vector<uint32_t> s16((size_t)hv.NS * 4, 0u);
@@ -1602,7 +1610,7 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
   auto* c = new grid_configs();
   c->B = B;
   c->D = s->t.D;
-  c->words_ns = (s->t.NS + 31) / 32 + 1;
+  c->words_v = s->t.W;
   c->cap = std::max(1, s->max_cd);
   c->vcap = std::max(1, s->max_vc);
   Arena& a = c->mem;
@@ -1613,8 +1621,8 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
       (rc = a.alloc(B * sizeof(RowCtx), (void**)&c->ctx)) ||
       (rc = a.alloc(B * sizeof(RowRanges), (void**)&c->rng)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->t.nselw) * 4, (void**)&c->sel)) ||
-      (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd0)) ||
-      (rc = a.alloc((size_t)B * c->words_ns * 4, (void**)&c->verd1)) ||
+      (rc = a.alloc((size_t)B * c->words_v * 4, (void**)&c->verd0)) ||
+      (rc = a.alloc((size_t)B * c->words_v * 4, (void**)&c->verd1)) ||
       (rc = a.alloc((size_t)B * 2 * s->t.T1 * 16, (void**)&c->A2)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->vcw) * 4, (void**)&c->vcbits)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->max_cd) * 4, (void**)&c->surv)) ||
@@ -1664,7 +1672,7 @@ struct MaskScratch {
   RowRanges* rng;
   uint32_t *sel, *verd0, *verd1, *A2, *vcbits;
   int32_t *surv, *vsurv;
-  int cap, vcap, words_ns;
+  int cap, vcap, words_v;
 };
 
 // The five kernels of one mask step on `st`; `ev` (6 events or NULL) is
@@ -1674,11 +1682,11 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
   const Tables& t = s->t;
   const int vcw = std::max(1, s->vcw);
   const int n_vcbits = B * 2 * vcw;
-  const size_t zero_words = (size_t)B * m.words_ns * 2 + n_vcbits;
+  const size_t zero_words = (size_t)B * m.words_v * 2 + n_vcbits;
   const int zero_blocks = std::min(128, (int)((zero_words / 8 + kRowWarps * 32 * 4 - 1) / (kRowWarps * 32 * 4)) + 1);
   if (ev) GRID_CUDA(cudaEventRecord(ev[0], st));
   GRID_CUDA(launch_pdl(k_row, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx, m.rng,
-                       m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_ns));
+                       m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
   const int cd_blocks = (s->max_cd + 255) / 256;
   const int vc_blocks = (s->max_vc + 255) / 256;
@@ -1688,12 +1696,12 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
   GRID_CUDA(launch_pdl(k_walk, dim3(s->walk_blocks), dim3(kWalkWarps * 32), t.blob_bytes, st, t, m.ctx,
                        (const RowRanges*)m.rng, (const uint16_t*)c.stack, (const int32_t*)m.surv, m.cap,
                        (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
-                       m.words_ns, B));
+                       m.words_v, B));
   if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
   GRID_CUDA(launch_pdl(k_pack, dim3((t.Vp + 1023) / 1024, (B + kPackRows - 1) / kPackRows), dim3(256),
                        (size_t)kPackRows * 2 * std::max(1, t.nselw) * 4, st, t, m.ctx, (const uint32_t*)m.sel,
                        (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                       m.words_ns, d_mask, d_status, B));
+                       m.words_v, d_mask, d_status, B));
   if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
@@ -1703,7 +1711,7 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
                           void* stream) {
   if (!s || !c || !d_mask || !d_status) return set_error(GRID_E_INVALID_ARG, "grid_masks: bad arguments");
   const MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
-                      c->surv, c->vsurv, c->cap, c->vcap, c->words_ns};
+                      c->surv, c->vsurv, c->cap, c->vcap, c->words_v};
   return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr);
 }
 
@@ -1749,7 +1757,7 @@ struct StaticCarve {
   size_t ctx, rng, sel, verd0, verd1, A2, vcbits, surv, vsurv, total;
 };
 
-StaticCarve carve_static(const grid_spec* s, int B, int words_ns) {
+StaticCarve carve_static(const grid_spec* s, int B, int words_v) {
   StaticCarve c{};
   size_t at = 0;
   auto take = [&](size_t bytes) {
@@ -1760,8 +1768,8 @@ StaticCarve carve_static(const grid_spec* s, int B, int words_ns) {
   c.ctx = take((size_t)B * sizeof(RowCtx));
   c.rng = take((size_t)B * sizeof(RowRanges));
   c.sel = take((size_t)B * 2 * std::max(1, s->t.nselw) * 4);
-  c.verd0 = take((size_t)B * words_ns * 4);
-  c.verd1 = take((size_t)B * words_ns * 4);
+  c.verd0 = take((size_t)B * words_v * 4);
+  c.verd1 = take((size_t)B * words_v * 4);
   c.A2 = take((size_t)B * 2 * s->t.T1 * 16);
   c.vcbits = take((size_t)B * 2 * std::max(1, s->vcw) * 4);
   c.surv = take((size_t)B * 2 * std::max(1, s->max_cd) * 4);
@@ -1789,8 +1797,8 @@ extern "C" int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, co
   if (dev < 0 || dev >= kStaticMaxDevices)
     return set_error(GRID_E_INVALID_ARG, "grid_masks_static: device ordinal " + std::to_string(dev) +
                                              " is beyond the " + std::to_string(kStaticMaxDevices) + " supported");
-  const int words_ns = (t.NS + 31) / 32 + 1;
-  const StaticCarve cv = carve_static(s, B, words_ns);
+  const int words_v = t.W;
+  const StaticCarve cv = carve_static(s, B, words_v);
   if (cv.total > kStaticScratchBytes)
     return set_error(GRID_E_TOO_LARGE, "grid_masks_static: B=" + std::to_string(B) + " needs " +
                                            std::to_string(cv.total) + " bytes of scratch with this spec, more than "
@@ -1820,7 +1828,7 @@ extern "C" int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, co
                       reinterpret_cast<int32_t*>(area + cv.vsurv),
                       std::max(1, s->max_cd),
                       std::max(1, s->max_vc),
-                      words_ns};
+                      words_v};
   // the kernels only read the configurations
   const DevConfigs c{const_cast<uint16_t*>(d_stack), const_cast<int32_t*>(d_depth),
                      const_cast<int32_t*>(d_dfa_state), const_cast<int32_t*>(d_lex_node),
