@@ -872,30 +872,14 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   extern __shared__ __align__(16) uint32_t s_sel[];  // kPackRows * 2 * nselw
   __shared__ int s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
   __shared__ uint32_t s_kill[kPackRows][8];
-  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int base = blockIdx.x * 1024 + warp * 128 + lane * 4;  // this thread's ids base .. base+3
   const int r0 = blockIdx.y * kPackRows;
   const int nr = min(kPackRows, B - r0);
   const int nw = t.nselw;
   const int code_vc = t.ncls + 3, code_walk = t.ncls + 4, code_never = t.ncls + 1;
-  for (int i = threadIdx.x; i < nr; i += blockDim.x) {
-    const RowCtx& rc = ctx[r0 + i];
-    s_tbl[i] = rc.tbl0;
-    s_fl[i] = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
-    s_any[i] = 0;
-  }
-  for (int i = threadIdx.x; i < nr * 8; i += blockDim.x) s_kill[i >> 3][i & 7] = ctx[r0 + (i >> 3)].kill[i & 7];
-  __syncthreads();
-  // class selections; a context that k_row did not select for (a completed
-  // row, sigma' without a forced emission, sigma without a table) reads zeros
-  for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) {
-    const int k = i / (2 * nw), cx = (i / nw) & 1;
-    const int fl = s_fl[k];
-    const bool valid = t.ci_on && !(fl & 4) && (cx ? (fl & 1) : s_tbl[k] >= 0);
-    s_sel[i] = valid ? sel[(size_t)r0 * 2 * nw + i] : 0u;
-  }
-  // per-id data of the four ids (the tables are padded to Vp ids)
+  // per-id data of the four ids (the tables are padded to Vp ids): spec
+  // tables only, read before the wait on the walks
   int sp[4] = {-1, -1, -1, -1}, b0[4] = {0, 0, 0, 0}, cs[4] = {code_never, code_never, code_never, code_never};
   uint32_t vs[4] = {0u, 0u, 0u, 0u};
   const bool have = base < t.Vp;
@@ -912,6 +896,23 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
   }
   const int eos_j = t.eos - base;  // the EOS id's slot in this thread, if 0..3
   if (eos_j >= 0 && eos_j < 4) sp[eos_j] = -1;  // EOS takes only the gate's bit
+  pdl_wait();
+  for (int i = threadIdx.x; i < nr; i += blockDim.x) {
+    const RowCtx& rc = ctx[r0 + i];
+    s_tbl[i] = rc.tbl0;
+    s_fl[i] = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
+    s_any[i] = 0;
+  }
+  for (int i = threadIdx.x; i < nr * 8; i += blockDim.x) s_kill[i >> 3][i & 7] = ctx[r0 + (i >> 3)].kill[i & 7];
+  __syncthreads();
+  // class selections; a context that k_row did not select for (a completed
+  // row, sigma' without a forced emission, sigma without a table) reads zeros
+  for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) {
+    const int k = i / (2 * nw), cx = (i / nw) & 1;
+    const int fl = s_fl[k];
+    const bool valid = t.ci_on && !(fl & 4) && (cx ? (fl & 1) : s_tbl[k] >= 0);
+    s_sel[i] = valid ? sel[(size_t)r0 * 2 * nw + i] : 0u;
+  }
   __syncthreads();
   const int wi = (blockIdx.x * 1024 + warp * 128) / 32 + (lane >> 3);
   for (int k = 0; k < nr; ++k) {
@@ -923,9 +924,16 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
       // the walks' verdicts of this word's ids, both contexts (one coalesced load each)
       const uint32_t wv[2] = {verd0[(size_t)b * words_v + wi] >> (base & 31),
                               (fl & 1) ? verd1[(size_t)b * words_v + wi] >> (base & 31) : 0u};
+      // sigma's class codes and verdict-class indices of the four ids (same
+      // table: an id coded "verdict class" has its index there)
       ushort4 ct = make_ushort4(code_walk, code_walk, code_walk, code_walk);
-      if (tb >= 0) ct = *reinterpret_cast<const ushort4*>(t.cls_by_id + (size_t)tb * t.Vp + base);
+      uint4 vt = make_uint4(0u, 0u, 0u, 0u);
+      if (tb >= 0) {
+        ct = *reinterpret_cast<const ushort4*>(t.cls_by_id + (size_t)tb * t.Vp + base);
+        vt = *reinterpret_cast<const uint4*>(t.vc_by_id + (size_t)tb * t.Vp + base);
+      }
       const int ctv[4] = {ct.x, ct.y, ct.z, ct.w};
+      const uint32_t vtv[4] = {vt.x, vt.y, vt.z, vt.w};
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         if (sp[j] < 0) continue;
@@ -934,7 +942,7 @@ __global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx
         uint32_t bit = (s_sel[(2 * k + cx) * nw + (code >> 5)] >> (code & 31)) & 1u;
         if (code >= code_vc && (!cx || (fl & 1))) {
           if (code == code_vc) {
-            const uint32_t v = cx ? vs[j] : t.vc_by_id[(size_t)tb * t.Vp + base + j];
+            const uint32_t v = cx ? vs[j] : vtv[j];
             bit = (vcbits[((size_t)b * 2 + cx) * vcw + (v >> 5)] >> (v & 31)) & 1u;
           } else {
             bit = (wv[cx] >> j) & 1u;
