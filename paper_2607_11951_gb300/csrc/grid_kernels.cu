@@ -61,6 +61,7 @@ constexpr int kWalkWarps = 8;    // warps per k_walk block
 constexpr int kSpan = 32;        // CD list entries per walk item (one warp batch)
 constexpr int kAdvWarps = 4;     // rows per k_advance block
 constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_row/k_advance
+constexpr int kFilterPer = 4;    // records per k_filter thread
 constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of (up to) this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
@@ -560,10 +561,9 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   if (threadIdx.x == 0) r.status = complete ? GRID_ST_COMPLETE : s_status;
 }
 
-
-
-// grid = (cd_blocks + vc_blocks, B, 2), 256 threads: compact, per row and
-// context, what the walk has to evaluate.
+// grid = (cd_blocks + vc_blocks, B, 2), 256 threads, kFilterPer records per
+// thread (few blocks, all resident at once): compact, per row and context,
+// what the walk has to evaluate.
 //  - blocks x < cd_blocks: the byte-walked CD spellings that a walk could
 //    admit: the class of the first stack-dependent emission must be selected
 //    for the context's allowed set and, for sigma', the first byte must end
@@ -588,29 +588,42 @@ __global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ c
   const bool vc = (int)blockIdx.x >= cd_blocks;
   const int bx = vc ? (int)blockIdx.x - cd_blocks : (int)blockIdx.x;
   const int len = vc ? t.vc_off[tb + 1] - t.vc_off[tb] : t.cd_off[tb + 1] - t.cd_off[tb];
-  if (bx * (int)blockDim.x >= len) return;
-  const int i = bx * blockDim.x + threadIdx.x;
+  const int i0 = bx * (int)blockDim.x * kFilterPer + threadIdx.x;  // records i0 + j * blockDim.x
+  if (i0 - (int)threadIdx.x >= len) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint32_t* csel = sel + ((size_t)b * 2 + cx) * t.nselw;
-  bool pass = false;
-  int s = -1;
-  if (i < len) {
-    if (vc) {
-      s = i;
-      const uint16_t k = t.vc_first[t.vc_off[tb] + i];
-      pass = (csel[k >> 5] >> (k & 31)) & 1u;
-    } else {
-      s = t.cd_list[t.cd_off[tb] + i];
-      const uint16_t k = t.cd_key[t.cd_off[tb] + i];
-      pass = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
-      if (pass && cx == 1 && q != kStart) {
-        const int b0 = (int)(__ldg(&t.spell16[s]).x & 0xFFu);
-        pass = t.next[q * t.C + t.byte_class[b0]] == kDead;
+  bool pass[kFilterPer];
+  int sv[kFilterPer];
+#pragma unroll
+  for (int j = 0; j < kFilterPer; ++j) {
+    const int i = i0 + j * (int)blockDim.x;
+    pass[j] = false;
+    sv[j] = -1;
+    if (i < len) {
+      if (vc) {
+        sv[j] = i;
+        const uint16_t k = t.vc_first[t.vc_off[tb] + i];
+        pass[j] = (csel[k >> 5] >> (k & 31)) & 1u;
+      } else {
+        const int s = t.cd_list[t.cd_off[tb] + i];
+        sv[j] = s;
+        const uint16_t k = t.cd_key[t.cd_off[tb] + i];
+        pass[j] = k == 0xFFFF || ((csel[k >> 5] >> (k & 31)) & 1u);
+        if (pass[j] && cx == 1 && q != kStart) {
+          const int b0 = (int)(__ldg(&t.spell16[s]).x & 0xFFu);
+          pass[j] = t.next[q * t.C + t.byte_class[b0]] == kDead;
+        }
       }
     }
   }
-  const uint32_t bal = __ballot_sync(0xffffffffu, pass);
-  if (lane == 0) s_warp[warp] = __popc(bal);
+  uint32_t bal[kFilterPer];
+  int cnt = 0;
+#pragma unroll
+  for (int j = 0; j < kFilterPer; ++j) {
+    bal[j] = __ballot_sync(0xffffffffu, pass[j]);
+    cnt += __popc(bal[j]);
+  }
+  if (lane == 0) s_warp[warp] = cnt;
   __syncthreads();
   if (threadIdx.x == 0) {
     int tot = 0;
@@ -622,12 +635,12 @@ __global__ void __launch_bounds__(256) k_filter(Tables t, RowCtx* __restrict__ c
     s_base = tot ? atomicAdd(vc ? &r.nvs[cx] : &r.nsurv[cx], tot) : 0;
   }
   __syncthreads();
-  if (pass) {
-    const int at = s_base + s_warp[warp] + __popc(bal & ((1u << lane) - 1u));
-    if (vc)
-      vsurv[((size_t)b * 2 + cx) * vcap + at] = s;
-    else
-      surv[((size_t)b * 2 + cx) * cap + at] = s;
+  int at = s_base + s_warp[warp];
+  int32_t* out = vc ? vsurv + ((size_t)b * 2 + cx) * vcap : surv + ((size_t)b * 2 + cx) * cap;
+#pragma unroll
+  for (int j = 0; j < kFilterPer; ++j) {
+    if (pass[j]) out[at + __popc(bal[j] & ((1u << lane) - 1u))] = sv[j];
+    at += __popc(bal[j]);
   }
 }
 
@@ -1696,8 +1709,8 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
   GRID_CUDA(launch_pdl(k_row, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx, m.rng,
                        m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
-  const int cd_blocks = (s->max_cd + 255) / 256;
-  const int vc_blocks = (s->max_vc + 255) / 256;
+  const int cd_blocks = (s->max_cd + 256 * kFilterPer - 1) / (256 * kFilterPer);
+  const int vc_blocks = (s->max_vc + 256 * kFilterPer - 1) / (256 * kFilterPer);
   GRID_CUDA(launch_pdl(k_filter, dim3(std::max(1, cd_blocks + vc_blocks), B, 2), dim3(256), 0, st, t, m.ctx,
                        (const uint32_t*)m.sel, m.surv, m.cap, m.vsurv, m.vcap, cd_blocks));
   if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
