@@ -16,15 +16,15 @@
 //                 by token id (coalesced in k_pack)
 //
 // Mask step (grid_masks, Def. 4):
-//   k_row    one block per row: A0 = A(sigma) by a set simulation of the reduce
-//            chains; in parallel the forced emission of the pending lexeme
+//   k_row    one block per row: the forced emission of the pending lexeme
 //            (what every token whose first byte ends the lexeme must go
-//            through) -> sigma' and A1 = A(sigma'), and the EOS gate (Sec. 3.2);
-//            the first bytes that end the lexeme; for rows without a table,
-//            the live first-byte ranges that continue it; then per context and
-//            allowed terminal tau the allowed set after shifting tau (walks
-//            simulate nothing before their second shift) and the class
-//            selections
+//            through) -> sigma', and the EOS gate (Sec. 3.2); the first bytes
+//            that end the lexeme; one lane per terminal tau and context runs
+//            tau's reduce chain (A0 = A(sigma), A1 = A(sigma') are the ballots)
+//            and, for allowed tau, the allowed set after shifting tau (walks
+//            simulate nothing before their second shift); then, for rows
+//            without a table, the live first-byte ranges that continue the
+//            lexeme, and the class selections
 //   k_filter per row and context: the byte-walked spellings and the verdict
 //            classes whose first stack-dependent emission can succeed
 //   k_walk   persistent; per row: each surviving verdict class evaluated once
