@@ -44,6 +44,32 @@ def _compare_full(wl, run, rows=None, split=False):
     return bits
 
 
+def _doubled(wl):
+    """The workload with a second id for every spelling: ids V..2V-1 repeat ids
+    0..V-1 as ordinary tokens (the copies of EOS and the specials included),
+    so that every spelling of the original vocabulary has an alias."""
+    w = dict(wl)
+    w["tokens"] = list(wl["tokens"]) + list(wl["tokens"])
+    return w
+
+
+@pytest.mark.parametrize("name", ["tiny", "admin"])
+def test_alias_ids_share_verdicts(name):
+    # alias ids (several ids, one spelling) share one verdict, whichever way
+    # the spelling is decided: a CI class, a verdict class, or a byte walk,
+    # whose verdict the walk sets for every id of the spelling
+    wl0 = configs.tiny_expr(B=16) if name == "tiny" else configs.sql_admin(B=8)
+    wl = _doubled(wl0)
+    run = GpuRun(wl)
+    st = run.build_configs()
+    assert (st == 0).all(), ("grid_advance status", st)
+    bits = _compare_full(wl, run, split=(name == "admin"))
+    V0 = len(wl0["tokens"])
+    own = np.ones(V0, dtype=bool)
+    own[[wl0["eos"]] + list(wl0["specials"])] = False
+    np.testing.assert_array_equal(bits[:, :V0][:, own], bits[:, V0:][:, own])
+
+
 def test_tiny_expr_full_parity():
     wl, run = _run("tiny", configs.tiny_expr)
     _compare_full(wl, run)
