@@ -1097,54 +1097,74 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
 // 1 KB of contiguous bytes (few, long-lived blocks: block scheduling, not
 // memory, bounds a grid of one short block per 256 sectors).  A sector whose
 // tokens are all rejected is written without being read; a mixed sector is
-// read, blended and written; a fully accepted sector is not touched.  Rows
-// whose sectors are not 32-byte aligned, and the ragged end of a row, are
-// done element by element.
+// read, blended and written; a fully accepted sector is not touched.  Each
+// thread takes kApplyBatch sectors at a time, with their mask words loaded
+// together, then their mixed sectors read together, then all stored, so that
+// a thread waits on two rounds of loads per batch instead of two per sector.
+// Rows whose sectors are not 32-byte aligned, and the ragged end of a row,
+// are done element by element.
+constexpr int kApplyBatch = 4;
 template <typename T>
 __global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask, T* __restrict__ logits, int B,
                                                int V, int W, long long stride, int vec_ok) {
   constexpr int E = 32 / sizeof(T);  // elements per sector
   constexpr uint32_t sfull = E == 32 ? 0xFFFFFFFFu : (1u << E) - 1u;
+  constexpr uint32_t fill = sizeof(T) == 4 ? 0xFF800000u : 0xFF80FF80u;  // -inf in every element of a word
   pdl_wait();
   const int b = blockIdx.y;
-  for (int sc = blockIdx.x * blockDim.x + threadIdx.x; sc * E < V; sc += gridDim.x * blockDim.x) {
-    const int e0 = sc * E;
-    const uint32_t word = mask[(size_t)b * W + (e0 >> 5)];
-    const uint32_t sb = (word >> (e0 & 31)) & sfull;
-    T* p = logits + (size_t)b * stride + e0;
-    const int n = min(E, V - e0);
-    if (vec_ok && n == E) {
-      if (sb == 0u) {
-        const uint32_t f = sizeof(T) == 4 ? 0xFF800000u : 0xFF80FF80u;
-        asm volatile("st.global.v8.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1};" ::"l"(p), "r"(f) : "memory");
-      } else if (sb != sfull) {
-        uint32_t u[8];
-        asm volatile("ld.global.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                     : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]), "=r"(u[7])
-                     : "l"(p)
-                     : "memory");
-        if (sizeof(T) == 4) {
+  const int nsec = (V + E - 1) / E;
+  const int step = gridDim.x * blockDim.x;
+  T* row = logits + (size_t)b * stride;
+  for (int s0 = blockIdx.x * blockDim.x + threadIdx.x; s0 < nsec; s0 += kApplyBatch * step) {
+    uint32_t sb[kApplyBatch];
 #pragma unroll
-          for (int k = 0; k < 8; ++k)
-            if (!((sb >> k) & 1u)) u[k] = 0xFF800000u;
+    for (int u = 0; u < kApplyBatch; ++u) {  // the sectors' accept bits
+      const int e0 = (s0 + u * step) * E;
+      sb[u] = s0 + u * step < nsec ? (mask[(size_t)b * W + (e0 >> 5)] >> (e0 & 31)) & sfull : sfull;
+    }
+    uint32_t v[kApplyBatch][8];
+#pragma unroll
+    for (int u = 0; u < kApplyBatch; ++u) {  // mixed whole sectors: read
+      const int e0 = (s0 + u * step) * E;
+      if (vec_ok && e0 + E <= V && sb[u] != 0u && sb[u] != sfull)
+        asm volatile("ld.global.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                     : "=r"(v[u][0]), "=r"(v[u][1]), "=r"(v[u][2]), "=r"(v[u][3]), "=r"(v[u][4]), "=r"(v[u][5]),
+                       "=r"(v[u][6]), "=r"(v[u][7])
+                     : "l"(row + e0)
+                     : "memory");
+    }
+#pragma unroll
+    for (int u = 0; u < kApplyBatch; ++u) {  // blend and store
+      const int e0 = (s0 + u * step) * E;
+      if (s0 + u * step >= nsec || sb[u] == sfull) continue;
+      T* p = row + e0;
+      const int n = min(E, V - e0);
+      if (vec_ok && n == E) {
+        uint32_t w[8];
+        if (sb[u] == 0u) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) w[k] = fill;
+        } else if (sizeof(T) == 4) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) w[k] = ((sb[u] >> k) & 1u) ? v[u][k] : fill;
         } else {
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const uint32_t lo = (sb >> (2 * k)) & 1u, hi = (sb >> (2 * k + 1)) & 1u;
-            u[k] = (lo ? (u[k] & 0xFFFFu) : 0xFF80u) | (hi ? (u[k] & 0xFFFF0000u) : 0xFF800000u);
+            const uint32_t lo = (sb[u] >> (2 * k)) & 1u, hi = (sb[u] >> (2 * k + 1)) & 1u;
+            w[k] = (lo ? (v[u][k] & 0xFFFFu) : 0xFF80u) | (hi ? (v[u][k] & 0xFFFF0000u) : 0xFF800000u);
           }
         }
-        asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(u[0]), "r"(u[1]), "r"(u[2]),
-                     "r"(u[3]), "r"(u[4]), "r"(u[5]), "r"(u[6]), "r"(u[7])
+        asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+                     "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
                      : "memory");
-      }
-    } else {
-      for (int k = 0; k < n; ++k) {
-        if (!((sb >> k) & 1u)) {
-          if (sizeof(T) == 4)
-            reinterpret_cast<uint32_t*>(p)[k] = 0xFF800000u;
-          else
-            reinterpret_cast<uint16_t*>(p)[k] = 0xFF80u;
+      } else {
+        for (int k = 0; k < n; ++k) {
+          if (!((sb[u] >> k) & 1u)) {
+            if (sizeof(T) == 4)
+              reinterpret_cast<uint32_t*>(p)[k] = 0xFF800000u;
+            else
+              reinterpret_cast<uint16_t*>(p)[k] = 0xFF80u;
+          }
         }
       }
     }
