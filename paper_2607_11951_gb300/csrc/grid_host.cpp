@@ -892,9 +892,17 @@ int build_lexicons(const RawGrammar& rg, const grid_lexicon* lex, int n_lex, Hos
     h.cat_term.push_back(it->second);
     h.catmask[it->second >> 5] |= 1u << (it->second & 31);
   }
-  // trie with map children during construction
-  std::vector<std::map<uint8_t, int>> kids(1);
-  std::vector<uint32_t> pc(1, 0), wc(1, 0);
+  // every word, checked against its category's regex, with its category
+  struct Word {
+    const uint8_t* p;
+    int len, cat;
+  };
+  std::vector<Word> all;
+  {
+    size_t n = 0;
+    for (int i = 0; i < n_lex; ++i) n += (size_t)std::max(0, lex[i].n_words);
+    all.reserve(n);
+  }
   for (int i = 0; i < n_lex; ++i) {
     const grid_lexicon& L = lex[i];
     if (!L.category) return set_error(GRID_E_INVALID_ARG, "lexicon without category");
@@ -908,6 +916,7 @@ int build_lexicons(const RawGrammar& rg, const grid_lexicon* lex, int n_lex, Hos
     for (int w = 0; w < L.n_words; ++w) {
       int64_t a = L.offsets[w], b = L.offsets[w + 1];
       if (b <= a) return set_error(GRID_E_INVALID_ARG, "empty or negative-length lexicon word");
+      if (b - a > (1 << 30)) return set_error(GRID_E_TOO_LARGE, "lexicon word longer than 2^30 bytes");
       // W_c subset of R_c: the word must reach a state accepting the category
       int q = kStart;
       for (int64_t k = a; k < b && q != kDead; ++k) q = h.next[(size_t)q * h.C + h.byte_class[L.words[k]]];
@@ -915,52 +924,79 @@ int build_lexicons(const RawGrammar& rg, const grid_lexicon* lex, int n_lex, Hos
         return set_error(GRID_E_LEXICON_NOT_IN_REGEX,
                          "lexicon word '" + std::string((const char*)L.words + a, (size_t)(b - a)) +
                              "' is not in the regex of " + rg.cats[cat]);
-      int node = 0;
-      pc[0] |= 1u << cat;
-      for (int64_t k = a; k < b; ++k) {
-        uint8_t ch = L.words[k];
-        auto f = kids[node].find(ch);
-        if (f == kids[node].end()) {
-          int nn = (int)kids.size();
-          kids.emplace_back();
-          pc.push_back(0);
-          wc.push_back(0);
-          kids[node][ch] = nn;
-          node = nn;
-        } else {
-          node = f->second;
-        }
-        pc[node] |= 1u << cat;
-      }
-      wc[node] |= 1u << cat;
+      all.push_back(Word{L.words + a, (int)(b - a), cat});
     }
   }
-  // flatten in BFS order with sorted children
-  const int N = (int)kids.size();
-  std::vector<int> order{0}, nid(N, -1);
-  nid[0] = 0;
-  for (size_t k = 0; k < order.size(); ++k)
-    for (auto& kv : kids[order[k]]) {
-      nid[kv.second] = (int)order.size();
-      order.push_back(kv.second);
+  // the trie in preorder from the words in byte order: a word adds nodes only
+  // after its longest common prefix with the word before it, so each node's
+  // children appear in increasing byte order
+  std::sort(all.begin(), all.end(), [](const Word& x, const Word& y) {
+    const int c = std::memcmp(x.p, y.p, (size_t)std::min(x.len, y.len));
+    return c != 0 ? c < 0 : x.len < y.len;
+  });
+  size_t bytes = 1;
+  for (const Word& w : all) bytes += (size_t)w.len;  // bounds the node count
+  std::vector<int> parent{-1};
+  std::vector<uint8_t> edge{0};
+  std::vector<uint32_t> pc(1, 0), wc(1, 0);
+  parent.reserve(bytes);
+  edge.reserve(bytes);
+  pc.reserve(bytes);
+  wc.reserve(bytes);
+  std::vector<int> path{0};  // path[d]: the current word's node at depth d
+  const Word* prev = nullptr;
+  for (const Word& w : all) {
+    int l = 0;
+    if (prev)
+      while (l < prev->len && l < w.len && prev->p[l] == w.p[l]) ++l;
+    path.resize(l + 1);
+    for (int k = l; k < w.len; ++k) {
+      path.push_back((int)parent.size());
+      parent.push_back(path[k]);
+      edge.push_back(w.p[k]);
+      pc.push_back(0);
+      wc.push_back(0);
     }
+    const uint32_t bit = 1u << w.cat;
+    for (int k = 0; k <= w.len; ++k) pc[path[k]] |= bit;
+    wc[path[w.len]] |= bit;
+    prev = &w;
+  }
+  // the flat arrays in BFS order with children sorted by byte.  Nodes of one
+  // depth appear in preorder in the order of their prefixes, which is also
+  // their BFS order, so BFS numbering is preorder stably sorted by depth; the
+  // children of a node then get consecutive BFS ids, and listing edges by
+  // their parents' BFS ids lists them by their children's: edge e leads to
+  // BFS node e + 1.
+  const int N = (int)parent.size();
+  std::vector<int> depth(N, 0), at;  // at[d]: next BFS id at depth d
+  int maxd = 0;
+  for (int v = 1; v < N; ++v) {
+    depth[v] = depth[parent[v]] + 1;  // parents come before children in preorder
+    maxd = std::max(maxd, depth[v]);
+  }
+  at.assign(maxd + 2, 0);
+  for (int v = 0; v < N; ++v) ++at[depth[v] + 1];
+  for (int d = 0; d <= maxd; ++d) at[d + 1] += at[d];
+  std::vector<int> bfs(N);
+  for (int v = 0; v < N; ++v) bfs[v] = at[depth[v]]++;
   h.LN = N;
   h.lx_cstart.assign(N + 1, 0);
-  h.lx_cbyte.clear();
-  h.lx_cnode.clear();
+  h.lx_cbyte.assign(std::max(0, N - 1), 0);
+  h.lx_cnode.resize(std::max(0, N - 1));
   h.lx_pcats.assign(N, 0);
   h.lx_wcats.assign(N, 0);
-  for (int k = 0; k < N; ++k) {
-    int o = order[k];
-    h.lx_cstart[k] = (int)h.lx_cbyte.size();
-    for (auto& kv : kids[o]) {
-      h.lx_cbyte.push_back(kv.first);
-      h.lx_cnode.push_back(nid[kv.second]);
+  for (int v = 0; v < N; ++v) {
+    const int k = bfs[v];
+    h.lx_pcats[k] = pc[v];
+    h.lx_wcats[k] = wc[v];
+    if (v > 0) {
+      h.lx_cbyte[k - 1] = edge[v];
+      ++h.lx_cstart[bfs[parent[v]] + 1];  // child counts, summed below
     }
-    h.lx_pcats[k] = pc[o];
-    h.lx_wcats[k] = wc[o];
   }
-  h.lx_cstart[N] = (int)h.lx_cbyte.size();
+  for (int k = 0; k < N; ++k) h.lx_cstart[k + 1] += h.lx_cstart[k];
+  for (int e = 0; e < N - 1; ++e) h.lx_cnode[e] = e + 1;
   return GRID_OK;
 }
 

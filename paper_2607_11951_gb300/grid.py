@@ -114,13 +114,13 @@ def _ptr(t):
 
 def _pack(items):
     """list of bytes -> (contiguous buffer, int64 offsets) kept alive by the caller."""
+    import numpy as np
     data = b"".join(items)
-    offs = [0]
-    for it in items:
-        offs.append(offs[-1] + len(it))
+    offs = np.zeros(len(items) + 1, dtype=np.int64)
+    if items:
+        np.cumsum(np.fromiter(map(len, items), dtype=np.int64, count=len(items)), out=offs[1:])
     buf = ctypes.create_string_buffer(data, max(1, len(data)))
-    arr = (ctypes.c_int64 * len(offs))(*offs)
-    return buf, arr
+    return buf, np.ctypeslib.as_ctypes(offs)
 
 
 # ---------------------------------------------------------------------------
