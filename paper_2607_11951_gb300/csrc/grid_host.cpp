@@ -930,10 +930,26 @@ int build_lexicons(const RawGrammar& rg, const grid_lexicon* lex, int n_lex, Hos
   // the trie in preorder from the words in byte order: a word adds nodes only
   // after its longest common prefix with the word before it, so each node's
   // children appear in increasing byte order
-  std::sort(all.begin(), all.end(), [](const Word& x, const Word& y) {
-    const int c = std::memcmp(x.p, y.p, (size_t)std::min(x.len, y.len));
-    return c != 0 ? c < 0 : x.len < y.len;
-  });
+  {
+    // sort on the first 8 bytes as a big-endian key (zero padded: where two
+    // keys differ they order as the words do), the full comparison only on
+    // equal keys
+    std::vector<std::pair<uint64_t, int>> kv(all.size());
+    for (size_t i = 0; i < all.size(); ++i) {
+      uint64_t key = 0;
+      for (int k = 0; k < 8; ++k) key = (key << 8) | (k < all[i].len ? all[i].p[k] : 0u);
+      kv[i] = {key, (int)i};
+    }
+    std::sort(kv.begin(), kv.end(), [&](const std::pair<uint64_t, int>& x, const std::pair<uint64_t, int>& y) {
+      if (x.first != y.first) return x.first < y.first;
+      const Word &a = all[x.second], &b = all[y.second];
+      const int c = std::memcmp(a.p, b.p, (size_t)std::min(a.len, b.len));
+      return c != 0 ? c < 0 : a.len < b.len;
+    });
+    std::vector<Word> sorted(all.size());
+    for (size_t i = 0; i < all.size(); ++i) sorted[i] = all[kv[i].second];
+    all.swap(sorted);
+  }
   size_t bytes = 1;
   for (const Word& w : all) bytes += (size_t)w.len;  // bounds the node count
   std::vector<int> parent{-1};
@@ -1080,26 +1096,55 @@ extern "C" int grid_load_vocab(const uint8_t* bytes, const int64_t* offsets, int
     if (offsets[t + 1] < offsets[t]) return set_error(GRID_E_VOCAB, "offsets must be non-decreasing");
   if (offsets[V] > (int64_t)1 << 30) return set_error(GRID_E_TOO_LARGE, "vocabulary bytes exceed 2^30");
   if (offsets[V] > 0 && !bytes) return set_error(GRID_E_INVALID_ARG, "bytes is NULL");
-  std::vector<std::pair<std::string, int>> sp;  // (spelling, id)
+  // the non-excluded ids in spelling order (bytes compared unsigned, shorter
+  // first on a common prefix, equal spellings by id), sorted in place on the
+  // caller's buffer
+  std::vector<int> ids;
+  ids.reserve(V);
   for (int t = 0; t < V; ++t) {
     if (excluded[t]) continue;
-    int64_t a = offsets[t], b = offsets[t + 1];
-    if (b == a) return set_error(GRID_E_VOCAB, "token " + std::to_string(t) + " has an empty spelling");
-    sp.push_back({std::string((const char*)bytes + a, (size_t)(b - a)), t});
+    if (offsets[t + 1] == offsets[t])
+      return set_error(GRID_E_VOCAB, "token " + std::to_string(t) + " has an empty spelling");
+    ids.push_back(t);
   }
-  std::sort(sp.begin(), sp.end());
+  auto spell_cmp = [&](int x, int y) {
+    const int64_t nx = offsets[x + 1] - offsets[x], ny = offsets[y + 1] - offsets[y];
+    const int c = std::memcmp(bytes + offsets[x], bytes + offsets[y], (size_t)std::min(nx, ny));
+    return c != 0 ? c : (nx != ny ? (nx < ny ? -1 : 1) : 0);
+  };
+  {
+    // sort on the first 8 bytes as a big-endian key (zero padded: where two
+    // keys differ they order as the spellings do), the full comparison only
+    // on equal keys
+    std::vector<std::pair<uint64_t, int>> kv(ids.size());
+    for (size_t i = 0; i < ids.size(); ++i) {
+      const int t = ids[i];
+      const int64_t n = std::min<int64_t>(8, offsets[t + 1] - offsets[t]);
+      uint64_t key = 0;
+      for (int64_t k = 0; k < 8; ++k) key = (key << 8) | (k < n ? bytes[offsets[t] + k] : 0u);
+      kv[i] = {key, t};
+    }
+    std::sort(kv.begin(), kv.end(), [&](const std::pair<uint64_t, int>& x, const std::pair<uint64_t, int>& y) {
+      if (x.first != y.first) return x.first < y.first;
+      const int c = spell_cmp(x.second, y.second);
+      return c != 0 ? c < 0 : x.second < y.second;
+    });
+    for (size_t i = 0; i < ids.size(); ++i) ids[i] = kv[i].second;
+  }
   auto* v = new grid_vocab();
   HostVocab& h = v->h;
   h.V = V;
   h.eos = eos_id;
   h.spell_of_id.assign(V, -1);
+  h.spell_off.reserve(ids.size() + 1);
   h.spell_off.push_back(0);
-  for (size_t i = 0; i < sp.size(); ++i) {
-    if (i == 0 || sp[i].first != sp[i - 1].first) {
-      h.spell_bytes.insert(h.spell_bytes.end(), sp[i].first.begin(), sp[i].first.end());
+  for (size_t i = 0; i < ids.size(); ++i) {
+    const int t = ids[i];
+    if (i == 0 || spell_cmp(ids[i - 1], t) != 0) {
+      h.spell_bytes.insert(h.spell_bytes.end(), bytes + offsets[t], bytes + offsets[t + 1]);
       h.spell_off.push_back((int32_t)h.spell_bytes.size());
     }
-    h.spell_of_id[sp[i].second] = (int32_t)h.spell_off.size() - 2;
+    h.spell_of_id[t] = (int32_t)h.spell_off.size() - 2;
   }
   h.NS = (int)h.spell_off.size() - 1;
   h.first_of_byte.assign(257, h.NS);
