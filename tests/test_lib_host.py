@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from paper_2607_11951_gb300 import grid as G
@@ -117,3 +118,28 @@ def test_vocab_errors_and_info():
         G.Vocab([b"a", b"", b"<eos>"], 2)
     with pytest.raises(G.GridError):
         G.Vocab([b"a", b"<eos>"], 5)
+
+
+def test_lexicon_trie_and_vocab_sizes_against_python():
+    # the identifier trie has one node per distinct prefix of the lexicon words
+    # (the empty prefix is the root), whichever category they belong to, and
+    # the vocabulary keeps one spelling per distinct non-excluded token
+    rng = np.random.default_rng(5)
+    alpha = b"abcdefghijklmnopqrstuvwxyz_0123456789"
+    def word():
+        n = int(rng.integers(1, 12))
+        w = bytes([alpha[int(rng.integers(0, 26))]]) + bytes(alpha[int(i)] for i in rng.integers(0, len(alpha), n - 1))
+        return w
+    tables = [word() for _ in range(300)]
+    cols = [word() for _ in range(700)] + tables[:50] + [b"a", b"ab", b"abc"]
+    g = G.Grammar(grammar_text("sql"), [], {"TABLE_NAME": tables, "COLUMN_NAME": cols})
+    prefixes = {w[:k] for w in tables + cols for k in range(len(w) + 1)}
+    assert g.info()["lexicon_nodes"] == len(prefixes)
+    toks = [word() for _ in range(3000)] + [b"\x00", b"\xff", b"a\x00", b"<eos>", b"<pad>"]
+    toks += toks[:100]  # aliases
+    eos, specials = toks.index(b"<eos>"), [toks.index(b"<pad>")]
+    v = G.Vocab(toks, eos, specials)
+    kept = {t for i, t in enumerate(toks) if i != eos and i not in specials}
+    info = v.info()
+    assert info["spellings"] == len(kept)
+    assert info["bytes"] == sum(len(t) for t in kept)
