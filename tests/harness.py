@@ -35,7 +35,7 @@ class GpuRun:
         self.torch = torch
         self.wl = wl
         self.dev = torch.device(device)
-        self.grammar = G.Grammar(wl["grammar"], wl["role"], wl["lexicons"])
+        self.grammar = G.Grammar(wl["grammar"], wl["role"], wl["lexicons"], wl.get("max_depth", 4096))
         self.vocab = G.Vocab(wl["tokens"], wl["eos"], wl["specials"])
         self.spec = G.Spec(self.grammar, self.vocab)
         self.V = len(wl["tokens"])
@@ -70,15 +70,23 @@ class GpuRun:
 
 # ---- oracle side (multiprocessing with spawn so CUDA state is never forked) ----
 _OG = None
+_VOCAB = None
 
 
-def _init_worker(grammar, role, lexicons):
-    global _OG
+def _init_worker(grammar, role, lexicons, vocab=None):
+    """Worker set-up: the oracle grammar, and optionally (tokens, eos,
+    specials) so that jobs need not carry the vocabulary."""
+    global _OG, _VOCAB
     _OG = (compile_grammar(grammar, role, lexicons))
+    _VOCAB = vocab
 
 
 def _oracle_rows(args):
-    prefix, tokens, eos, specials, ids = args
+    if len(args) == 2:
+        prefix, ids = args
+        tokens, eos, specials = _VOCAB
+    else:
+        prefix, tokens, eos, specials, ids = args
     og = _OG
     cfg = og.config_from_ids(prefix, tokens, eos, specials)
     if cfg is None:
@@ -113,13 +121,15 @@ def oracle_masks(wl, rows=None, ids_per_row=None, procs=None):
     jobs = []
     for k, r in enumerate(rows):
         ids = None if ids_per_row is None else list(ids_per_row[k])
-        jobs.append((wl["prefixes"][r], wl["tokens"], wl["eos"], wl["specials"], ids))
+        jobs.append((list(wl["prefixes"][r]), ids))
+    vocab = (wl["tokens"], wl["eos"], wl["specials"])
     procs = procs or min(len(jobs), os.cpu_count() or 1)
     if procs <= 1:
-        _init_worker(wl["grammar"], wl["role"], wl["lexicons"])
+        _init_worker(wl["grammar"], wl["role"], wl["lexicons"], vocab)
         return [_oracle_rows(j) for j in jobs]
     ctx = mp.get_context("spawn")
-    with ctx.Pool(procs, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])) as pool:
+    with ctx.Pool(procs, initializer=_init_worker,
+                  initargs=(wl["grammar"], wl["role"], wl["lexicons"], vocab)) as pool:
         return pool.map(_oracle_rows, jobs, chunksize=1)
 
 
@@ -131,10 +141,11 @@ def oracle_masks_split(wl, rows=None, procs=None, parts=8):
     jobs = []
     for r in rows:
         for a, b in zip(bounds[:-1], bounds[1:]):
-            jobs.append((wl["prefixes"][r], wl["tokens"], wl["eos"], wl["specials"], list(range(a, b))))
+            jobs.append((list(wl["prefixes"][r]), list(range(a, b))))
     procs = procs or (os.cpu_count() or 1)
     ctx = mp.get_context("spawn")
-    with ctx.Pool(procs, initializer=_init_worker, initargs=(wl["grammar"], wl["role"], wl["lexicons"])) as pool:
+    with ctx.Pool(procs, initializer=_init_worker,
+                  initargs=(wl["grammar"], wl["role"], wl["lexicons"], (wl["tokens"], wl["eos"], wl["specials"]))) as pool:
         res = pool.map(_oracle_rows, jobs, chunksize=1)
     out = []
     for i in range(len(rows)):

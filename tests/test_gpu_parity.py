@@ -87,45 +87,61 @@ def test_sql_select_only_full_parity():
     assert bits.sum(axis=1).min() > 0
 
 
-@pytest.mark.parametrize("n,depth", [(100, 1), (100, 64), (1000, 8), (16000, 1), (16000, 64)])
-def test_sweep_cells_sampled(n, depth):
-    """Flatness sweep cells at full size: per row, 2,000 random ids plus up to
-    2,000 GPU-admitted ids are recomputed one by one by the oracle."""
-    wl = configs.sql_sweep_cell(n, depth)
-    run = GpuRun(wl)
-    st = run.build_configs()
-    assert (st == 0).all(), st
-    words, status = run.masks()
-    assert (status == 0).all(), status
-    bits = unpack(words, run.V)
-    rng = np.random.default_rng(n + depth)
-    rows = list(range(0, run.B, 4))
-    ids = []
-    for r in rows:
-        adm = np.nonzero(bits[r])[0]
-        pick = np.concatenate([rng.choice(run.V, 2000, replace=False),
-                               rng.choice(adm, min(2000, adm.size), replace=False) if adm.size else []])
-        ids.append(np.unique(pick.astype(np.int64)))
-    want = oracle_masks(wl, rows, ids)
-    for k, r in enumerate(rows):
-        assert want[k] is not None
-        got = bits[r][ids[k]]
-        w = np.asarray(want[k], dtype=np.uint8)
-        assert (got == w).all(), (n, depth, r, ids[k][np.nonzero(got != w)[0][:10]])
+def test_tiny_pick_full_parity():
+    """Pick grammar: a word of both lexicons where both identifier categories
+    are parser-viable is read as the earlier-declared TABLE_NAME."""
+    wl, run = _run("pick", configs.tiny_pick)
+    _compare_full(wl, run)
 
 
-def test_cold_schema_rows_full_parity():
-    """Cold-schema workload (B=256, 50k identifiers): full masks of 16 rows."""
+def test_sql_shared_words_full_parity():
+    """SQL admin workload whose schema shares words between tables and
+    columns; a quarter of the rows end with such a word where a column may
+    stand, so the pending lexeme has two parser-viable candidates."""
+    wl, run = _run("shared", configs.sql_shared)
+    bits = _compare_full(wl, run, split=True)
+    # the priority is observable on these rows: "," after the shared word
+    # is rejected (it was read as a table name, which needs "."), "." admitted
+    comma, dot = wl["tokens"].index(b","), wl["tokens"].index(b".")
+    tail = range(run.B - run.B // 4, run.B)
+    assert all(bits[r][comma] == 0 and bits[r][dot] == 1 for r in tail)
+
+
+SWEEP_N, SWEEP_D = (100, 1000, 4000, 16000), (1, 8, 32, 64)
+
+
+def test_sweep_cells_full_parity():
+    """Flatness sweep at full size: all 16 cells (n x depth) x 32 rows, every
+    row's full V = 128,256 mask against the oracle."""
+    from tests.harness import oracle_masks
+    cells = [(n, d) for d in SWEEP_D for n in SWEEP_N]
+    first = configs.sql_sweep_cell(*cells[0])
+    run = GpuRun(first)
+    merged = dict(first)
+    merged["prefixes"] = []
+    gpu_bits = []
+    for n, d in cells:
+        wl = configs.sql_sweep_cell(n, d)
+        assert wl["tokens"] is first["tokens"] and wl["lexicons"] == first["lexicons"]
+        st = run.build_configs(prefixes=wl["prefixes"])
+        assert (st == 0).all(), (n, d, st)
+        words, status = run.masks()
+        assert (status == 0).all(), (n, d, status)
+        gpu_bits.append(unpack(words, run.V))
+        merged["prefixes"] += list(wl["prefixes"])
+    want = oracle_masks(merged)
+    for c, (n, d) in enumerate(cells):
+        for r in range(run.B):
+            w = want[c * run.B + r]
+            assert w is not None, (n, d, r)
+            diff = np.nonzero(gpu_bits[c][r] != np.asarray(w, dtype=np.uint8))[0]
+            assert diff.size == 0, (n, d, r, diff[:10].tolist())
+
+
+def test_cold_schema_full_parity():
+    """Cold-schema workload (B=256, 50k identifiers): every row's full mask."""
     wl, run = _run("cold", configs.sql_cold_schema)
-    words, status = run.masks()
-    assert (status == 0).all(), status
-    bits = unpack(words, run.V)
-    rows = list(range(0, 256, 16))
-    want = oracle_masks_split(wl, rows)
-    for k, r in enumerate(rows):
-        assert want[k] is not None
-        diff = np.nonzero(bits[r] != np.asarray(want[k], dtype=np.uint8))[0]
-        assert diff.size == 0, (r, diff[:10].tolist())
+    _compare_full(wl, run)
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])

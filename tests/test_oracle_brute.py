@@ -124,6 +124,103 @@ def test_lexicon_grammar_random_longer():
         assert not bad, bad[:10]
 
 
+# ---------------------------------------------------------------------------
+# Pick grammar: a qualified column TABLE_NAME "." COLUMN_NAME beside a bare
+# COLUMN_NAME, so that right after "g" or "," both categories are
+# parser-viable and a word in both lexicons ("ab") is decided by the priority
+# order alone.  Completion set argument: a viable pending lexeme r is finished
+# into a lexicon word r.x, x a suffix of a word (every category lexeme is
+# emitted only as a word); the pick of r.x depends on the stack and the word
+# only, and leaves the parser at one of eight positions, each finished by a
+# tail in Y that starts with a byte ending r.x (variants with and without a
+# leading blank): start -> "g a o ab;", after GET or ',' -> "a o ab;", after
+# a TABLE_NAME of a column -> ".c o ab;", after '.' -> "c o ab;", after a
+# column -> "o ab;", after OF -> "ab;", after the table -> ";", after ';' -> "".
+# ---------------------------------------------------------------------------
+_XP = [b"", b"a", b"b", b"c", b"ab", b"bc", b"abc", b"ba"]
+_YP = [b"", b";", b" ;", b" ab;", b"ab;", b" o ab;", b"o ab;", b" a o ab;", b"a o ab;", b"g a o ab;",
+       b".c o ab;", b" .c o ab;", b"c o ab;", b" c o ab;"]
+_PICK_COMPL = [x + y for x in _XP for y in _YP]
+
+
+def brute_verdicts(bg, alpha: bytes, max_len: int, completions):
+    """(s, s in Prefix(L), s in L) for every s over ``alpha`` with |s| <= max_len.
+    Prefix(L) is prefix-closed, so an extension of a string outside it is
+    outside it too (and outside L) without a completion search."""
+    out, level = [], [b""]
+    for L in range(max_len + 1):
+        nxt = []
+        for s in level:
+            v = bg.in_prefix_L(s, completions(s))
+            out.append((s, v, bg.in_L(s) if v else False))
+            if v and L < max_len:
+                nxt.extend(s + bytes([c]) for c in alpha)
+            elif L < max_len:
+                stack = [s]
+                while stack:  # every extension of s: (False, False)
+                    u = stack.pop()
+                    for c in alpha:
+                        w = u + bytes([c])
+                        out.append((w, False, False))
+                        if len(w) < max_len:
+                            stack.append(w)
+        level = nxt
+    return out
+
+
+def _check_verdicts(og, verdicts):
+    bad = []
+    for s, v_bf, e_bf in verdicts:
+        cfg = og.feed_bytes(og.start_config(), s)
+        if (cfg is not None and og.live_end(cfg)) != v_bf:
+            bad.append(("viable", s))
+        if (cfg is not None and og.eos_ok(cfg)) != e_bf:
+            bad.append(("eos", s))
+    return bad
+
+
+def test_pick_grammar_exhaustive():
+    """Priority order of the contextual pick (Sec. 2; TABLE_NAME before
+    COLUMN_NAME as in the worked example of Sec. 7.1) at points where both
+    candidates are parser-viable."""
+    text = grammar_text("lexpick")
+    og = compile_grammar(text, lexicons=LEX)
+    bg = BruteGrammar(text, lexicons=LEX)
+    verdicts = brute_verdicts(bg, b"abcgo.,; ", 5, lambda s: _PICK_COMPL)
+    assert len(verdicts) == sum(9 ** k for k in range(6))
+    # the pick is observable: a shared word right after "g" is a table and
+    # needs ".", a word of the column lexicon only is a bare column
+    v = {s: (a, b) for s, a, b in verdicts}
+    assert v[b"g ab"] == (True, False) and v[b"g ab."] == (True, False)
+    assert v[b"g ab,"] == (False, False) and v[b"g abo"] == (False, False)
+    assert v[b"g a o"] == (True, False) and v[b"g c,"] == (True, False)
+    bad = _check_verdicts(og, verdicts)
+    assert not bad, bad[:10]
+
+
+def test_pick_grammar_random_sentences():
+    text = grammar_text("lexpick")
+    og = compile_grammar(text, lexicons=LEX)
+    bg = BruteGrammar(text, lexicons=LEX)
+    rng = np.random.default_rng(13)
+    strings = []
+    for _ in range(500):
+        cols = []
+        for _ in range(int(rng.integers(1, 4))):
+            if rng.random() < 0.5:
+                cols.append(["a", "c", "ab"][int(rng.integers(3))])  # "ab" bare: read as a table
+            else:
+                cols.append(["ab", "abc", "ba"][int(rng.integers(3))] + "." + ["a", "ab", "c"][int(rng.integers(3))])
+        s = ("g " + ",".join(cols) + " o " + ["ab", "abc", "ba"][int(rng.integers(3))] + ";").encode()
+        s = s[:int(rng.integers(0, len(s) + 1))]
+        if s and rng.random() < 0.4:
+            i = int(rng.integers(0, len(s)))
+            s = s[:i] + bytes([b"abcgo.,; "[int(rng.integers(9))]]) + s[i + 1:]
+        strings.append(s)
+    bad = _check(og, bg, strings, lambda s: _PICK_COMPL)
+    assert not bad, bad[:10]
+
+
 def test_contextual_pick_shared_word():
     """'ab' is in both lexicons: a column after 'g', a table after 'o'."""
     og = compile_grammar(grammar_text("lexfix"), lexicons=LEX)

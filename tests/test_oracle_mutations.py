@@ -4,9 +4,8 @@ Each case plants one mistake in a freshly compiled oracle -- a dropped step,
 a missing condition, a wrong set, an off-by-one -- and checks that the
 brute-force verdicts of ``test_oracle_brute`` (or the ``re`` pin of the lexer
 DFA) disagree with it.  The unmodified oracle agrees with the same verdicts.
-(Candidate priority is not among them: in these grammars no lexeme has two
-candidates that are viable at the same point, so its order is not observable
-here; the SQL parity tests and the shared-word test cover the pick.)"""
+The candidate priority of the contextual pick is pinned on the pick grammar,
+where a word of both lexicons meets two parser-viable candidates."""
 import functools
 import types
 
@@ -15,13 +14,16 @@ import pytest
 from oracle import compile_grammar
 from oracle.core import Config
 from tests.brute import BruteGrammar
-from tests.test_oracle_brute import LEX, _LEX_COMPL, _expr_completions, _strings
+from tests.test_oracle_brute import LEX, _LEX_COMPL, _PICK_COMPL, _expr_completions, _strings, brute_verdicts
 from workloads import grammar_text
 
 
 @functools.lru_cache(maxsize=None)
 def _brute(name):
     """Brute-force verdicts (viable, in L) of every short string, computed once."""
+    if name == "lexpick":
+        return brute_verdicts(BruteGrammar(grammar_text("lexpick"), lexicons=LEX), b"abcgo.,; ", 4,
+                              lambda s: _PICK_COMPL)
     if name == "expr":
         bg = BruteGrammar(grammar_text("expr"))
         strings, compl = list(_strings(b"a1+*() ", 4)), _expr_completions
@@ -50,6 +52,14 @@ def _lex_bad(og):
     return _disagree(og, "lexfix")
 
 
+def _pick_bad(og):
+    return _disagree(og, "lexpick")
+
+
+def _pick():
+    return compile_grammar(grammar_text("lexpick"), lexicons=LEX)
+
+
 def _expr():
     return compile_grammar(grammar_text("expr"))
 
@@ -61,6 +71,11 @@ def _lex():
 # ---- the mistakes -----------------------------------------------------------
 def m_emit_accepts_prefix_of_word(og):
     og.candidates = lambda q, r: [t for t in sorted(og.dfa.acc[q]) if t not in og.categories or r in og.P[t]]
+
+
+def m_priority_reversed(og):
+    og.candidates = lambda q, r: [t for t in sorted(og.dfa.acc[q], reverse=True)
+                                  if t not in og.categories or r in og.W[t]]
 
 
 def m_emit_ignores_lexicon(og):
@@ -142,6 +157,7 @@ def m_trailing_skips_parser(og):
 CASES = [
     (m_emit_accepts_prefix_of_word, _lex, _lex_bad),
     (m_emit_ignores_lexicon, _lex, _lex_bad),
+    (m_priority_reversed, _pick, _pick_bad),
     (m_live_ignores_lexicon_prefix, _lex, _lex_bad),
     (m_ignored_needs_shift, _expr, _expr_bad),
     (m_killing_byte_dropped, _expr, _expr_bad),

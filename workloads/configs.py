@@ -11,7 +11,7 @@ import numpy as np
 
 from . import grammar_text, grammar_keywords
 from .gen import (GreedyTokenizer, SqlGen, expr_sentence, expr_vocab, make_schema,
-                  render, sql_vocab)
+                  pick_sentence, render, sql_vocab)
 
 SQL_V_HEADLINE = 151_936
 SQL_V_SWEEP = 128_256
@@ -58,6 +58,28 @@ def tiny_expr(seed: int = 1001, B: int = 64, V: int = 512):
                 seed=seed)
 
 
+PICK_LEXICONS = {"TABLE_NAME": ["ab", "abc", "ba"], "COLUMN_NAME": ["a", "ab", "c"]}
+
+
+def tiny_pick(seed: int = 1006, B: int = 64, V: int = 300):
+    """Pick grammar (a bare or qualified column, so that both identifier
+    categories are parser-viable at one point) with the word "ab" in both
+    lexicons; V ids over the alphabet [abcgo.,; ]; B prefixes truncated at a
+    uniformly random byte offset of a random sentence."""
+    rng = np.random.default_rng(seed)
+    toks, eos, specials = expr_vocab(seed, V, n_alias=4, alpha=b"abcgo.,; ")
+    tk = GreedyTokenizer(toks, specials + [eos])
+    prefixes, texts = [], []
+    for _ in range(B):
+        s = pick_sentence(rng).encode()
+        cut = int(rng.integers(0, len(s) + 1))
+        texts.append(s[:cut])
+        prefixes.append(tk.encode(s[:cut]))
+    return dict(name="tiny_pick", grammar=grammar_text("lexpick"), role=None,
+                lexicons={k: list(v) for k, v in PICK_LEXICONS.items()},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B, seed=seed)
+
+
 def _sql_prefixes(rng, gen: SqlGen, tk: GreedyTokenizer, lens):
     prefixes, texts = [], []
     for n in lens:
@@ -96,6 +118,36 @@ def sql_admin(seed: int = 1002, B: int = 32, V: int = SQL_V_ADMIN):
                 lexicons={"TABLE_NAME": tables, "COLUMN_NAME": words},
                 tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
                 seed=seed)
+
+
+def sql_shared(seed: int = 1007, B: int = 32, V: int = SQL_V_ADMIN, shared: int = 8):
+    """SQL admin workload whose schema has ``shared`` column names that are
+    also table names (20 x 10 schema, V=32,000, prefixes of U[20,200]
+    tokens): where a column may stand, both identifier categories are
+    parser-viable and such a word is read as TABLE_NAME, the earlier one."""
+    kws = grammar_keywords(grammar_text("sql"))
+    tables, cols, words = make_schema(seed, 20, 10, kws, col_pool=60, shared=shared)
+    toks, eos, specials = _sql_vocab_cached(V, 1002, 0.0)
+    tk = GreedyTokenizer(toks, specials + [eos])
+    rng = np.random.default_rng(seed + 1)
+    both = sorted(set(tables) & set(words))
+    n_end = B // 4
+    lens = [int(x) for x in rng.integers(20, 201, size=B - n_end)]
+    gen = SqlGen(rng, tables, cols, dml=True)
+    prefixes, texts = _sql_prefixes(rng, gen, tk, lens)
+    # a quarter of the rows end with a shared word where a column may stand,
+    # so that the pending lexeme's two candidates are both parser-viable
+    for k in range(n_end):
+        head = [["select"], ["select", "*", "from", gen.table(), "where"],
+                ["select", gen._pick(gen.all_cols), "from", gen.table(), "order", "by"]][k % 3]
+        text = render(head + [both[k % len(both)]], rng).encode()
+        ids = tk.encode(text)
+        prefixes.append(ids)
+        texts.append(b"".join(tk_tokens(tk, ids)))
+    return dict(name="sql_shared", grammar=grammar_text("sql"), role=["dml"],
+                lexicons={"TABLE_NAME": tables, "COLUMN_NAME": words},
+                tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B,
+                seed=seed, shared=sorted(set(tables) & set(words)))
 
 
 def sql_select_only(seed: int = 1003, B: int = 32, V: int = SQL_V_HEADLINE,

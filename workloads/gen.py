@@ -57,10 +57,13 @@ def snake_names(rng, syl: list[str], count: int, exclude: set, parts=(1, 3)) -> 
     return out
 
 
-def make_schema(seed: int, n_tables: int, n_cols: int, keywords, col_pool: int | None = None):
+def make_schema(seed: int, n_tables: int, n_cols: int, keywords, col_pool: int | None = None,
+                shared: int = 0):
     """Return (tables, table->columns dict, sorted distinct column words).
 
-    Tables and columns are disjoint and never equal a keyword.  ``col_pool``
+    Names never equal a keyword.  Tables and columns are disjoint, except that
+    with ``shared`` > 0 that many column names are also table names (real
+    catalogs have a column ``order`` beside a table ``order``).  ``col_pool``
     bounds the distinct column names (columns repeat across tables, as real
     catalogs do); ``None`` makes every column name distinct."""
     rng = np.random.default_rng(seed)
@@ -69,6 +72,10 @@ def make_schema(seed: int, n_tables: int, n_cols: int, keywords, col_pool: int |
     tables = snake_names(rng, syl, n_tables, kw, parts=(1, 2))
     pool_n = n_tables * n_cols if col_pool is None else col_pool
     pool = snake_names(rng, syl, pool_n, kw | set(tables), parts=(1, 3))
+    if shared:
+        pick = rng.choice(len(tables), size=min(shared, len(tables), pool_n), replace=False)
+        for k, j in enumerate(sorted(int(x) for x in pick)):
+            pool[k] = tables[j]
     cols = {}
     if col_pool is None:
         for i, t in enumerate(tables):
@@ -170,7 +177,11 @@ class SqlGen:
         self.rng = rng
         self.tables = tables
         self.cols = cols
-        self.all_cols = sorted({c for cs in cols.values() for c in cs})
+        # a column name that is also a table name is written qualified
+        # (t.c) where a bare column may stand: there both categories are
+        # parser-viable and the earlier-declared TABLE_NAME is picked
+        ts = set(tables)
+        self.all_cols = sorted({c for cs in cols.values() for c in cs} - ts)
         self.dml = dml
 
     def _p(self, p):
@@ -341,6 +352,31 @@ class SqlGen:
         return out + closers + [";"]
 
 
+def pick_sentence(rng) -> str:
+    """A random sentence of the pick grammar (q -> g cols o TABLE ;, a column
+    bare or qualified) over the lexicons TABLE {ab, abc, ba} and COLUMN
+    {a, ab, c}, with random blanks.  Bare columns are the column-only words;
+    the shared word "ab" appears as a table of a qualified column or after "."."""
+    cols = []
+    for _ in range(int(rng.integers(1, 4))):
+        if rng.random() < 0.5:
+            cols.append([["a", "c"][int(rng.integers(2))]])
+        else:
+            cols.append([["ab", "abc", "ba"][int(rng.integers(3))], ".", ["a", "ab", "c"][int(rng.integers(3))]])
+    lex = ["g"]
+    for i, c in enumerate(cols):
+        if i:
+            lex.append(",")
+        lex.extend(c)
+    lex += ["o", ["ab", "abc", "ba"][int(rng.integers(3))], ";"]
+    out = []
+    for i, t in enumerate(lex):
+        if i:
+            out.append(" " * int(rng.choice([0, 0, 1, 2])))
+        out.append(t)
+    return "".join(out)
+
+
 # --------------------------------------------------------------------------
 # vocabularies
 # --------------------------------------------------------------------------
@@ -458,12 +494,11 @@ def sql_vocab(seed: int, V: int, keywords, multiword_frac: float = 0.0,
     return toks, eos, specials
 
 
-def expr_vocab(seed: int, V: int = 512, n_alias: int = 5):
-    """V ids over the alphabet [a-z0-9+*() ]: its 41 single bytes, distinct
-    random strings of length 2-4 drawn uniformly from it, ``n_alias`` duplicate
-    spellings, and EOS as the last id.  Returns (tokens, eos_id, [])."""
+def expr_vocab(seed: int, V: int = 512, n_alias: int = 5, alpha: bytes = b"abcdefghijklmnopqrstuvwxyz0123456789+*() "):
+    """V ids over the alphabet (default [a-z0-9+*() ]): its single bytes,
+    distinct random strings of length 2-4 drawn uniformly from it, ``n_alias``
+    duplicate spellings, and EOS as the last id.  Returns (tokens, eos_id, [])."""
     rng = np.random.default_rng(seed)
-    alpha = b"abcdefghijklmnopqrstuvwxyz0123456789+*() "
     toks = [bytes([c]) for c in alpha]
     seen = set(toks)
     n_rand = V - 1 - len(alpha) - n_alias
