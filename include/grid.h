@@ -203,6 +203,18 @@ int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
 int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
                void* stream);
 
+/* grid_masks and grid_apply_mask in one pass: writes M(kappa_b) into d_mask
+ * exactly as grid_masks does and, in the same kernel that packs each mask
+ * word, sets d_logits[b*row_stride + t] to -inf where bit t is 0 (accepted
+ * values bit-identical), as grid_apply_mask would on the finished mask; the
+ * logits of a completed row become all -inf.  Fusing the fill into the
+ * packing saves re-reading the mask and one launch per decoding step (Sec. 2
+ * masked decoding, Def. 4).  d_logits: device memory of `dtype`
+ * (GRID_DTYPE_F32 or GRID_DTYPE_BF16), row_stride >= V elements.  The same
+ * scratch and overlap rule as grid_masks.  Enqueue only. */
+int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
+                     void* d_logits, int32_t dtype, int64_t row_stride, void* stream);
+
 /* Measurement hook: with n_events == 5, every later grid_masks on `c` records
  * events[0..4] (cudaEvent_t, created by the caller) on its stream before its
  * first kernel and after each of its four kernels (per-row allowed sets, EOS

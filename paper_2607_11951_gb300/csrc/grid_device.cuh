@@ -81,7 +81,7 @@ struct Bits4 {
 struct Tables {
   int n_term, T1, S, NNT, P, Q, C, n_cat, LN;
   int NS, V, eos, W, D;
-  int Vp;     // V rounded up to a multiple of 4: the row length of the id-indexed tables
+  int Vp;     // V rounded up to a multiple of 32: the row length of the id-indexed tables
   Bits4 ign;  // ignored terminals (the set I)
   Bits4 cm;   // category terminals
   int cat_term[32];
@@ -121,6 +121,7 @@ struct Tables {
   const int32_t* next_alias;   // Vp: the next larger id with the same spelling, -1 after the last
   const int32_t* first_of_byte;
   const uint8_t* first_byte_by_id;
+  const uint32_t* id_valid;    // W words: bit set for the ids with a spelling (not EOS, special or padding)
   // CI tables (one per lexer state in the precomputed set; table 0 = start state)
   int ci_on;
   int n_tbl;

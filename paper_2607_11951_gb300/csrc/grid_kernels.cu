@@ -48,6 +48,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <type_traits>
 #include <unordered_map>
 #include <utility>
 #include <vector>
@@ -62,7 +63,6 @@ constexpr int kSpan = 32;        // CD list entries per walk item (one warp batc
 constexpr int kAdvWarps = 4;     // rows per k_advance block
 constexpr int kStackWin = 1024;  // stacks up to this depth are copied to shared memory in k_row/k_advance
 constexpr int kFilterPer = 4;    // records per k_filter thread
-constexpr int kPackRows = 8;     // rows per k_pack block
 constexpr int kRangeSpan = 32;   // continuing first-byte ranges are walked in items of (up to) this many spellings
 constexpr int kWalkWin = 512;    // k_walk mirrors row stacks up to this depth per warp
 constexpr int kRowWarps = 6;     // k_row: warps per row block
@@ -868,158 +868,229 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
 }
 
-// grid = (ceil(Vp/1024), ceil(B/kPackRows)), 256 threads: four consecutive
-// token ids per thread (vector loads of the id tables) and kPackRows rows per
-// block, whose context (flags, kill bits, class selections) is staged in
-// shared memory.  Per row, a token's code indexes the context's class
-// selection (CI, always, never in one bit test) and only verdict-class and
-// walked codes look further; the eight lanes that hold a mask word's 32 ids
-// combine their 4-bit pieces with shuffles and one of them stores it.  The
-// last block to finish writes every row's status (EMPTY_MASK for a viable row
-// with no bit set).
-__global__ void __launch_bounds__(256) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
-                                              const uint32_t* __restrict__ vcbits, int vcw,
-                                              const uint32_t* __restrict__ verd0, const uint32_t* __restrict__ verd1,
-                                              int words_v, uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
-                                              int B) {
-  extern __shared__ __align__(16) uint32_t s_sel[];  // kPackRows * 2 * nselw
-  __shared__ int s_tbl[kPackRows], s_fl[kPackRows], s_any[kPackRows];
-  __shared__ uint32_t s_kill[kPackRows][8];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int base = blockIdx.x * 1024 + warp * 128 + lane * 4;  // this thread's ids base .. base+3
-  const int r0 = blockIdx.y * kPackRows;
-  const int nr = min(kPackRows, B - r0);
+// grid = (ceil(W / kPackWords), B), kPackWords threads: thread (b, wi) makes
+// mask word wi of row b, the 32 token ids 32 wi .. 32 wi + 31 (the id tables
+// are padded to a multiple of 32 ids, so each thread reads its ids' first
+// bytes and class codes with 16-byte loads).  Per id: the first byte decides
+// the context (it ends the pending lexeme: sigma' and the start state's
+// table; otherwise sigma and the pending state's table, or the walk when the
+// state has none), the class code indexes that context's class selection (CI,
+// always and never in one bit test), and only verdict-class and walked codes
+// look further: the verdict-class bits of the row (staged in shared memory
+// with its class selections) or the walks' verdict word.  The last block of a
+// row writes its status (EMPTY_MASK for a viable row with no bit set).
+//
+// With APPLY (1 = fp32, 2 = bf16 logits) the thread also masks the logits of
+// its 32 ids (Sec. 2 masked decoding, as grid_apply_mask): a 32-byte sector
+// whose ids are all rejected is written with -inf without being read, a mixed
+// sector is read, blended and written, an accepted sector is not touched.
+constexpr int kPackWords = 256;
+template <int APPLY>
+__global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
+                                                     const uint32_t* __restrict__ vcbits, int vcw,
+                                                     const uint32_t* __restrict__ verd0,
+                                                     const uint32_t* __restrict__ verd1, int words_v,
+                                                     uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
+                                                     void* __restrict__ logits, long long stride, int vec_ok) {
+  extern __shared__ __align__(16) uint32_t s_dyn[];  // class selections (2 nselw) | verdict-class bits (2 vcw)
+  __shared__ int s_fl, s_tb, s_any;
+  __shared__ uint32_t s_kill[8];
+  const int b = blockIdx.y;
+  const int wi = blockIdx.x * kPackWords + threadIdx.x;
+  const bool have = wi < t.W;
   const int nw = t.nselw;
-  const int code_vc = t.ncls + 3, code_walk = t.ncls + 4, code_never = t.ncls + 1;
-  // per-id data of the four ids (the tables are padded to Vp ids): spec
-  // tables only, read before the wait on the walks
-  int sp[4] = {-1, -1, -1, -1}, b0[4] = {0, 0, 0, 0}, cs[4] = {code_never, code_never, code_never, code_never};
-  uint32_t vs[4] = {0u, 0u, 0u, 0u};
-  const bool have = base < t.Vp;
+  const int code_vc = t.ncls + 3, code_walk = t.ncls + 4;
+  // spec tables only, read before the wait on the walks: the ids' first
+  // bytes, which ids have a spelling, the start state's class codes
+  uint4 fb4[2], c04[4];
+  uint32_t valid = 0u;
   if (have) {
-    const int4 s4 = *reinterpret_cast<const int4*>(t.spell_of_id + base);
-    const uchar4 f4 = *reinterpret_cast<const uchar4*>(t.first_byte_by_id + base);
-    const ushort4 c4 = *reinterpret_cast<const ushort4*>(t.cls_by_id + base);
-    sp[0] = s4.x, sp[1] = s4.y, sp[2] = s4.z, sp[3] = s4.w;
-    b0[0] = f4.x, b0[1] = f4.y, b0[2] = f4.z, b0[3] = f4.w;
-    cs[0] = c4.x, cs[1] = c4.y, cs[2] = c4.z, cs[3] = c4.w;
+    const uint4* f = reinterpret_cast<const uint4*>(t.first_byte_by_id) + 2 * wi;
+    fb4[0] = f[0];
+    fb4[1] = f[1];
+    const uint4* c = reinterpret_cast<const uint4*>(t.cls_by_id) + 4 * wi;
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (cs[j] == code_vc) vs[j] = t.vc_by_id[base + j];
+    for (int k = 0; k < 4; ++k) c04[k] = c[k];
+    valid = t.id_valid[wi];
   }
-  const int eos_j = t.eos - base;  // the EOS id's slot in this thread, if 0..3
-  if (eos_j >= 0 && eos_j < 4) sp[eos_j] = -1;  // EOS takes only the gate's bit
   pdl_wait();
-  for (int i = threadIdx.x; i < nr; i += blockDim.x) {
-    const RowCtx& rc = ctx[r0 + i];
-    s_tbl[i] = rc.tbl0;
-    s_fl[i] = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
-    s_any[i] = 0;
+  const RowCtx& rc = ctx[b];
+  if (threadIdx.x == 0) {
+    s_tb = rc.tbl0;
+    s_fl = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
+    s_any = 0;
   }
-  for (int i = threadIdx.x; i < nr * 8; i += blockDim.x) s_kill[i >> 3][i & 7] = ctx[r0 + (i >> 3)].kill[i & 7];
+  if (threadIdx.x < 8) s_kill[threadIdx.x] = rc.kill[threadIdx.x];
   __syncthreads();
-  // class selections; a context that k_row did not select for (a completed
-  // row, sigma' without a forced emission, sigma without a table) reads zeros
-  for (int i = threadIdx.x; i < nr * 2 * nw; i += blockDim.x) {
-    const int k = i / (2 * nw), cx = (i / nw) & 1;
-    const int fl = s_fl[k];
-    const bool valid = t.ci_on && !(fl & 4) && (cx ? (fl & 1) : s_tbl[k] >= 0);
-    s_sel[i] = valid ? sel[(size_t)r0 * 2 * nw + i] : 0u;
+  const int fl = s_fl, tb = s_tb;
+  // a context that k_row did not select for (a completed row, sigma' without
+  // a forced emission, sigma without a table) reads zeros
+  {
+    const bool v0 = t.ci_on && !(fl & 4) && tb >= 0, v1 = t.ci_on && !(fl & 4) && (fl & 1);
+    for (int i = threadIdx.x; i < 2 * nw; i += kPackWords)
+      s_dyn[i] = (i < nw ? v0 : v1) ? sel[(size_t)b * 2 * nw + i] : 0u;
+    const uint32_t* vb = vcbits + (size_t)b * 2 * vcw;
+    for (int i = threadIdx.x; i < 2 * vcw; i += kPackWords) s_dyn[2 * nw + i] = vb[i];
   }
   __syncthreads();
-  const int wi = (blockIdx.x * 1024 + warp * 128) / 32 + (lane >> 3);
-  for (int k = 0; k < nr; ++k) {
-    const int b = r0 + k;
-    const int fl = s_fl[k];
-    const int tb = s_tbl[k];
-    uint32_t nib = 0u;
-    if (have && !(fl & 4)) {
-      // the walks' verdicts of this word's ids, both contexts (one coalesced load each)
-      const uint32_t wv[2] = {verd0[(size_t)b * words_v + wi] >> (base & 31),
-                              (fl & 1) ? verd1[(size_t)b * words_v + wi] >> (base & 31) : 0u};
-      // sigma's class codes and verdict-class indices of the four ids (same
-      // table: an id coded "verdict class" has its index there)
-      ushort4 ct = make_ushort4(code_walk, code_walk, code_walk, code_walk);
-      uint4 vt = make_uint4(0u, 0u, 0u, 0u);
-      if (tb >= 0) {
-        ct = *reinterpret_cast<const ushort4*>(t.cls_by_id + (size_t)tb * t.Vp + base);
-        vt = *reinterpret_cast<const uint4*>(t.vc_by_id + (size_t)tb * t.Vp + base);
-      }
-      const int ctv[4] = {ct.x, ct.y, ct.z, ct.w};
-      const uint32_t vtv[4] = {vt.x, vt.y, vt.z, vt.w};
+  const uint32_t* sel0 = s_dyn;
+  const uint32_t* sel1 = s_dyn + nw;
+  const uint32_t* vcb0 = s_dyn + 2 * nw;
+  const uint32_t* vcb1 = s_dyn + 2 * nw + vcw;
+  uint32_t m = 0u;
+  if (have && !(fl & 4)) {
+    const uint32_t wv0 = verd0[(size_t)b * words_v + wi];
+    const uint32_t wv1 = (fl & 1) ? verd1[(size_t)b * words_v + wi] : 0u;
+    uint4 ct4[4];
+    if (tb >= 0) {
+      const uint4* c = reinterpret_cast<const uint4*>(t.cls_by_id + (size_t)tb * t.Vp) + 4 * wi;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        if (sp[j] < 0) continue;
-        const int cx = (s_kill[k][b0[j] >> 5] >> (b0[j] & 31)) & 1u;
-        const int code = cx ? cs[j] : ctv[j];
-        uint32_t bit = (s_sel[(2 * k + cx) * nw + (code >> 5)] >> (code & 31)) & 1u;
-        if (code >= code_vc && (!cx || (fl & 1))) {
-          if (code == code_vc) {
-            const uint32_t v = cx ? vs[j] : vtv[j];
-            bit = (vcbits[((size_t)b * 2 + cx) * vcw + (v >> 5)] >> (v & 31)) & 1u;
+      for (int k = 0; k < 4; ++k) ct4[k] = c[k];
+    }
+    const uint32_t fbw[8] = {fb4[0].x, fb4[0].y, fb4[0].z, fb4[0].w, fb4[1].x, fb4[1].y, fb4[1].z, fb4[1].w};
+    const uint32_t c0w[16] = {c04[0].x, c04[0].y, c04[0].z, c04[0].w, c04[1].x, c04[1].y, c04[1].z, c04[1].w,
+                              c04[2].x, c04[2].y, c04[2].z, c04[2].w, c04[3].x, c04[3].y, c04[3].z, c04[3].w};
+    uint32_t ctw[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) ctw[k] = code_walk | ((uint32_t)code_walk << 16);
+    if (tb >= 0) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        ctw[4 * k] = ct4[k].x;
+        ctw[4 * k + 1] = ct4[k].y;
+        ctw[4 * k + 2] = ct4[k].z;
+        ctw[4 * k + 3] = ct4[k].w;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      if (!((valid >> j) & 1u)) continue;
+      const int by = (fbw[j >> 2] >> ((j & 3) * 8)) & 0xFF;
+      const int cx = (s_kill[by >> 5] >> (by & 31)) & 1u;
+      const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
+      uint32_t bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
+      if (code >= code_vc && (!cx || (fl & 1))) {
+        if (code == code_vc) {
+          const uint32_t v = t.vc_by_id[(size_t)(cx ? 0 : tb) * t.Vp + 32 * wi + j];
+          bit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
+        } else {
+          bit = ((cx ? wv1 : wv0) >> j) & 1u;
+        }
+      }
+      m |= bit << j;
+    }
+    const int ej = t.eos - 32 * wi;
+    if (ej >= 0 && ej < 32 && (fl & 2)) m |= 1u << ej;
+  }
+  if (have) {
+    mask[(size_t)b * t.W + wi] = m;
+    if (m) s_any = 1;
+  }
+  if (APPLY && have) {
+    using T = typename std::conditional<APPLY == 1, uint32_t, uint16_t>::type;
+    constexpr int E = 32 / sizeof(T);  // elements per 32-byte sector
+    constexpr int NS = 32 / E;         // sectors per mask word
+    constexpr uint32_t sfull = E == 32 ? 0xFFFFFFFFu : (1u << E) - 1u;
+    constexpr uint32_t fill = sizeof(T) == 4 ? 0xFF800000u : 0xFF80FF80u;
+    T* row = reinterpret_cast<T*>(logits) + (size_t)b * stride;
+    const int V = t.V;
+    uint32_t v[NS][8];
+#pragma unroll
+    for (int u = 0; u < NS; ++u) {  // mixed whole sectors: read
+      const int e0 = 32 * wi + u * E;
+      const uint32_t sb = (m >> (u * E)) & sfull;
+      if (vec_ok && e0 + E <= V && sb != 0u && sb != sfull)
+        asm volatile("ld.global.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                     : "=r"(v[u][0]), "=r"(v[u][1]), "=r"(v[u][2]), "=r"(v[u][3]), "=r"(v[u][4]), "=r"(v[u][5]),
+                       "=r"(v[u][6]), "=r"(v[u][7])
+                     : "l"(row + e0)
+                     : "memory");
+    }
+#pragma unroll
+    for (int u = 0; u < NS; ++u) {  // blend and store
+      const int e0 = 32 * wi + u * E;
+      const uint32_t sb = (m >> (u * E)) & sfull;
+      if (e0 >= V || sb == sfull) continue;
+      T* p = row + e0;
+      if (vec_ok && e0 + E <= V) {
+        uint32_t w[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (sizeof(T) == 4) {
+            w[k] = ((sb >> k) & 1u) ? v[u][k] : fill;
           } else {
-            bit = (wv[cx] >> j) & 1u;
+            const uint32_t lo = (sb >> (2 * k)) & 1u, hi = (sb >> (2 * k + 1)) & 1u;
+            w[k] = sb == 0u ? fill : (lo ? (v[u][k] & 0xFFFFu) : 0xFF80u) | (hi ? (v[u][k] & 0xFFFF0000u) : 0xFF800000u);
           }
         }
-        nib |= bit << j;
+        asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+                     "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                     : "memory");
+      } else {
+        for (int k = 0; k < E && e0 + k < V; ++k)
+          if (!((sb >> k) & 1u)) p[k] = (T)fill;
       }
-      if (eos_j >= 0 && eos_j < 4 && (fl & 2)) nib |= 1u << eos_j;
-    }
-    uint32_t v = nib << (4 * (lane & 7));
-    v |= __shfl_xor_sync(0xffffffffu, v, 1);
-    v |= __shfl_xor_sync(0xffffffffu, v, 2);
-    v |= __shfl_xor_sync(0xffffffffu, v, 4);
-    if ((lane & 7) == 0 && wi < t.W) {
-      mask[(size_t)b * t.W + wi] = v;
-      if (v) s_any[k] = 1;
     }
   }
   __syncthreads();
-  // one atomic per row counts the block and carries whether it set a bit; the
-  // row's last block writes its status
-  if (threadIdx.x < nr) {
-    const int b = r0 + threadIdx.x;
-    const unsigned long long old =
-        atomicAdd(&ctx[b].pack_done, 1ull + (s_any[threadIdx.x] ? (1ull << 32) : 0ull));
+  // one atomic per block counts the block for its row and carries whether it
+  // set a bit; the row's last block writes the status
+  if (threadIdx.x == 0) {
+    const unsigned long long old = atomicAdd(&ctx[b].pack_done, 1ull + (s_any ? (1ull << 32) : 0ull));
     if ((uint32_t)old == gridDim.x - 1) {
       int st = atomicAdd(&ctx[b].status, 0);
-      if (st == GRID_ST_OK && (old >> 32) == 0ull && !s_any[threadIdx.x]) st = GRID_ST_EMPTY_MASK;
+      if (st == GRID_ST_OK && (old >> 32) == 0ull && !s_any) st = GRID_ST_EMPTY_MASK;
       d_status[b] = st;
     }
   }
 }
 
-// One warp per row; lane 0 feeds the tokens, all lanes copy for out-of-place.
+// One warp per row.  The lanes copy the row's stack for an out-of-place
+// advance and mirror it in shared memory (16-byte accesses when the row
+// stride allows them); lane 0 then feeds the tokens, with its overlay and
+// simulation scratch in shared memory.
 __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs cin, DevConfigs cout,
                                                              const int32_t* __restrict__ tokens, int n_steps,
                                                              int32_t* __restrict__ d_status, int B, int copy) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
-  __shared__ uint16_t s_stk[kAdvWarps][kStackWin];
+  __shared__ __align__(16) uint16_t s_stk[kAdvWarps][kStackWin];
+  __shared__ uint16_t s_lo[kAdvWarps][kMaxOvl], s_ls[kAdvWarps][kMaxOvl];
   stage_tables(t, ts, smem);
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x * kAdvWarps + warp;
   if (b >= B) return;
-  if (copy) {
-    const int d = cin.depth[b];
-    for (int i = lane; i < d; i += 32) cout.stack[(size_t)b * t.D + i] = cin.stack[(size_t)b * t.D + i];
-    if (lane == 0) {
-      cout.depth[b] = d;
-      cout.q[b] = cin.q[b];
-      cout.lx[b] = cin.lx[b];
-      cout.flags[b] = cin.flags[b];
-    }
-    __syncwarp();
-  }
+  const DevConfigs& from = copy ? cin : cout;
+  const int depth0 = from.depth[b];
+  const uint16_t* src = from.stack + (size_t)b * t.D;
   uint16_t* stack = cout.stack + (size_t)b * t.D;
   // the row's stack is mirrored in shared memory while it fits; the global
   // copy is always written and stays authoritative
-  const int depth0 = copy ? cin.depth[b] : cout.depth[b];
-  const uint16_t* src = copy ? cin.stack + (size_t)b * t.D : stack;
   bool use_win = depth0 <= kStackWin;
-  if (use_win)
-    for (int i = lane; i < depth0; i += 32) s_stk[warp][i] = src[i];
+  if (t.D % 8 == 0) {  // rows start on 16-byte boundaries: 8 entries per access
+    const int n8 = (depth0 + 7) >> 3;  // (n8 * 8 <= D: the last access stays inside the row)
+    const uint4* s4 = reinterpret_cast<const uint4*>(src);
+    uint4* d4 = reinterpret_cast<uint4*>(stack);
+    uint4* w4 = reinterpret_cast<uint4*>(s_stk[warp]);
+    for (int i = lane; i < n8; i += 32) {
+      const uint4 v = s4[i];
+      if (copy) d4[i] = v;
+      if (use_win) w4[i] = v;
+    }
+  } else {
+    for (int i = lane; i < depth0; i += 32) {
+      const uint16_t v = src[i];
+      if (copy) stack[i] = v;
+      if (use_win) s_stk[warp][i] = v;
+    }
+  }
+  if (copy && lane == 0) {
+    cout.depth[b] = depth0;
+    cout.q[b] = cin.q[b];
+    cout.lx[b] = cin.lx[b];
+    cout.flags[b] = cin.flags[b];
+  }
   __syncwarp();
   if (lane != 0) return;
   int depth = depth0, q = cout.q[b], lx = cout.lx[b], flags = cout.flags[b];
@@ -1027,7 +1098,7 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
   int status = GRID_ST_OK;
   const int mc = max_chain_of(t);
   Walker w;
-  uint16_t lo[kMaxOvl], ls[kMaxOvl];
+  const LArr lo{s_lo[warp], 1}, ls{s_ls[warp], 1};
   for (int k = 0; k < n_steps; ++k) {
     const int tok = tokens[(size_t)b * n_steps + k];
     if (tok < 0) continue;
@@ -1039,8 +1110,8 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
       status = GRID_ST_TOKEN_NOT_ALLOWED;
       break;
     }
-    walker_init(w, LArr{lo, 1}, LArr{ls, 1}, kMaxOvl, use_win ? s_stk[warp] : stack, depth, nullptr, 0, q, lx, pc,
-                wcat, nullptr, nullptr);
+    walker_init(w, lo, ls, kMaxOvl, use_win ? s_stk[warp] : stack, depth, nullptr, 0, q, lx, pc, wcat, nullptr,
+                nullptr);
     if (tok == t.eos) {
       const int e = eos_gate(ts, w, mc);
       if (e < 0) {
@@ -1264,10 +1335,10 @@ static int set_smem_limits() {
   const int dyn = kMaxStage;
   GRID_CUDA(cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_events, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
-  // k_pack: the class selections of kPackRows rows, two contexts, at most
-  // kClsFirstCode + kPackCodes codes
-  GRID_CUDA(cudaFuncSetAttribute(k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kPackRows * 2 * ((kClsFirstCode + kPackCodes + 31) / 32) * 4));
+  // k_pack: one row's class selections and verdict-class bits, two contexts
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
@@ -1405,10 +1476,18 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     t.root_pc = h.LN > 0 ? h.lx_pcats[0] : 0u;
     t.root_wc = h.LN > 0 ? h.lx_wcats[0] : 0u;
   }
-  // id-indexed tables are padded to Vp ids (a multiple of 4) for 4-id vector loads
-  t.Vp = (hv.V + 3) & ~3;
+  // id-indexed tables are padded to Vp ids (a multiple of 32), so that the
+  // ids of one mask word are read with 16-byte loads
+  t.Vp = (hv.V + 31) & ~31;
   std::vector<int32_t> spell_of_id_p(hv.spell_of_id);
   spell_of_id_p.resize(t.Vp, -1);
+  {
+    std::vector<uint32_t> valid(t.W, 0u);  // ids with a spelling: not EOS, special or padding
+    for (int id = 0; id < hv.V; ++id)
+      if (spell_of_id_p[id] >= 0) valid[id >> 5] |= 1u << (id & 31);
+    int rcv = s->mem.upload(valid, &t.id_valid);
+    if (rcv) return fail(rcv);
+  }
   // the ids of each spelling (aliases), for the walks' id-indexed verdicts
   std::vector<int32_t> id_of_spell(std::max(1, t.NS), -1), next_alias(t.Vp, -1);
   for (int id = t.Vp - 1; id >= 0; --id) {
@@ -1614,6 +1693,9 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   GRID_CUDA(cudaStreamSynchronize(st));
   tmp.release();
   s->n_vc = vcoff.back();
+  if ((size_t)(2 * std::max(1, t.nselw) + 2 * std::max(1, s->vcw)) * 4 > (size_t)kMaxStage)
+    return fail(set_error(GRID_E_TOO_LARGE, "grid_specialize: the class selections and verdict-class bits of one "
+                                            "row exceed the packing kernel's shared memory"));
   s->n1 = (counts[0] + kSpan - 1) / kSpan;
   s->max_cd = *std::max_element(counts.begin(), counts.end());
   int per_sm = 0;
@@ -1716,10 +1798,17 @@ struct MaskScratch {
   int cap, vcap, words_v;
 };
 
-// The five kernels of one mask step on `st`; `ev` (6 events or NULL) is
+// Logits to mask in the same pass as the mask (grid_masks_apply), or none.
+struct FusedLogits {
+  void* p = nullptr;
+  int dtype = GRID_DTYPE_F32;
+  long long stride = 0;
+};
+
+// The four kernels of one mask step on `st`; `ev` (5 events or NULL) is
 // recorded before the first kernel and after each.
 static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, int B, uint32_t* d_mask,
-                        int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev) {
+                        int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg = {}) {
   const Tables& t = s->t;
   const int vcw = std::max(1, s->vcw);
   const int n_vcbits = B * 2 * vcw;
@@ -1739,10 +1828,22 @@ static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScrat
                        (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
                        m.words_v, B));
   if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
-  GRID_CUDA(launch_pdl(k_pack, dim3((t.Vp + 1023) / 1024, (B + kPackRows - 1) / kPackRows), dim3(256),
-                       (size_t)kPackRows * 2 * std::max(1, t.nselw) * 4, st, t, m.ctx, (const uint32_t*)m.sel,
-                       (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                       m.words_v, d_mask, d_status, B));
+  const dim3 pgrid((t.W + kPackWords - 1) / kPackWords, B);
+  const size_t psmem = (size_t)(2 * std::max(1, t.nselw) + 2 * vcw) * 4;
+  const int esz = lg.dtype == GRID_DTYPE_F32 ? 4 : 2;
+  const int vec_ok = lg.p && ((uintptr_t)lg.p % 32 == 0) && ((lg.stride * esz) % 32 == 0);  // 32-byte sectors
+  if (!lg.p)
+    GRID_CUDA(launch_pdl(k_pack<0>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
+                         (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
+                         m.words_v, d_mask, d_status, (void*)nullptr, 0ll, 0));
+  else if (lg.dtype == GRID_DTYPE_F32)
+    GRID_CUDA(launch_pdl(k_pack<1>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
+                         (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
+                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok));
+  else
+    GRID_CUDA(launch_pdl(k_pack<2>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
+                         (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
+                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok));
   if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
@@ -1754,6 +1855,20 @@ extern "C" int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d
   const MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
                       c->surv, c->vsurv, c->cap, c->vcap, c->words_v};
   return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr);
+}
+
+extern "C" int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
+                                void* d_logits, int32_t dtype, int64_t row_stride, void* stream) {
+  if (!s || !c || !d_mask || !d_status || !d_logits || row_stride < s->t.V ||
+      (dtype != GRID_DTYPE_F32 && dtype != GRID_DTYPE_BF16))
+    return set_error(GRID_E_INVALID_ARG, "grid_masks_apply: bad arguments");
+  const MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
+                      c->surv, c->vsurv, c->cap, c->vcap, c->words_v};
+  FusedLogits lg;
+  lg.p = d_logits;
+  lg.dtype = dtype;
+  lg.stride = row_stride;
+  return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr, lg);
 }
 
 extern "C" int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events) {

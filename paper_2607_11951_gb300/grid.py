@@ -24,7 +24,7 @@ GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
-            "grid_advance", "grid_masks", "grid_configs_set_events", "grid_masks_static", "grid_apply_mask", "grid_configs_export"]
+            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_apply_mask", "grid_configs_export"]
 
 
 class GridLibraryMissing(RuntimeError):
@@ -75,6 +75,7 @@ def lib():
         "grid_configs_reset": (I32, [P, P, P]),
         "grid_advance": (I32, [P, P, P, P, I32, P, P]),
         "grid_masks": (I32, [P, P, P, P, P]),
+        "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
         "grid_configs_set_events": (I32, [P, P, I32]),
         "grid_masks_static": (I32, [P, P, P, P, P, P, I32, I32, P, P, P]),
         "grid_apply_mask": (I32, [P, P, I32, I32, I32, I64, P]),
@@ -210,6 +211,16 @@ def grid_masks(spec, cfg, mask, status, stream=None):
     """mask: int32 CUDA tensor [B, ceil(V/32)] (uint32 words); status: int32 [B]."""
     assert mask.is_contiguous() and status.is_contiguous()
     _check(lib().grid_masks(spec, cfg, _ptr(mask), _ptr(status), _stream(stream)))
+
+
+def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
+    """grid_masks plus the -inf fill of ``logits`` (float32 or bfloat16 CUDA
+    tensor [B, >=V], unit stride along V) in the same pass."""
+    import torch
+    dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
+    assert mask.is_contiguous() and status.is_contiguous() and logits.stride(1) == 1
+    _check(lib().grid_masks_apply(spec, cfg, _ptr(mask), _ptr(status), _ptr(logits), dt, logits.stride(0),
+                                  _stream(stream)))
 
 
 def grid_configs_set_events(cfg, events):

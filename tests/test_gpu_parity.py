@@ -170,6 +170,42 @@ def test_masked_logits_bit_exact(dtype):
         assert torch.equal(got.view(iv), ref.view(iv))
 
 
+@pytest.mark.parametrize("name", ["headline", "tiny_ragged"])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_masks_apply_fused_equals_masks_then_apply(name, dtype):
+    """grid_masks_apply: the same mask words and statuses as grid_masks, and
+    the same logits bit for bit as grid_apply_mask on that mask (NaN
+    payloads kept), for 32-byte aligned rows and unaligned strides and a
+    vocabulary whose last mask word is ragged."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    if name == "headline":
+        wl, run = _run("headline", configs.sql_select_only)
+    else:
+        wl = configs.tiny_expr(B=5, V=517)
+        run = GpuRun(wl)
+        assert (run.build_configs() == 0).all()
+    words, status = run.masks()
+    lg = torch.from_numpy(configs.logits(11, run.B, run.V))
+    lg[0, :5] = float("nan")
+    lg[1, 3] = float("nan")
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    iv = torch.int32 if dtype == "f32" else torch.int16
+    for stride in (run.V, run.V + 1, run.V + 16):
+        buf = torch.zeros(run.B, stride, dtype=tdt)
+        buf[:, :run.V] = lg.to(tdt)
+        ref = buf.cuda()
+        G.grid_apply_mask(run.mask, ref[:, :run.V])
+        got = buf.cuda()
+        m2 = torch.zeros_like(run.mask)
+        st2 = torch.full_like(run.status, -1)
+        G.grid_masks_apply(run.spec.h, run.cfg.h, m2, st2, got[:, :run.V])
+        torch.cuda.synchronize()
+        assert (m2.cpu().numpy().view(np.uint32) == words).all()
+        assert (st2.cpu().numpy() == status).all()
+        assert torch.equal(got.cpu().view(iv), ref.cpu().view(iv)), stride
+
+
 def test_advance_semantics_and_status():
     """Out-of-place advance leaves its input alone; a token outside the mask,
     an out-of-range id and a special id give TOKEN_NOT_ALLOWED and keep the
