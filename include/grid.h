@@ -173,8 +173,9 @@ void grid_spec_free(grid_spec* s);
 int grid_spec_info(const grid_spec* s, int64_t out[8]);
 
 /* Create B configurations, all at the start configuration (empty output),
- * with the device scratch that grid_masks needs for B rows.  Allocates device
- * memory and synchronizes.  Free with grid_configs_free. */
+ * with the device scratch that grid_masks needs for B rows (1 <= B <= 65535;
+ * GRID_E_TOO_LARGE above).  Allocates device memory and synchronizes.  Free
+ * with grid_configs_free. */
 int grid_configs_create(const grid_spec* s, int32_t B, grid_configs** out);
 void grid_configs_free(grid_configs* c);
 
@@ -249,13 +250,30 @@ int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_even
  * about 175 KB per row for the SQL grammar at V = 151,936, so about 48 rows).
  * The first call on a device looks up the array's device address (set-up,
  * once per device, with that device current); make that first call before any
- * stream capture.  Every call on a device shares the array: calls whose kernels
+ * stream capture.  The address is kept for the life of the process, so the
+ * device's primary context must stay alive between calls (no
+ * cudaDeviceReset), and calls must run with that primary context current.
+ * B <= 65535 (GRID_E_TOO_LARGE above, as for any scratch that does not fit).  Every call on a device shares the array: calls whose kernels
  * overlap on the GPU (other streams, other threads) race and corrupt each
  * other's masks, so serialize them.  Each call clears what must start at zero
  * itself.  The spec must live on the current device.  Enqueue only. */
 int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, const int32_t* d_depth,
                       const int32_t* d_dfa_state, const int32_t* d_lex_node, const int32_t* d_flags, int32_t B,
                       int32_t stack_stride, uint32_t* d_mask, int32_t* d_status, void* stream);
+
+/* Sec. 6.1 step 6, jump-forward: per row, while the mask of the row's
+ * configuration admits exactly one token id (EOS included), that token is
+ * forced: it is appended to the row's span and the row is advanced by it (in
+ * place), up to max_span tokens (0 <= max_span <= 4096).  On return d_span
+ * [B][max_span] holds each row's forced ids in order (-1 after its span),
+ * d_span_len[B] their count, and d_mask / d_status the mask and status of the
+ * row's final configuration, as grid_masks writes them; a forced token that
+ * cannot be advanced stops the row with grid_advance's status.  Runs one mask
+ * step per span position (max_span + 1 in all) whatever the spans' lengths,
+ * so choose max_span by the longest forced run worth taking.  Uses the
+ * scratch held by `c`; enqueue only. */
+int grid_forced_span(const grid_spec* s, grid_configs* c, int32_t max_span, uint32_t* d_mask, int32_t* d_span,
+                     int32_t* d_span_len, int32_t* d_status, void* stream);
 
 /* Sec. 2 masked decoding: for b < B, t < V, set d_logits[b*row_stride + t] to
  * -inf (fp32 0xFF800000 / bf16 0xFF80) where mask bit t of row b is 0; accepted

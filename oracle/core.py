@@ -213,6 +213,23 @@ class OracleGrammar:
             return None
         return c
 
+    def forced_span(self, cfg: Config, tokens, eos: int, specials=(), max_span: int = 16):
+        """Jump-forward (Sec. 6.1 step 6): while the mask of the configuration
+        has exactly one bit set (over token ids, EOS included), that token is
+        forced: append it and advance.  Returns (span ids, final config)."""
+        span = []
+        while len(span) < max_span and not cfg.complete:
+            m = self.mask(cfg, tokens, eos, specials)
+            if sum(m) != 1:
+                break
+            t = m.index(1)
+            nxt = self.advance(cfg, t, tokens, eos, specials)
+            if nxt is None:
+                break
+            span.append(t)
+            cfg = nxt
+        return span, cfg
+
     def config_from_ids(self, ids, tokens, eos: int, specials=()):
         cfg = self.start_config()
         for t in ids:

@@ -53,7 +53,7 @@
 #include <utility>
 #include <vector>
 
-#include "grid_device.cuh"
+#include "grid_state.cuh"
 
 namespace grid {
 namespace {
@@ -74,46 +74,7 @@ constexpr int kPackCodes = 5;  // ncls + 0 always, +1 never, +2 n/a, +3 verdict 
 constexpr int kWalkRowsCached = 256;  // rows whose queue bounds k_walk keeps in shared memory
 constexpr int kLaneOvl = 32;     // overlay / scratch entries per walk lane (shared memory)
 constexpr int kMaxStage = 96 * 1024;
-
-#define GRID_CUDA(call)                                                                  \
-  do {                                                                                   \
-    cudaError_t e_ = (call);                                                             \
-    if (e_ != cudaSuccess)                                                               \
-      return set_error(GRID_E_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
-  } while (0)
-
-// Per-row scratch of one grid_masks call.
-struct RowCtx {
-  uint32_t A0[4];   // allowed terminals at sigma
-  uint32_t A1[4];   // allowed terminals at sigma' (after the forced emission)
-  int32_t q, lx, depth, tbl0;
-  uint32_t pc0, wc0;  // category bits of the pending lexeme's trie node
-  int32_t emit_ok, eos_ok, status, complete;
-  unsigned long long pack_done;  // k_pack blocks done with the row (low half) and with a set bit (high half)
-  int32_t keep1, m1;
-  int32_t work0;          // next item of the row's walk queue
-  int32_t nrange;         // items over the continuing first-byte ranges (rows without a CI table)
-  int32_t nsurv[2];       // CD spellings that survived k_filter, per context (0: sigma, 1: sigma')
-  int32_t nvs[2];         // verdict classes that survived k_filter, per context
-  int32_t nrng;
-  uint32_t kill[8];  // bit b: first byte b ends the pending lexeme
-  uint16_t ovl1[kMaxOvl];
-};
-
-// Continuing first-byte ranges of a row without a CI table.
-struct RowRanges {
-  int32_t lo[256];
-  int32_t hi[256];
-  int32_t cpre[257];
-};
-
-struct DevConfigs {
-  uint16_t* stack;  // B*D
-  int32_t* depth;
-  int32_t* q;
-  int32_t* lx;
-  int32_t* flags;   // bit 0 = complete
-};
+constexpr int kMaxRows = 65535;  // rows of one configurations object (a grid dimension of the mask kernels)
 
 // ---------------------------------------------------------------------------
 __global__ void k_reset(DevConfigs c, int B, int D) {
@@ -1261,30 +1222,6 @@ static cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
-// ---------------------------------------------------------------------------
-struct Arena {
-  std::vector<void*> owned;
-  template <typename T>
-  int upload(const std::vector<T>& v, const T** out) {
-    void* p = nullptr;
-    size_t n = std::max<size_t>(v.size(), 1) * sizeof(T);
-    GRID_CUDA(cudaMalloc(&p, n));
-    owned.push_back(p);
-    if (!v.empty()) GRID_CUDA(cudaMemcpy(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice));
-    *out = static_cast<const T*>(p);
-    return GRID_OK;
-  }
-  int alloc(size_t n, void** out) {
-    GRID_CUDA(cudaMalloc(out, std::max<size_t>(n, 16)));
-    owned.push_back(*out);
-    return GRID_OK;
-  }
-  void release() {
-    for (void* p : owned) cudaFree(p);
-    owned.clear();
-  }
-};
-
 size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 }  // namespace
@@ -1292,41 +1229,7 @@ size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 using namespace grid;
 
-static int g_sms = 152;  // SM count of the current device, set by grid_specialize
-
-struct grid_spec {
-  const grid_grammar* g = nullptr;
-  const grid_vocab* v = nullptr;
-  Tables t;
-  Arena mem;
-  int device = 0;
-  int sms = 152;
-  int n1 = 0;  // walk chunks of the start state's CD list
-  int walk_blocks = 0;  // persistent k_walk grid: resident blocks per SM x SMs
-  int max_cd = 0;       // longest CD list of a table
-  int vcw = 0;          // words of the largest table's verdict-class bitset
-  int n_vc = 0;         // verdict classes over all tables
-  int max_vc = 0;       // verdict classes of the largest table
-};
-
-constexpr int kMaskKernels = 4;  // k_row, k_filter, k_walk, k_pack
-
-struct grid_configs {
-  int B = 0, D = 0, words_v = 0;
-  DevConfigs c;
-  RowCtx* ctx = nullptr;
-  RowRanges* rng = nullptr;
-  uint32_t* sel = nullptr;
-  uint32_t* verd0 = nullptr;
-  uint32_t* verd1 = nullptr;
-  uint32_t* A2 = nullptr;
-  uint32_t* vcbits = nullptr;
-  int32_t* surv = nullptr;
-  int32_t* vsurv = nullptr;
-  int cap = 0, vcap = 0;
-  cudaEvent_t ev[kMaskKernels + 1] = {};  // optional per-kernel timing events
-  Arena mem;
-};
+int grid::g_sms = 152;  // SM count of the current device, set by grid_specialize
 
 // The dynamic shared-memory cap is a per-function attribute shared by every
 // spec in the process, so it is raised once to the largest staged block
@@ -1729,6 +1632,8 @@ extern "C" void grid_spec_free(grid_spec* s) {
 
 extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs** out) {
   if (!s || !out || B <= 0) return set_error(GRID_E_INVALID_ARG, "grid_configs_create: bad arguments");
+  if (B > kMaxRows)
+    return set_error(GRID_E_TOO_LARGE, "grid_configs_create: more than " + std::to_string(kMaxRows) + " rows");
   *out = nullptr;
   auto* c = new grid_configs();
   c->B = B;
@@ -1749,7 +1654,8 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
       (rc = a.alloc((size_t)B * 2 * s->t.T1 * 16, (void**)&c->A2)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->vcw) * 4, (void**)&c->vcbits)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->max_cd) * 4, (void**)&c->surv)) ||
-      (rc = a.alloc((size_t)B * 2 * c->vcap * 4, (void**)&c->vsurv))) {
+      (rc = a.alloc((size_t)B * 2 * c->vcap * 4, (void**)&c->vsurv)) ||
+      (rc = a.alloc((size_t)B * 4 * 4, (void**)&c->aux))) {
     grid_configs_free(c);
     return rc;
   }
@@ -1776,39 +1682,26 @@ extern "C" int grid_configs_reset(const grid_spec* s, grid_configs* c, void* str
   return GRID_OK;
 }
 
-extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
-                            const int32_t* d_tokens, int32_t n_steps, int32_t* d_status, void* stream) {
-  if (!s || !in || !out || !d_tokens || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
-    return set_error(GRID_E_INVALID_ARG, "grid_advance: bad arguments");
-  const int B = in->B;
-  GRID_CUDA(launch_pdl(k_advance, dim3((B + kAdvWarps - 1) / kAdvWarps), dim3(kAdvWarps * 32), s->t.blob_bytes,
-                       (cudaStream_t)stream, s->t, in->c, out->c, d_tokens, n_steps, d_status, B,
-                       in != out ? 1 : 0));
+int grid::launch_advance(const grid_spec* s, const DevConfigs& in, const DevConfigs& out, int B,
+                         const int32_t* d_tokens, int32_t n_steps, int32_t* d_status, int copy, cudaStream_t st) {
+  GRID_CUDA(launch_pdl(k_advance, dim3((B + kAdvWarps - 1) / kAdvWarps), dim3(kAdvWarps * 32), s->t.blob_bytes, st,
+                       s->t, in, out, d_tokens, n_steps, d_status, B, copy));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
 }
 
-// Buffers of one mask step (owned by a grid_configs, or carved out of the
-// static area of grid_masks_static).
-struct MaskScratch {
-  RowCtx* ctx;
-  RowRanges* rng;
-  uint32_t *sel, *verd0, *verd1, *A2, *vcbits;
-  int32_t *surv, *vsurv;
-  int cap, vcap, words_v;
-};
-
-// Logits to mask in the same pass as the mask (grid_masks_apply), or none.
-struct FusedLogits {
-  void* p = nullptr;
-  int dtype = GRID_DTYPE_F32;
-  long long stride = 0;
-};
+extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_configs* out,
+                            const int32_t* d_tokens, int32_t n_steps, int32_t* d_status, void* stream) {
+  if (!s || !in || !out || !d_tokens || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
+    return set_error(GRID_E_INVALID_ARG, "grid_advance: bad arguments");
+  return launch_advance(s, in->c, out->c, in->B, d_tokens, n_steps, d_status, in != out ? 1 : 0,
+                        (cudaStream_t)stream);
+}
 
 // The four kernels of one mask step on `st`; `ev` (5 events or NULL) is
 // recorded before the first kernel and after each.
-static int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, int B, uint32_t* d_mask,
-                        int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg = {}) {
+int grid::launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, int B, uint32_t* d_mask,
+                       int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg) {
   const Tables& t = s->t;
   const int vcw = std::max(1, s->vcw);
   const int n_vcbits = B * 2 * vcw;
@@ -1942,6 +1835,8 @@ extern "C" int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, co
   if (!s || !d_stack || !d_depth || !d_dfa_state || !d_lex_node || !d_flags || !d_mask || !d_status || B <= 0)
     return set_error(GRID_E_INVALID_ARG, "grid_masks_static: bad arguments");
   const Tables& t = s->t;
+  if (B > kMaxRows)
+    return set_error(GRID_E_TOO_LARGE, "grid_masks_static: more than " + std::to_string(kMaxRows) + " rows");
   if (stack_stride != t.D)
     return set_error(GRID_E_INVALID_ARG, "grid_masks_static: stack_stride " + std::to_string(stack_stride) +
                                              " differs from the grammar's max_depth " + std::to_string(t.D));

@@ -24,7 +24,7 @@ GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
-            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_apply_mask", "grid_configs_export"]
+            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_forced_span", "grid_apply_mask", "grid_configs_export"]
 
 
 class GridLibraryMissing(RuntimeError):
@@ -76,6 +76,7 @@ def lib():
         "grid_advance": (I32, [P, P, P, P, I32, P, P]),
         "grid_masks": (I32, [P, P, P, P, P]),
         "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
+        "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P]),
         "grid_configs_set_events": (I32, [P, P, I32]),
         "grid_masks_static": (I32, [P, P, P, P, P, P, I32, I32, P, P, P]),
         "grid_apply_mask": (I32, [P, P, I32, I32, I32, I64, P]),
@@ -208,9 +209,17 @@ def grid_advance(spec, cin, cout, tokens, status, stream=None):
 
 
 def grid_masks(spec, cfg, mask, status, stream=None):
-    """mask: int32 CUDA tensor [B, ceil(V/32)] (uint32 words); status: int32 [B]."""
-    assert mask.is_contiguous() and status.is_contiguous()
-    _check(lib().grid_masks(spec, cfg, _ptr(mask), _ptr(status), _stream(stream)))
+    """mask: int32 CUDA tensor [B, ceil(V/32)] (uint32 words); status: int32 [B].
+    ``spec`` and ``cfg`` are handles, or Spec / Configs objects (then the
+    shapes are checked against V and B)."""
+    import torch
+    assert mask.is_contiguous() and status.is_contiguous() and mask.is_cuda and status.is_cuda
+    assert mask.dtype == torch.int32 and status.dtype == torch.int32 and mask.dim() == 2
+    B, W = getattr(cfg, "B", None), getattr(spec, "W", None)
+    assert B is None or (mask.shape[0] == B and tuple(status.shape) == (B,)), "mask [B, W] and status [B] expected"
+    assert W is None or mask.shape[1] == W, "mask [B, ceil(V/32)] expected"
+    _check(lib().grid_masks(getattr(spec, "h", spec), getattr(cfg, "h", cfg), _ptr(mask), _ptr(status),
+                            _stream(stream)))
 
 
 def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
@@ -220,6 +229,16 @@ def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
     dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
     assert mask.is_contiguous() and status.is_contiguous() and logits.stride(1) == 1
     _check(lib().grid_masks_apply(spec, cfg, _ptr(mask), _ptr(status), _ptr(logits), dt, logits.stride(0),
+                                  _stream(stream)))
+
+
+def grid_forced_span(spec, cfg, max_span, mask, span, span_len, status, stream=None):
+    """Jump-forward: span int32 CUDA tensor [B, max_span], span_len and status
+    int32 [B], mask int32 [B, W] (the final configurations' masks)."""
+    for x in (mask, span, span_len, status):
+        assert x.is_contiguous()
+    assert span.dim() == 2 and span.shape[1] == max_span
+    _check(lib().grid_forced_span(spec, cfg, max_span, _ptr(mask), _ptr(span), _ptr(span_len), _ptr(status),
                                   _stream(stream)))
 
 
@@ -234,11 +253,20 @@ def grid_masks_static(spec, stack, depth, dfa_state, lex_node, flags, mask, stat
     """grid_masks for callers that cannot allocate: the configurations come as
     device arrays the caller owns (stack: int16/uint16 CUDA tensor [B, max_depth]
     holding uint16 LALR states; depth, dfa_state, lex_node, flags: int32 [B]),
-    and the step's scratch is the library's fixed static device area."""
+    and the step's scratch is the library's fixed static device area.  ``spec``
+    is a Spec (then the mask's width is checked too) or its handle."""
+    import torch
     B = depth.shape[0]
+    dev = stack.device
     for x in (stack, depth, dfa_state, lex_node, flags, mask, status):
-        assert x.is_contiguous()
+        assert x.is_contiguous() and x.is_cuda and x.device == dev, "device tensors on one device expected"
+    for x in (depth, dfa_state, lex_node, flags, status):
+        assert x.dtype == torch.int32 and tuple(x.shape) == (B,), "int32 [B] expected"
     assert stack.dim() == 2 and stack.shape[0] == B and stack.element_size() == 2
+    W = getattr(spec, "W", None)
+    assert mask.dtype == torch.int32 and mask.dim() == 2 and mask.shape[0] == B, "int32 [B, ceil(V/32)] mask expected"
+    assert W is None or mask.shape[1] == W, "int32 [B, ceil(V/32)] mask expected"
+    spec = getattr(spec, "h", spec)
     _check(lib().grid_masks_static(spec, _ptr(stack), _ptr(depth), _ptr(dfa_state), _ptr(lex_node), _ptr(flags),
                                    B, stack.shape[1], _ptr(mask), _ptr(status), _stream(stream)))
 

@@ -116,3 +116,55 @@ def test_masks_static_refuses_batch_beyond_area():
     w, s = _masks_static(run, torch, _state_arrays(run, torch))
     np.testing.assert_array_equal(s, ref_s)
     np.testing.assert_array_equal(w, ref_w)
+
+
+def test_masks_static_headline_and_capacity_boundary():
+    """At the headline vocabulary (V = 151,936) the static call matches
+    grid_masks on the 32 headline rows; the largest batch the area holds
+    (found by the refusals themselves) runs and matches grid_masks, and one
+    row more is refused."""
+    torch = _torch()
+    from paper_2607_11951_gb300 import grid as G
+    run = GpuRun(configs.sql_select_only())
+    assert (run.build_configs() == 0).all()
+    ref_w, ref_s = run.masks()
+    w, s = _masks_static(run, torch, _state_arrays(run, torch))
+    np.testing.assert_array_equal(s, ref_s)
+    np.testing.assert_array_equal(w, ref_w)
+
+    dev = run.dev
+
+    def start_rows(B):
+        return [torch.zeros((B, MAX_DEPTH), dtype=torch.int16, device=dev),
+                torch.ones(B, dtype=torch.int32, device=dev), torch.ones(B, dtype=torch.int32, device=dev),
+                torch.zeros(B, dtype=torch.int32, device=dev), torch.zeros(B, dtype=torch.int32, device=dev)]
+
+    def fits(B):
+        mask = torch.zeros((B, run.W), dtype=torch.int32, device=dev)
+        status = torch.zeros(B, dtype=torch.int32, device=dev)
+        try:
+            G.grid_masks_static(run.spec.h, *start_rows(B), mask, status)
+        except G.GridError as e:
+            assert e.code == GRID_E_TOO_LARGE
+            return None
+        torch.cuda.synchronize()
+        return mask.cpu().numpy().view(np.uint32), status.cpu().numpy()
+
+    lo, hi = 1, 4096
+    assert fits(lo) is not None and fits(hi) is None
+    while hi - lo > 1:
+        mid = (lo + hi) // 2
+        if fits(mid) is None:
+            hi = mid
+        else:
+            lo = mid
+    assert 8 <= lo < 4096
+    w, s = fits(lo)
+    assert fits(lo + 1) is None
+    ref = G.Configs(run.spec, lo)  # every row at the start configuration
+    m = torch.zeros((lo, run.W), dtype=torch.int32, device=dev)
+    st = torch.zeros(lo, dtype=torch.int32, device=dev)
+    G.grid_masks(run.spec.h, ref.h, m, st)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(w, m.cpu().numpy().view(np.uint32))
+    np.testing.assert_array_equal(s, st.cpu().numpy())

@@ -80,6 +80,29 @@ def tiny_pick(seed: int = 1006, B: int = 64, V: int = 300):
                 tokens=toks, eos=eos, specials=specials, prefixes=prefixes, texts=texts, B=B, seed=seed)
 
 
+def forced_pick():
+    """Pick grammar with a small vocabulary that is not byte-complete, so that
+    some configurations admit exactly one token (jump-forward spans)."""
+    toks = [b"g", b" a", b" o", b" ab", b";", b".c", b",", b" ba", b"<eos>"]
+    prefixes = [[], [0], [0, 3], [0, 3, 5], [0, 1], [0, 1, 6], [0, 3, 5, 2], [0, 3, 5, 2, 7], [0, 3, 5, 2, 7, 4]]
+    return dict(name="forced_pick", grammar=grammar_text("lexpick"), role=None,
+                lexicons={k: list(v) for k, v in PICK_LEXICONS.items()},
+                tokens=toks, eos=len(toks) - 1, specials=[], prefixes=prefixes, B=len(prefixes), seed=0)
+
+
+def forced_sql():
+    """SQL SELECT-only projection, a one-table one-column schema and a small
+    vocabulary of blank-led words (not byte-complete): after "select *" the
+    words "from" and the table are forced, after "group" or "order" "by" is."""
+    toks = [b" select", b" *", b" from", b" t", b" where", b" x", b" =", b" 1", b";", b" and", b" or", b" (",
+            b" )", b" count", b"(", b"*", b")", b" order", b" by", b" group", b"<eos>"]
+    prefixes = [[], [0], [0, 1], [0, 1, 2], [0, 1, 2, 3], [0, 5, 2, 3, 4], [0, 5, 2, 3, 17], [0, 5, 2, 3, 19],
+                [0, 13], [0, 13, 14, 15], [0, 1, 2, 3, 8]]
+    return dict(name="forced_sql", grammar=grammar_text("sql"), role=[],
+                lexicons={"TABLE_NAME": ["t"], "COLUMN_NAME": ["x"]},
+                tokens=toks, eos=len(toks) - 1, specials=[], prefixes=prefixes, B=len(prefixes), seed=0)
+
+
 def _sql_prefixes(rng, gen: SqlGen, tk: GreedyTokenizer, lens):
     prefixes, texts = [], []
     for n in lens:
