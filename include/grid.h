@@ -270,10 +270,87 @@ int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, const int32_t
  * row's final configuration, as grid_masks writes them; a forced token that
  * cannot be advanced stops the row with grid_advance's status.  Runs one mask
  * step per span position (max_span + 1 in all) whatever the spans' lengths,
- * so choose max_span by the longest forced run worth taking.  Uses the
- * scratch held by `c`; enqueue only. */
+ * so choose max_span by the longest forced run worth taking.  With audit
+ * enabled on `c`, every forced token is audited (record kind 1, see
+ * grid_audit_append) into d_records [B][max_span] records of 80 bytes (row
+ * b's k-th forced token at d_records + (b * max_span + k) * 80); d_records
+ * must then be given, and must be NULL otherwise.  Uses the scratch held by
+ * `c`; enqueue only. */
 int grid_forced_span(const grid_spec* s, grid_configs* c, int32_t max_span, uint32_t* d_mask, int32_t* d_span,
-                     int32_t* d_span_len, int32_t* d_status, void* stream);
+                     int32_t* d_span_len, int32_t* d_status, uint8_t* d_records, void* stream);
+
+/* ---- audit chain (Sec. 6.4) ----
+ * Every decoding step of a row appends a record, chained by BLAKE2b-128 from
+ * a genesis constant.  Record layout (80 bytes, little-endian):
+ *   0  u64 step           records of the row so far (0, 1, 2, ...)
+ *   8  u64 config_hash    rolling hash of the top stack node of the
+ *                         configuration the step's mask was computed at:
+ *                         H(root) = 0, H(node) = low 64 bits (LE) of
+ *                         BLAKE2b-128(u64 H(parent) || u32 kind || u32 id),
+ *                         (kind, id) the symbol entering the node: (0,
+ *                         terminal index) or (1, rank of the nonterminal's
+ *                         name in byte order among the grammar's nonterminals)
+ *   16 u8[16] mask id     BLAKE2b-128("GRIDmask" || u32 V || u32 chunks ||
+ *                         BLAKE2b-128 of each 1,024-byte chunk of the mask row)
+ *   32 i32 token          the sampled or forced id (the seal: stop reason)
+ *   36 u32 blocked        ids < V the mask rejects (the seal: mode flags)
+ *   40 u32 kind           caller's label (0 sampled, 1 forced, 2 EOS tail by
+ *                         convention), 3 = seal
+ *   44 u8[16] prev        the previous record's hash (genesis for step 0)
+ *   60 u32 zero
+ *   64 u8[16] hash        BLAKE2b-128 of bytes 0..59
+ * The hashes are kept on the device next to the configurations; appending
+ * costs O(1) per push and O(V/32) per record, independent of the position. */
+
+/* Enable auditing on `c`: allocates the node hashes (B x max_depth x 8 bytes)
+ * and the per-row chain heads, hashes every row's current stack and starts a
+ * fresh chain per row.  Synchronizes.  Afterwards grid_advance on `c` keeps
+ * the node hashes (both configurations of an advance must have audit on, or
+ * neither), and grid_configs_reset restarts every row's chain. */
+int grid_configs_enable_audit(const grid_spec* s, grid_configs* c, void* stream);
+
+/* Append one record per row b with d_tokens[b] >= 0 (other rows are left
+ * alone) to d_records + b * 80: the configuration hash of the row as it is
+ * now, the id of d_mask's row b (which must be the mask of that
+ * configuration), the token, the rejected-id count and `kind` (>= 0).  Call
+ * it after the mask step and before grid_advance with the same token.
+ * Enqueue only. */
+int grid_audit_append(const grid_spec* s, grid_configs* c, const uint32_t* d_mask, const int32_t* d_tokens,
+                      int32_t kind, uint8_t* d_records, void* stream);
+
+/* Seal every row's log: a record of kind 3 with the final configuration's
+ * hash, the spec's fingerprint in place of the mask id, d_reason[b] (the stop
+ * reason, caller-defined) as the token and mode_flags as the blocked count,
+ * written to d_records + b * 80.  Enqueue only. */
+int grid_audit_seal(const grid_spec* s, grid_configs* c, const int32_t* d_reason, uint32_t mode_flags,
+                    uint8_t* d_records, void* stream);
+
+/* Chain head (16 bytes) and record count of one row (synchronous). */
+int grid_audit_head(const grid_configs* c, int32_t row, uint8_t* head, uint64_t* n_records);
+
+/* Host-side check of one row's log of n records (host memory, in order): each
+ * record's step is its index, its prev is the previous record's hash (or
+ * `genesis`, NULL = the library's constant), and its hash matches its bytes.
+ * Returns the index of the first record that fails, or -1 when all pass
+ * (a negative GRID_E_* on bad arguments). */
+int64_t grid_audit_verify(const uint8_t* records, int64_t n, const uint8_t* genesis);
+
+/* The genesis constant: BLAKE2b-128 of the 24 bytes "GRID audit chain genesis". */
+int grid_audit_genesis(uint8_t* out16);
+
+/* BLAKE2b (RFC 7693, unkeyed) of n bytes of host memory, out_bytes in 1..64;
+ * the hash the audit chain is built from. */
+int grid_blake2b(const void* data, size_t n, uint8_t* out, int32_t out_bytes);
+
+/* Fingerprint (16 bytes) of exactly one of: a grammar (BLAKE2b-128 of
+ * "GRIDgram", u64 text length, the text, the role list as passed (u64 length
+ * and bytes, or u64 all ones when NULL), u64 lexicon count, per lexicon in
+ * call order u64 name length, name, u64 word count, u64 length and bytes of
+ * each word, then u64 max_depth), a vocabulary (BLAKE2b-128 of "GRIDvoca", u64
+ * V, i64 eos, u64 special count, i64 each special id, then u64 length and
+ * bytes of every token), or a spec (BLAKE2b-128 of "GRIDspec" and the two).
+ * The other two pointers must be NULL. */
+int grid_fingerprint(const grid_grammar* g, const grid_vocab* v, const grid_spec* s, uint8_t* out16);
 
 /* Sec. 2 masked decoding: for b < B, t < V, set d_logits[b*row_stride + t] to
  * -inf (fp32 0xFF800000 / bf16 0xFF80) where mask bit t of row b is 0; accepted

@@ -101,6 +101,9 @@ class LR1:
         init = frozenset([((0, 0), frozenset([self.END]))])
         index = {init: 0}
         states = [init]
+        # the grammar symbol on which each state is entered (a nonterminal
+        # name or a terminal id; None for the start state)
+        self.access = [None]
         self.ACTION = []
         self.GOTO = []
         k = 0
@@ -119,6 +122,7 @@ class LR1:
                 if key not in index:
                     index[key] = len(states)
                     states.append(key)
+                    self.access.append(X)
                 j = index[key]
                 if X in self.is_nt:
                     gto[X] = j

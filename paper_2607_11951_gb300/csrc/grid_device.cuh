@@ -140,6 +140,7 @@ struct Tables {
   const uint32_t* vc_by_id;   // n_tbl * V: verdict class (within its table) of kClsVC spellings
   const uint32_t* cls_sets;   // ncls * 4: terminal set of every class id
   const uint32_t* cls_mask;   // T1 * nselw: bit c of row tau = tau is in class c's set
+  const uint32_t* acc_sym;    // S: the symbol entering each state (audit node hash)
 };
 
 // Membership test in a 4-word set stored in memory.

@@ -20,6 +20,7 @@
 #include <unordered_map>
 #include <vector>
 
+#include "grid_blake2b.cuh"
 #include "grid_internal.h"
 
 namespace grid {
@@ -833,6 +834,19 @@ int build_parser(const RawGrammar& rg, const char* role_keep, HostGrammar& h) {
     for (auto& e : edges)
       if (la[e.s1][e.k1].merge(la[e.s0][e.k0])) ch = true;
   }
+  // the symbol entering each state, for the audit's node hash
+  {
+    std::vector<std::string> ntname(NNT);
+    for (auto& kv : ntid) ntname[kv.second] = kv.first;
+    std::map<std::string, int> rank;  // nts is ordered by name (bytes)
+    for (auto& n : nts) rank.emplace(n, (int)rank.size());
+    h.acc_sym.assign(S, 0xFFFFFFFFu);
+    for (int s = 1; s < S; ++s) {
+      const int it = kernels[s][0], p = it / 256, d = it % 256;  // every kernel item of s > 0 has d >= 1
+      const int X = P[p].rhs[d - 1];
+      h.acc_sym[s] = X < T1 ? (uint32_t)X : ((1u << 16) | (uint32_t)rank.at(ntname[X - T1]));
+    }
+  }
   // tables
   h.T1 = T1;
   h.S = S;
@@ -1059,6 +1073,37 @@ extern "C" int grid_compile(const char* grammar_text, size_t len, const char* ro
     delete g;
     return rc;
   }
+  {
+    // fingerprint of the inputs (the audit seal names the artifacts by it):
+    // BLAKE2b-128 of "GRIDgram", the text, the role list (all ones when
+    // absent), the lexicons in call order and max_depth, lengths as u64
+    Blake2b b;
+    b.init(16);
+    b.update("GRIDgram", 8);
+    b.put_u64(len);
+    b.update(grammar_text, len);
+    if (role_keep) {
+      const size_t n = std::strlen(role_keep);
+      b.put_u64(n);
+      b.update(role_keep, n);
+    } else {
+      b.put_u64(~0ull);
+    }
+    b.put_u64((uint64_t)n_lex);
+    for (int i = 0; i < n_lex; ++i) {
+      const size_t n = std::strlen(lex[i].category);
+      b.put_u64(n);
+      b.update(lex[i].category, n);
+      b.put_u64((uint64_t)lex[i].n_words);
+      for (int w = 0; w < lex[i].n_words; ++w) {
+        const int64_t a = lex[i].offsets[w], z = lex[i].offsets[w + 1];
+        b.put_u64((uint64_t)(z - a));
+        b.update(lex[i].words + a, (size_t)(z - a));
+      }
+    }
+    b.put_u64((uint64_t)h.max_depth);
+    b.final(h.fingerprint);
+  }
   *out = g;
   return GRID_OK;
 }
@@ -1155,6 +1200,22 @@ extern "C" int grid_load_vocab(const uint8_t* bytes, const int64_t* offsets, int
   for (int s = 0; s < h.NS; ++s)
     if (h.spell_off[s + 1] - h.spell_off[s] == 1) ++singles;
   h.byte_complete = singles == 256;
+  {
+    // fingerprint of the inputs: BLAKE2b-128 of "GRIDvoca", V, eos, the
+    // special ids in call order and every spelling, lengths as u64
+    Blake2b b;
+    b.init(16);
+    b.update("GRIDvoca", 8);
+    b.put_u64((uint64_t)V);
+    b.put_u64((uint64_t)(int64_t)eos_id);
+    b.put_u64((uint64_t)n_special);
+    for (int i = 0; i < n_special; ++i) b.put_u64((uint64_t)(int64_t)special_ids[i]);
+    for (int t = 0; t < V; ++t) {
+      b.put_u64((uint64_t)(offsets[t + 1] - offsets[t]));
+      b.update(bytes + offsets[t], (size_t)(offsets[t + 1] - offsets[t]));
+    }
+    b.final(h.fingerprint);
+  }
   *out = v;
   return GRID_OK;
 }

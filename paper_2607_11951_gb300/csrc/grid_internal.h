@@ -52,6 +52,12 @@ struct HostGrammar {
   std::vector<uint32_t> lx_wcats;  // category bits c with node string in W_c
 
   int max_depth = 4096;
+
+  // audit: the symbol entering each LALR state (kind << 16 | id: kind 0 =
+  // terminal id, kind 1 = rank of the nonterminal's name in byte order among
+  // all nonterminals of the grammar text; 0xFFFFFFFF for the start state)
+  std::vector<uint32_t> acc_sym;
+  uint8_t fingerprint[16] = {};  // BLAKE2b-128 of the compile inputs
 };
 
 // Byte trie of the vocabulary (Def. 3), stored as the lexicographically sorted
@@ -66,6 +72,7 @@ struct HostVocab {
   std::vector<int32_t> spell_of_id; // V, -1 for EOS/special
   std::vector<int32_t> first_of_byte;  // 257: spellings with first byte b are [f[b], f[b+1])
   bool byte_complete = false;
+  uint8_t fingerprint[16] = {};  // BLAKE2b-128 of the vocabulary inputs
 };
 
 }  // namespace grid

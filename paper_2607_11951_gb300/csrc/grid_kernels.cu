@@ -81,6 +81,7 @@ __global__ void k_reset(DevConfigs c, int B, int D) {
   int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   c.stack[(size_t)b * D] = 0;
+  if (c.hs) c.hs[(size_t)b * D] = 0;  // H(root) = 0
   c.depth[b] = 1;
   c.q[b] = kStart;
   c.lx[b] = 0;
@@ -1046,6 +1047,11 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
       if (use_win) s_stk[warp][i] = v;
     }
   }
+  if (copy && cout.hs) {  // the node hashes travel with the stack
+    const uint64_t* hsrc = cin.hs + (size_t)b * t.D;
+    uint64_t* hdst = cout.hs + (size_t)b * t.D;
+    for (int i = lane; i < depth0; i += 32) hdst[i] = hsrc[i];
+  }
   if (copy && lane == 0) {
     cout.depth[b] = depth0;
     cout.q[b] = cin.q[b];
@@ -1105,6 +1111,14 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
       break;
     }
     for (int i = 0; i < w.m; ++i) stack[w.keep + i] = w.ovl[i];
+    if (cout.hs) {  // rolling hash of every pushed node: O(1) per push
+      uint64_t* hrow = cout.hs + (size_t)b * t.D;
+      uint64_t hp = hrow[w.keep - 1];
+      for (int i = 0; i < w.m; ++i) {
+        hp = node_hash(hp, t.acc_sym[w.ovl[i]]);
+        hrow[w.keep + i] = hp;
+      }
+    }
     if (use_win && w.keep + w.m <= kStackWin) {
       for (int i = 0; i < w.m; ++i) s_stk[warp][w.keep + i] = w.ovl[i];
     } else {
@@ -1437,7 +1451,16 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   t.n_tbl = (int)tq.size();
   t.ncls = t.ci_on ? (int)ncls : 0;
   t.nselw = (t.ncls + kPackCodes + 31) / 32;
-  if ((rc = a.upload(tq, &t.tbl_q)) || (rc = a.upload(tbl_of_q, &t.tbl_of_q))) return fail(rc);
+  if ((rc = a.upload(tq, &t.tbl_q)) || (rc = a.upload(tbl_of_q, &t.tbl_of_q)) || (rc = a.upload(h.acc_sym, &t.acc_sym)))
+    return fail(rc);
+  {
+    Blake2b fb;
+    fb.init(16);
+    fb.update("GRIDspec", 8);
+    fb.update(h.fingerprint, 16);
+    fb.update(hv.fingerprint, 16);
+    fb.final(s->fingerprint);
+  }
   if ((rc = set_smem_limits())) return fail(rc);
   int dev = 0;
   cudaGetDevice(&dev);
@@ -1679,7 +1702,7 @@ extern "C" int grid_configs_reset(const grid_spec* s, grid_configs* c, void* str
   if (!s || !c) return set_error(GRID_E_INVALID_ARG, "grid_configs_reset: bad arguments");
   k_reset<<<(c->B + 127) / 128, 128, 0, (cudaStream_t)stream>>>(c->c, c->B, c->D);
   GRID_CUDA(cudaGetLastError());
-  return GRID_OK;
+  return audit_reset(s, c, (cudaStream_t)stream);  // a fresh chain for every row, when audit is on
 }
 
 int grid::launch_advance(const grid_spec* s, const DevConfigs& in, const DevConfigs& out, int B,
@@ -1694,6 +1717,8 @@ extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_con
                             const int32_t* d_tokens, int32_t n_steps, int32_t* d_status, void* stream) {
   if (!s || !in || !out || !d_tokens || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
     return set_error(GRID_E_INVALID_ARG, "grid_advance: bad arguments");
+  if ((in->c.hs != nullptr) != (out->c.hs != nullptr))
+    return set_error(GRID_E_INVALID_ARG, "grid_advance: audit must be enabled on both configurations or on neither");
   return launch_advance(s, in->c, out->c, in->B, d_tokens, n_steps, d_status, in != out ? 1 : 0,
                         (cudaStream_t)stream);
 }

@@ -102,9 +102,14 @@ __global__ void k_force_final(int32_t* __restrict__ d_status, const int32_t* __r
 using namespace grid;
 
 extern "C" int grid_forced_span(const grid_spec* s, grid_configs* c, int32_t max_span, uint32_t* d_mask,
-                                int32_t* d_span, int32_t* d_span_len, int32_t* d_status, void* stream) {
+                                int32_t* d_span, int32_t* d_span_len, int32_t* d_status, uint8_t* d_records,
+                                void* stream) {
   if (!s || !c || !d_mask || (!d_span && max_span > 0) || !d_span_len || !d_status || max_span < 0 || max_span > 4096)
     return set_error(GRID_E_INVALID_ARG, "grid_forced_span: bad arguments");
+  const bool audit = c->c.hs != nullptr;
+  if (audit != (d_records != nullptr) && max_span > 0)
+    return set_error(GRID_E_INVALID_ARG, audit ? "grid_forced_span: audit is on: pass the records of the forced tokens"
+                                               : "grid_forced_span: records given but audit is not enabled");
   cudaStream_t st = (cudaStream_t)stream;
   const int B = c->B;
   const MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
@@ -117,6 +122,10 @@ extern "C" int grid_forced_span(const grid_spec* s, grid_configs* c, int32_t max
     if ((rc = launch_masks(s, c->c, m, B, d_mask, d_status, st, nullptr))) return rc;
     k_force<<<(B + 3) / 4, 128, 0, st>>>(d_mask, s->t.W, d_status, d_span, d_span_len, c->aux, B, pos, max_span);
     GRID_CUDA(cudaGetLastError());
+    // every interior token of a span is audited (kind 1), at the configuration
+    // its mask was computed at, before the advance
+    if (audit && (rc = audit_append(s, c, d_mask, c->aux, 1u, d_records + (size_t)pos * 80, (long long)max_span * 80, st)))
+      return rc;
     if ((rc = launch_advance(s, c->c, c->c, B, c->aux, 1, c->aux + 2 * B, 0, st))) return rc;
   }
   if ((rc = launch_masks(s, c->c, m, B, d_mask, d_status, st, nullptr))) return rc;

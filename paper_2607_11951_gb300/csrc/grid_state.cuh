@@ -9,6 +9,7 @@
 #include <string>
 #include <vector>
 
+#include "grid_blake2b.cuh"
 #include "grid_device.cuh"
 
 #define GRID_CUDA(call)                                                                  \
@@ -51,6 +52,7 @@ struct DevConfigs {
   int32_t* q;
   int32_t* lx;
   int32_t* flags;   // bit 0 = complete
+  uint64_t* hs;     // B*D rolling node hashes parallel to the stacks (audit on), or NULL
 };
 
 struct Arena {
@@ -112,6 +114,7 @@ struct grid_spec {
   int vcw = 0;          // words of the largest table's verdict-class bitset
   int n_vc = 0;         // verdict classes over all tables
   int max_vc = 0;       // verdict classes of the largest table
+  uint8_t fingerprint[16] = {};  // BLAKE2b-128 of the grammar and vocabulary fingerprints
 };
 
 struct grid_configs {
@@ -128,6 +131,10 @@ struct grid_configs {
   int32_t* vsurv = nullptr;
   int cap = 0, vcap = 0;
   int32_t* aux = nullptr;  // 4 x B ints of per-row working state for forced spans and reserves
+  // audit chain (grid_configs_enable_audit): node hashes (c.hs), per-row
+  // chain heads (16 bytes) and record counters
+  uint8_t* heads = nullptr;
+  uint64_t* steps = nullptr;
   cudaEvent_t ev[grid::kMaskKernels + 1] = {};  // optional per-kernel timing events
   grid::Arena mem;
 };
@@ -144,5 +151,12 @@ int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, 
 // of place) on `st`.
 int launch_advance(const grid_spec* s, const DevConfigs& in, const DevConfigs& out, int B, const int32_t* d_tokens,
                    int32_t n_steps, int32_t* d_status, int copy, cudaStream_t st);
+
+// Audit chain (grid_audit.cu): a fresh chain and node hashes of the current
+// stacks when audit is enabled on `c` (no-op otherwise), and one record per
+// row with a non-negative token (records at d_records + b * rec_stride).
+int audit_reset(const grid_spec* s, grid_configs* c, cudaStream_t st);
+int audit_append(const grid_spec* s, grid_configs* c, const uint32_t* d_mask, const int32_t* d_tokens, uint32_t kind,
+                 uint8_t* d_records, long long rec_stride, cudaStream_t st);
 
 }  // namespace grid

@@ -24,7 +24,9 @@ GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
-            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_forced_span", "grid_apply_mask", "grid_configs_export"]
+            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_forced_span",
+            "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
+            "grid_audit_genesis", "grid_blake2b", "grid_fingerprint", "grid_apply_mask", "grid_configs_export"]
 
 
 class GridLibraryMissing(RuntimeError):
@@ -76,7 +78,15 @@ def lib():
         "grid_advance": (I32, [P, P, P, P, I32, P, P]),
         "grid_masks": (I32, [P, P, P, P, P]),
         "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
-        "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P]),
+        "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P, P]),
+        "grid_configs_enable_audit": (I32, [P, P, P]),
+        "grid_audit_append": (I32, [P, P, P, P, I32, P, P]),
+        "grid_audit_seal": (I32, [P, P, P, ctypes.c_uint32, P, P]),
+        "grid_audit_head": (I32, [P, I32, P, ctypes.POINTER(ctypes.c_uint64)]),
+        "grid_audit_verify": (I64, [P, I64, P]),
+        "grid_audit_genesis": (I32, [P]),
+        "grid_blake2b": (I32, [P, SZ, P, I32]),
+        "grid_fingerprint": (I32, [P, P, P, P]),
         "grid_configs_set_events": (I32, [P, P, I32]),
         "grid_masks_static": (I32, [P, P, P, P, P, P, I32, I32, P, P, P]),
         "grid_apply_mask": (I32, [P, P, I32, I32, I32, I64, P]),
@@ -232,14 +242,71 @@ def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
                                   _stream(stream)))
 
 
-def grid_forced_span(spec, cfg, max_span, mask, span, span_len, status, stream=None):
+def grid_forced_span(spec, cfg, max_span, mask, span, span_len, status, records=None, stream=None):
     """Jump-forward: span int32 CUDA tensor [B, max_span], span_len and status
-    int32 [B], mask int32 [B, W] (the final configurations' masks)."""
+    int32 [B], mask int32 [B, W] (the final configurations' masks); with audit
+    on, records is a uint8 CUDA tensor [B, max_span, 80]."""
     for x in (mask, span, span_len, status):
         assert x.is_contiguous()
     assert span.dim() == 2 and span.shape[1] == max_span
-    _check(lib().grid_forced_span(spec, cfg, max_span, _ptr(mask), _ptr(span), _ptr(span_len), _ptr(status),
+    rp = ctypes.c_void_p(None) if records is None else _ptr(records)
+    if records is not None:
+        assert records.is_contiguous() and records.numel() == span.shape[0] * max_span * 80
+    _check(lib().grid_forced_span(spec, cfg, max_span, _ptr(mask), _ptr(span), _ptr(span_len), _ptr(status), rp,
                                   _stream(stream)))
+
+
+def grid_configs_enable_audit(spec, cfg, stream=None):
+    _check(lib().grid_configs_enable_audit(spec, cfg, _stream(stream)))
+
+
+def grid_audit_append(spec, cfg, mask, tokens, kind, records, stream=None):
+    """records: uint8 CUDA tensor [B, 80]; tokens int32 [B] (-1 = no record)."""
+    assert records.is_contiguous() and records.shape[-1] == 80 and tokens.is_contiguous()
+    _check(lib().grid_audit_append(spec, cfg, _ptr(mask), _ptr(tokens), kind, _ptr(records), _stream(stream)))
+
+
+def grid_audit_seal(spec, cfg, reason, mode_flags, records, stream=None):
+    assert records.is_contiguous() and records.shape[-1] == 80 and reason.is_contiguous()
+    _check(lib().grid_audit_seal(spec, cfg, _ptr(reason), mode_flags, _ptr(records), _stream(stream)))
+
+
+def grid_audit_head(cfg, row):
+    head = (ctypes.c_uint8 * 16)()
+    n = ctypes.c_uint64()
+    _check(lib().grid_audit_head(cfg, row, head, ctypes.byref(n)))
+    return bytes(head), n.value
+
+
+def grid_audit_verify(records: bytes, genesis: bytes | None = None) -> int:
+    """records: the concatenated 80-byte records of one row, in order."""
+    assert len(records) % 80 == 0
+    buf = ctypes.create_string_buffer(bytes(records), max(1, len(records)))
+    g = None if genesis is None else ctypes.create_string_buffer(genesis, 16)
+    r = lib().grid_audit_verify(buf, len(records) // 80, g)
+    if r < -1:
+        _check(int(r))
+    return int(r)
+
+
+def grid_audit_genesis() -> bytes:
+    out = (ctypes.c_uint8 * 16)()
+    _check(lib().grid_audit_genesis(out))
+    return bytes(out)
+
+
+def grid_blake2b(data: bytes, out_bytes: int = 64) -> bytes:
+    out = (ctypes.c_uint8 * out_bytes)()
+    buf = ctypes.create_string_buffer(data, max(1, len(data)))
+    _check(lib().grid_blake2b(buf, len(data), out, out_bytes))
+    return bytes(out)
+
+
+def grid_fingerprint(grammar=None, vocab=None, spec=None) -> bytes:
+    out = (ctypes.c_uint8 * 16)()
+    h = lambda x: None if x is None else getattr(x, "h", x)
+    _check(lib().grid_fingerprint(h(grammar), h(vocab), h(spec), out))
+    return bytes(out)
 
 
 def grid_configs_set_events(cfg, events):

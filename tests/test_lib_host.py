@@ -24,7 +24,7 @@ def built():
 
 def _declared():
     text = open(os.path.join(ROOT, "include", "grid.h")).read()
-    return sorted(set(re.findall(r"^\s*(?:int|void|size_t)\s+(grid_[a-z_]+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^\s*(?:int|void|size_t|int64_t)\s+(grid_[a-z0-9_]+)\s*\(", text, re.M)))
 
 
 def test_exports_every_declared_symbol():
