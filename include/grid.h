@@ -279,6 +279,31 @@ int grid_masks_static(const grid_spec* s, const uint16_t* d_stack, const int32_t
 int grid_forced_span(const grid_spec* s, grid_configs* c, int32_t max_span, uint32_t* d_mask, int32_t* d_span,
                      int32_t* d_span_len, int32_t* d_status, uint8_t* d_records, void* stream);
 
+/* Sec. 5 Prop. 9 (Termination) and Sec. 6.1 step 3: the token-denominated
+ * reserve of every row -- the cheapest legal completion of the row's output
+ * plus EOS, counted in vocabulary tokens -- so that a decoding loop whose
+ * remaining budget falls to the reserve plus a safety margin writes that
+ * completion instead of sampling (every stop then lies in L).
+ * Cost model (the paper's: terminal costs in tokens, summed over a
+ * completion): terminal tau is written as a blank and its lexeme l(tau) (the
+ * shortest, then bytewise smallest, string whose first emission candidate is
+ * tau; a lexicon word for a category), split greedily into vocabulary tokens;
+ * the pending lexeme either ends as it stands or is first extended, in
+ * single-byte tokens, to one live terminal's shortest lexeme, then ends by
+ * the blank of the first rendering (or the lexer state's separator byte, a
+ * token of its own); the completion's terminals minimise the summed
+ * rendering lengths exactly (over the LR items of the stack, see
+ * grid_span.cu).  Writes d_cost[b] = tokens of the completion including EOS
+ * (0 for a completed row, -1 when none exists) and the tokens themselves to
+ * d_tokens[b*cap ...] (-1 after them); d_status[b] = GRID_ST_OK,
+ * GRID_ST_COMPLETE, GRID_ST_NONVIABLE (no completion under this cost model)
+ * or GRID_ST_BOUND (the completion is longer than cap -- d_cost still holds
+ * its length -- or the search space of a very deep stack ran out).  With
+ * d_budget given, d_fire[b] = 1 when d_budget[b] <= d_cost[b] + safety (the
+ * reserve trigger), else 0.  Uses the scratch held by `c`; enqueue only. */
+int grid_reserve(const grid_spec* s, const grid_configs* c, int32_t* d_cost, int32_t* d_tokens, int32_t cap,
+                 int32_t* d_status, const int32_t* d_budget, int32_t safety, int32_t* d_fire, void* stream);
+
 /* ---- audit chain (Sec. 6.4) ----
  * Every decoding step of a row appends a record, chained by BLAKE2b-128 from
  * a genesis constant.  Record layout (80 bytes, little-endian):

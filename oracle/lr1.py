@@ -104,6 +104,7 @@ class LR1:
         # the grammar symbol on which each state is entered (a nonterminal
         # name or a terminal id; None for the start state)
         self.access = [None]
+        self.kernel_states = states  # kernel items (core, lookaheads) of each state
         self.ACTION = []
         self.GOTO = []
         k = 0

@@ -103,7 +103,22 @@ struct Blake2b {
   }
   GRID_HD void update(const void* p, size_t n) {
     const uint8_t* b = static_cast<const uint8_t*>(p);
-    for (size_t i = 0; i < n; ++i) put_byte(b[i]);
+    size_t i = 0;
+    while (i < n && (fill & 7)) put_byte(b[i++]);  // to a word boundary
+    // whole little-endian words while the block has room and input follows it
+    for (; i + 8 <= n; i += 8) {
+      if (fill == 128) {
+        t += 128;
+        blake2b_compress(h, buf, t, false);
+        for (int k = 0; k < 16; ++k) buf[k] = 0;
+        fill = 0;
+      }
+      uint64_t w = 0;
+      for (int k = 0; k < 8; ++k) w |= (uint64_t)b[i + k] << (8 * k);
+      buf[fill >> 3] = w;
+      fill += 8;
+    }
+    for (; i < n; ++i) put_byte(b[i]);
   }
   GRID_HD void put_u32(uint32_t x) {
     for (int i = 0; i < 4; ++i) put_byte((uint8_t)(x >> (8 * i)));

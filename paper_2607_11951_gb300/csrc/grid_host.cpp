@@ -847,6 +847,23 @@ int build_parser(const RawGrammar& rg, const char* role_keep, HostGrammar& h) {
       h.acc_sym[s] = X < T1 ? (uint32_t)X : ((1u << 16) | (uint32_t)rank.at(ntname[X - T1]));
     }
   }
+  // kernel items and productions for the reserve completion
+  h.kitem_off.assign(1, 0);
+  h.kitem_p.clear();
+  h.kitem_d.clear();
+  for (int s = 0; s < S; ++s) {
+    for (int it : kernels[s]) {
+      h.kitem_p.push_back(it / 256);
+      h.kitem_d.push_back(it % 256);
+    }
+    h.kitem_off.push_back((int32_t)h.kitem_p.size());
+  }
+  h.prod_off.assign(1, 0);
+  h.prod_rhs.clear();
+  for (auto& pr : P) {
+    for (int x : pr.rhs) h.prod_rhs.push_back(x);
+    h.prod_off.push_back((int32_t)h.prod_rhs.size());
+  }
   // tables
   h.T1 = T1;
   h.S = S;
@@ -1030,6 +1047,215 @@ int build_lexicons(const RawGrammar& rg, const grid_lexicon* lex, int n_lex, Hos
   return GRID_OK;
 }
 
+// Tables of the reserve completion that depend on the grammar and lexicons
+// only (Sec. 5, Prop. 9; see include/grid.h, grid_reserve).
+int build_completion_tables(const RawGrammar& rg, HostGrammar& h) {
+  const int Q = h.Q, T1 = h.T1, LN = h.LN, NC = std::max(1, h.n_cat);
+  auto has = [](const std::vector<uint32_t>& v, int q, int t) { return (v[(size_t)q * 4 + (t >> 5)] >> (t & 31)) & 1u; };
+  auto step = [&](int q, int b) { return (int)h.next[(size_t)q * h.C + h.byte_class[b]]; };
+  auto is_cat = [&](int t) { return (h.catmask[t >> 5] >> (t & 31)) & 1u; };
+  auto is_ign = [&](int t) { return (h.ignored[t >> 5] >> (t & 31)) & 1u; };
+  // the emission candidates of a lexeme at DFA state q with lexicon word
+  // categories wc: its first one (lowest terminal index), or -1
+  auto first_cand = [&](int q, uint32_t wc) {
+    for (int t = 0; t < h.n_term; ++t) {
+      if (!has(h.acc, q, t)) continue;
+      if (is_cat(t)) {
+        int c = -1;
+        for (int k = 0; k < h.n_cat; ++k)
+          if (h.cat_term[k] == t) c = k;
+        if (c < 0 || !((wc >> c) & 1u)) continue;
+      }
+      return t;
+    }
+    return -1;
+  };
+  // lexicon trie: parent, edge byte and DFA state of every node (BFS ids)
+  std::vector<int> par(LN, -1), qn(LN, kStart);
+  std::vector<uint8_t> eb(LN, 0);
+  for (int n = 0; n < LN; ++n)
+    for (int e = h.lx_cstart[n]; e < h.lx_cstart[n + 1]; ++e) {
+      const int ch = h.lx_cnode[e];
+      par[ch] = n;
+      eb[ch] = h.lx_cbyte[e];
+      qn[ch] = qn[n] == kDead ? kDead : step(qn[n], h.lx_cbyte[e]);
+    }
+  // shortest word below each node per category (children in byte order, so
+  // the first child reaching the minimum gives the smallest word)
+  h.lx_wdist.assign((size_t)LN * NC, 0xFFFF);
+  h.lx_wbyte.assign((size_t)LN * NC, 0);
+  for (int n = LN - 1; n >= 0; --n)
+    for (int c = 0; c < h.n_cat; ++c) {
+      uint16_t& d = h.lx_wdist[(size_t)n * NC + c];
+      if ((h.lx_wcats[n] >> c) & 1u) {
+        d = 0;
+        continue;
+      }
+      for (int e = h.lx_cstart[n]; e < h.lx_cstart[n + 1]; ++e) {
+        const uint16_t dc = h.lx_wdist[(size_t)h.lx_cnode[e] * NC + c];
+        if (dc != 0xFFFF && dc + 1 < d) {
+          d = (uint16_t)(dc + 1);
+          h.lx_wbyte[(size_t)n * NC + c] = h.lx_cbyte[e];
+        }
+      }
+    }
+  // shortest accepting continuation per (DFA state, terminal), smallest first byte
+  h.dfa_tdist.assign((size_t)Q * T1, 0xFF);
+  h.dfa_tbyte.assign((size_t)Q * T1, 0);
+  for (int q = 1; q < Q; ++q)
+    for (int t = 0; t < h.n_term; ++t)
+      if (has(h.acc, q, t)) h.dfa_tdist[(size_t)q * T1 + t] = 0;
+  {
+    // breadth-first from the accepting states over reversed transitions, per
+    // terminal; then the first byte: the smallest one whose successor is one
+    // step closer (byte classes visited in order of their smallest byte)
+    std::vector<int> cls_first(h.C, -1), order;
+    for (int b = 0; b < 256; ++b)
+      if (cls_first[h.byte_class[b]] < 0) {
+        cls_first[h.byte_class[b]] = b;
+        order.push_back(h.byte_class[b]);
+      }
+    std::vector<std::vector<int>> rev(Q);
+    for (int q = 1; q < Q; ++q)
+      for (int c = 0; c < h.C; ++c) {
+        const int r = h.next[(size_t)q * h.C + c];
+        if (r != kDead) rev[r].push_back(q);
+      }
+    std::vector<int> queue;
+    for (int t = 0; t < h.n_term; ++t) {
+      queue.clear();
+      for (int q = 1; q < Q; ++q)
+        if (h.dfa_tdist[(size_t)q * T1 + t] == 0) queue.push_back(q);
+      for (size_t k = 0; k < queue.size(); ++k) {
+        const int r = queue[k];
+        const uint8_t dr = h.dfa_tdist[(size_t)r * T1 + t];
+        if (dr >= 0xFE) continue;
+        for (int q : rev[r])
+          if (h.dfa_tdist[(size_t)q * T1 + t] == 0xFF) {
+            h.dfa_tdist[(size_t)q * T1 + t] = (uint8_t)(dr + 1);
+            queue.push_back(q);
+          }
+      }
+      for (int q = 1; q < Q; ++q) {
+        const uint8_t d = h.dfa_tdist[(size_t)q * T1 + t];
+        if (d == 0 || d == 0xFF) continue;
+        for (int c : order) {
+          const int r = h.next[(size_t)q * h.C + c];
+          if (r != kDead && h.dfa_tdist[(size_t)r * T1 + t] == d - 1) {
+            h.dfa_tbyte[(size_t)q * T1 + t] = (uint8_t)cls_first[c];
+            break;
+          }
+        }
+      }
+    }
+  }
+  // separator per state: a byte after which the lexer is where it would be
+  // had the pending lexeme been emitted and the byte started an ignored
+  // lexeme that stays ignored (the byte ends the lexeme, or extends an
+  // ignored one into that same state, as a blank after a blank); the blank
+  // when it qualifies
+  h.sep_byte.assign(Q, -1);
+  auto sep_ok = [&](int q, int b) {
+    const int r = step(kStart, b);
+    if (r == kDead) return false;
+    const int x = step(q, b);
+    if (x != kDead && x != r) return false;
+    bool acc_ign = false, live_other = false;
+    for (int t = 0; t < h.n_term; ++t) {
+      if (has(h.acc, r, t) && is_ign(t)) acc_ign = true;
+      if (has(h.live, r, t) && !is_ign(t)) live_other = true;
+    }
+    return acc_ign && !live_other;
+  };
+  for (int q = 1; q < Q; ++q) {
+    if (sep_ok(q, ' ')) {
+      h.sep_byte[q] = ' ';
+      continue;
+    }
+    for (int b = 0; b < 256; ++b)
+      if (sep_ok(q, b)) {
+        h.sep_byte[q] = (int16_t)b;
+        break;
+      }
+  }
+  // the lexeme rendering each non-ignored terminal: the shortest (then
+  // smallest) string whose first emission candidate is the terminal; for a
+  // category a word of its lexicon
+  h.render_lex.assign(T1, std::string());
+  std::vector<char> done(T1, 0);
+  auto word_of = [&](int n) {
+    std::string w;
+    for (int x = n; x > 0; x = par[x]) w.push_back((char)eb[x]);
+    std::reverse(w.begin(), w.end());
+    return w;
+  };
+  int cat_todo = h.n_cat;
+  for (int n = 1; n < LN && cat_todo > 0; ++n) {  // BFS order: by length, then bytes
+    if (!h.lx_wcats[n] || qn[n] == kDead) continue;
+    const int t = first_cand(qn[n], h.lx_wcats[n]);
+    if (t >= 0 && is_cat(t) && !done[t]) {
+      done[t] = 1;
+      h.render_lex[t] = word_of(n);
+      --cat_todo;
+    }
+  }
+  // literal terminals: their literal, if it is their own first candidate
+  for (int t = 0; t < h.n_term; ++t) {
+    if (is_ign(t) || is_cat(t) || !rg.terms[t].literal) continue;
+    done[t] = 1;
+    const std::string& lit = rg.terms[t].pattern;
+    int q = kStart, lx = LN > 0 ? 0 : -1;
+    for (unsigned char b : lit) {
+      q = q == kDead ? kDead : step(q, b);
+      int nl = -1;
+      if (lx >= 0)
+        for (int e = h.lx_cstart[lx]; e < h.lx_cstart[lx + 1]; ++e)
+          if (h.lx_cbyte[e] == b) nl = h.lx_cnode[e];
+      lx = nl;
+    }
+    if (q != kDead && first_cand(q, lx >= 0 ? h.lx_wcats[lx] : 0u) == t) h.render_lex[t] = lit;
+  }
+  {
+    // the other terminals: breadth-first over (DFA state, lexicon node) pairs
+    // in byte order, up to 32 bytes
+    int todo = 0;
+    for (int t = 0; t < h.n_term; ++t)
+      if (!is_ign(t) && !is_cat(t) && !done[t]) ++todo;
+    struct Node {
+      int q, lx;
+      std::string s;
+    };
+    std::vector<Node> level{{kStart, LN > 0 ? 0 : -1, std::string()}};
+    std::unordered_map<int64_t, char> seen;
+    seen[(int64_t)kStart * (LN + 1) + (LN > 0 ? 1 : 0)] = 1;
+    for (int len = 1; len <= 32 && todo > 0 && !level.empty(); ++len) {
+      std::vector<Node> nxt;
+      for (const Node& nd : level)
+        for (int b = 0; b < 256; ++b) {
+          const int r = step(nd.q, b);
+          if (r == kDead) continue;
+          int lx = -1;
+          if (nd.lx >= 0)
+            for (int e = h.lx_cstart[nd.lx]; e < h.lx_cstart[nd.lx + 1]; ++e)
+              if (h.lx_cbyte[e] == b) lx = h.lx_cnode[e];
+          const int64_t key = (int64_t)r * (LN + 1) + (lx + 1);
+          if (seen.count(key)) continue;
+          seen[key] = 1;
+          Node m{r, lx, nd.s + (char)b};
+          const int t = first_cand(r, lx >= 0 ? h.lx_wcats[lx] : 0u);
+          if (t >= 0 && !is_cat(t) && !is_ign(t) && !done[t]) {
+            done[t] = 1;
+            h.render_lex[t] = m.s;
+            --todo;
+          }
+          nxt.push_back(std::move(m));
+        }
+      level.swap(nxt);
+    }
+  }
+  return GRID_OK;
+}
+
 }  // namespace
 }  // namespace grid
 
@@ -1069,7 +1295,7 @@ extern "C" int grid_compile(const char* grammar_text, size_t len, const char* ro
     return set_error(GRID_E_INVALID_ARG, "max_depth out of range");
   }
   if ((rc = build_lexer(rg, h)) || (rc = build_parser(rg, role_keep, h)) ||
-      (rc = build_lexicons(rg, lex, n_lex, h))) {
+      (rc = build_lexicons(rg, lex, n_lex, h)) || (rc = build_completion_tables(rg, h))) {
     delete g;
     return rc;
   }

@@ -53,6 +53,22 @@ struct HostGrammar {
 
   int max_depth = 4096;
 
+  // reserve completion (Sec. 5, Prop. 9): LR(0) kernel items per state
+  // (production, dot), the productions' right-hand sides (< T1 terminal,
+  // else T1 + nonterminal), per lexicon node and category the length of and
+  // first byte towards the shortest word below (0xFFFF: none), per DFA state
+  // and terminal the length of and first byte towards the shortest
+  // accepting continuation (0xFF: none), per DFA state the byte that ends
+  // the pending lexeme and starts an ignored one (-1: none), and per terminal
+  // the lexeme that renders it (empty: none)
+  std::vector<int32_t> kitem_off, kitem_p, kitem_d;
+  std::vector<int32_t> prod_off, prod_rhs;
+  std::vector<uint16_t> lx_wdist;
+  std::vector<uint8_t> lx_wbyte;
+  std::vector<uint8_t> dfa_tdist, dfa_tbyte;
+  std::vector<int16_t> sep_byte;
+  std::vector<std::string> render_lex;
+
   // audit: the symbol entering each LALR state (kind << 16 | id: kind 0 =
   // terminal id, kind 1 = rank of the nonterminal's name in byte order among
   // all nonterminals of the grammar text; 0xFFFFFFFF for the start state)

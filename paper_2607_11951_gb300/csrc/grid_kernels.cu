@@ -1627,6 +1627,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   int per_sm = 0;
   GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, t.blob_bytes));
   s->walk_blocks = std::max(1, per_sm) * s->sms;
+  if ((rc = build_reserve_tables(s))) return fail(rc);
   *out = s;
   return GRID_OK;
 }
@@ -1678,7 +1679,8 @@ extern "C" int grid_configs_create(const grid_spec* s, int32_t B, grid_configs**
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->vcw) * 4, (void**)&c->vcbits)) ||
       (rc = a.alloc((size_t)B * 2 * std::max(1, s->max_cd) * 4, (void**)&c->surv)) ||
       (rc = a.alloc((size_t)B * 2 * c->vcap * 4, (void**)&c->vsurv)) ||
-      (rc = a.alloc((size_t)B * 4 * 4, (void**)&c->aux))) {
+      (rc = a.alloc((size_t)B * 4 * 4, (void**)&c->aux)) ||
+      (rc = a.alloc((size_t)B * reserve_scratch_bytes(s), (void**)&c->rscratch))) {
     grid_configs_free(c);
     return rc;
   }

@@ -101,6 +101,30 @@ extern int g_sms;  // SM count of the current device, set by grid_specialize
 
 }  // namespace grid
 
+// Device tables of the reserve completion (grid_reserve), built by
+// grid_specialize from the grammar's completion tables and the vocabulary.
+struct ReserveTables {
+  int ok = 0;            // 1 when built
+  int NC = 1;            // categories (at least 1: the row stride of lx_wdist)
+  int E = 0;             // search entries per row
+  const int32_t* item_off = nullptr;  // S + 1: kernel items of each state
+  const int32_t* item_p = nullptr;    // production of each kernel item
+  const int32_t* item_d = nullptr;    // dot of each kernel item (the length of alpha)
+  const uint32_t* item_cost = nullptr;  // tokens of beta's cheapest rendering
+  const int32_t* prod_off = nullptr;  // P + 1
+  const int32_t* prod_rhs = nullptr;  // symbols: < T1 terminal, else T1 + nonterminal
+  const int32_t* ny_off = nullptr;    // NNT + 1: the cheapest terminal yield of each nonterminal
+  const int32_t* ny = nullptr;
+  const int32_t* rend_off = nullptr;  // T1 + 1: the tokens rendering each terminal
+  const int32_t* rend_tok = nullptr;
+  const uint16_t* lx_wdist = nullptr;  // LN * NC
+  const uint8_t* lx_wbyte = nullptr;
+  const uint8_t* dfa_tdist = nullptr;  // Q * T1
+  const uint8_t* dfa_tbyte = nullptr;
+  const int16_t* sep_byte = nullptr;   // Q
+  const int32_t* byte_tok = nullptr;   // 256: the id spelling each single byte, or -1
+};
+
 struct grid_spec {
   const grid_grammar* g = nullptr;
   const grid_vocab* v = nullptr;
@@ -115,6 +139,7 @@ struct grid_spec {
   int n_vc = 0;         // verdict classes over all tables
   int max_vc = 0;       // verdict classes of the largest table
   uint8_t fingerprint[16] = {};  // BLAKE2b-128 of the grammar and vocabulary fingerprints
+  ReserveTables rt;
 };
 
 struct grid_configs {
@@ -131,6 +156,7 @@ struct grid_configs {
   int32_t* vsurv = nullptr;
   int cap = 0, vcap = 0;
   int32_t* aux = nullptr;  // 4 x B ints of per-row working state for forced spans and reserves
+  int32_t* rscratch = nullptr;  // per-row search space of grid_reserve (entries and level heads)
   // audit chain (grid_configs_enable_audit): node hashes (c.hs), per-row
   // chain heads (16 bytes) and record counters
   uint8_t* heads = nullptr;
@@ -151,6 +177,12 @@ int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, 
 // of place) on `st`.
 int launch_advance(const grid_spec* s, const DevConfigs& in, const DevConfigs& out, int B, const int32_t* d_tokens,
                    int32_t n_steps, int32_t* d_status, int copy, cudaStream_t st);
+
+// Reserve completion tables (grid_span.cu), built at the end of
+// grid_specialize into s->rt (device memory owned by s->mem).
+int build_reserve_tables(grid_spec* s);
+// Bytes of grid_reserve's search space per row.
+size_t reserve_scratch_bytes(const grid_spec* s);
 
 // Audit chain (grid_audit.cu): a fresh chain and node hashes of the current
 // stacks when audit is enabled on `c` (no-op otherwise), and one record per

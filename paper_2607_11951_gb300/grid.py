@@ -25,7 +25,7 @@ EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_gramma
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
             "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_forced_span",
-            "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
+            "grid_reserve", "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
             "grid_audit_genesis", "grid_blake2b", "grid_fingerprint", "grid_apply_mask", "grid_configs_export"]
 
 
@@ -79,6 +79,7 @@ def lib():
         "grid_masks": (I32, [P, P, P, P, P]),
         "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
         "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P, P]),
+        "grid_reserve": (I32, [P, P, P, P, I32, P, P, I32, P, P]),
         "grid_configs_enable_audit": (I32, [P, P, P]),
         "grid_audit_append": (I32, [P, P, P, P, I32, P, P]),
         "grid_audit_seal": (I32, [P, P, P, ctypes.c_uint32, P, P]),
@@ -254,6 +255,17 @@ def grid_forced_span(spec, cfg, max_span, mask, span, span_len, status, records=
         assert records.is_contiguous() and records.numel() == span.shape[0] * max_span * 80
     _check(lib().grid_forced_span(spec, cfg, max_span, _ptr(mask), _ptr(span), _ptr(span_len), _ptr(status), rp,
                                   _stream(stream)))
+
+
+def grid_reserve(spec, cfg, cost, tokens, status, budget=None, safety=0, fire=None, stream=None):
+    """cost, status (and budget, fire) int32 CUDA tensors [B]; tokens int32 [B, cap]."""
+    for x in (cost, tokens, status):
+        assert x.is_contiguous()
+    assert tokens.dim() == 2
+    nul = ctypes.c_void_p(None)
+    _check(lib().grid_reserve(spec, cfg, _ptr(cost), _ptr(tokens), tokens.shape[1], _ptr(status),
+                              nul if budget is None else _ptr(budget), safety, nul if fire is None else _ptr(fire),
+                              _stream(stream)))
 
 
 def grid_configs_enable_audit(spec, cfg, stream=None):
