@@ -6,8 +6,10 @@ configurations at prefixes of U[50, 2000] tokens, fp32 logits N(0, 3).
 
 One step = the whole per-token hot path for one batch, through the C ABI:
   grid_advance (out-of-place, one admitted token per row)
-  -> grid_masks (allowed sets + EOS gate, trie walk, id-order packing)
-  -> grid_apply_mask (in-place -inf fill of the fp32 logits).
+  -> grid_masks_apply (allowed sets + EOS gate, trie walk, id-order packing,
+     with the in-place -inf fill of the fp32 logits fused into the packing).
+The standalone grid_apply_mask kernel is timed on its own for its HBM
+roofline (fp32 headline batch; bf16 B=256 in the cold-schema line).
 Steps rotate over 16 distinct pre-built batches (512 prefixes); their logits
 (16 x 19.45 MB = 311 MB) exceed the 129 MB L2, so every step reads cold logits.
 
@@ -32,8 +34,9 @@ METRIC = "cold full-vocab masks/s (batch-32 mask step at V=151,936)"
 
 
 MASK_KERNELS = ["k_row", "k_filter", "k_walk", "k_pack"]
-PROFILE = os.path.join(ROOT, "profiles", "%s_sql_select_only.md")
+COUNTERS = os.path.join(ROOT, "profiles", "counters_sql_select_only.json")
 SMSP_PER_SM = 4  # warp schedulers per SM, each issuing at most one warp instruction per clock
+LANES = 32       # a warp-wide shared-memory access serves 32 lanes in one pipe cycle
 
 
 def _peaks():
@@ -51,7 +54,7 @@ def _source_sha():
     import hashlib
     import re
     h = hashlib.sha256()
-    for f in ("grid_kernels.cu", "grid_device.cuh"):
+    for f in ("grid_kernels.cu", "grid_device.cuh", "grid_state.cuh"):
         with open(os.path.join(ROOT, "paper_2607_11951_gb300", "csrc", f)) as fh:
             for line in fh:
                 code = re.sub(r"//.*", "", line).strip()
@@ -61,18 +64,15 @@ def _source_sha():
 
 
 def _counters(kernel):
-    """Per-launch ncu counters of `kernel` from the committed summary of this
-    workload, if they were taken on the current kernel sources."""
+    """Per-launch ncu counters of `kernel` on this workload, from the committed
+    JSON summary, if they were taken on the current kernel sources."""
     try:
-        kv = {}
-        with open(PROFILE % kernel) as f:
-            for line in f:
-                if line.startswith("- ") and ":" in line:
-                    k, v = line[2:].split(":", 1)
-                    kv[k.strip()] = v.strip().strip("`")
-        if kv.get("source_sha") != _source_sha():
+        with open(COUNTERS) as f:
+            d = json.load(f)
+        if d.get("source_sha") != _source_sha():
             return None
-        return {"inst": float(kv["warp_inst_per_launch"]), "dram": float(kv["dram_bytes_per_launch"])}
+        k = d["kernels"][kernel]
+        return {"inst": float(k["warp_inst_per_launch"]), "dram": float(k["dram_bytes_per_launch"])}
     except Exception:
         return None
 
@@ -189,6 +189,14 @@ def _oracle_throughput(pool, cores, wl, rows, jobs_per_row, ids_per_job, seed):
     return checks / (busy / cores), checks, busy
 
 
+def headline_config(B, V):
+    """The workload named by both arms' lines."""
+    return {"workload": "sql_select_only", "B": B, "V": V, "prefix_tokens": "U[50,2000]",
+            "schema": "200 tables x 30 columns", "logits": "f32 N(0,3)",
+            "batches": N_BATCHES, "l2": "rotating inputs: 16 logits batches = 311 MB > L2",
+            "step": "grid_advance + grid_masks_apply (mask step with the logits fill fused)"}
+
+
 def run_reference(args):
     """The CPU oracle as it stands, on the host cores: each step is a bounded
     sample of the headline workload (``--ref-tokens`` token ids of one
@@ -211,11 +219,14 @@ def run_reference(args):
                 checks += n
     tot = sum(times)
     value = checks / V / tot
+    B = wl["B"]
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "masks/s", "n_gpus": ws,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+            "steps": args.steps, "warmup": args.warmup,
+            # the time of one batch-32 full-vocabulary step at the measured rate
+            "ms_per_step": 1e3 * B / value, "sample_ms_per_step": 1e3 * tot / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
             "data": "synthetic",
-            "config": {"workload": "sql_select_only", "B": 32, "V": V},
+            "config": headline_config(B, V),
             "cpu_baseline": {"value": value, "unit": "masks/s", "cores": cores, "kind": "oracle",
                              "sample": "per step: %d random token ids of one configuration (rows rotate), split "
                                        "over %d spawn workers; worker time inside the mask only" %
@@ -253,17 +264,45 @@ def _time_steps(fn, steps, warmup, stream):
     return sorted(a.elapsed_time(b) * 1e3 for a, b in evs)
 
 
+def _apply_alone(G, mask, logits, steps, stream):
+    """Mean device time (us) of grid_apply_mask alone, launched back to back
+    over rotating logits buffers (larger than L2 together)."""
+    import torch
+    for k in range(3):
+        G.grid_apply_mask(mask, logits[k % len(logits)], stream)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for k in range(steps):
+        G.grid_apply_mask(mask, logits[k % len(logits)], stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) * 1e3 / steps
+
+
+def _roof_apply(B, V, esz, us, label):
+    hbm_peak, peak_kind = _peaks()
+    W = (V + 31) // 32
+    nbytes = B * W * 4 + B * V * esz  # the mask read once + every logit written once
+    ach = nbytes / (us * 1e-6) / 1e9
+    return {"kernel": label, "bound": "hbm", "achieved": ach, "peak": hbm_peak,
+            "peak_kind": peak_kind + " copy bandwidth", "unit": "GB/s", "frac": ach / hbm_peak,
+            "bytes_per_launch": nbytes, "us_per_launch": us,
+            "timing": "back-to-back launches over rotating logits buffers (> L2), CUDA events"}
+
+
 def run_sweep(args):
     """Flatness of the per-step cost (the paper's requirement R): grid_masks on
     B=32 configurations per cell, n in {100, 1k, 4k, 16k} prefix tokens x
     nesting depth in {1, 8, 32, 64}; p50 per cell and, per depth, the OLS slope
-    of step time vs n."""
+    of step time vs n.  One JSON line with the clocks sampled meanwhile."""
     import numpy as np
     import torch
     from paper_2607_11951_gb300 import grid as G
     from workloads import configs
     dev = torch.device("cuda", 0)
     stream = torch.cuda.current_stream()
+    warmup = max(3, args.warmup)
     ns, depths = [100, 1000, 4000, 16000], [1, 8, 32, 64]
     first = configs.sql_sweep_cell(ns[0], depths[0])
     grammar = G.Grammar(first["grammar"], first["role"], first["lexicons"])
@@ -273,7 +312,7 @@ def run_sweep(args):
     W = (V + 31) // 32
     mask = torch.zeros((B, W), dtype=torch.int32, device=dev)
     status = torch.zeros(B, dtype=torch.int32, device=dev)
-    cells = {}
+    built = {}
     for d in depths:
         for n in ns:
             wl = configs.sql_sweep_cell(n, d)
@@ -284,33 +323,47 @@ def run_sweep(args):
             G.grid_advance(spec.h, c.h, c.h, torch.from_numpy(tt).to(dev), status)
             torch.cuda.synchronize()
             assert (status.cpu().numpy() == 0).all(), (n, d, status)
-            t = _time_steps(lambda k: G.grid_masks(spec.h, c.h, mask, status, stream), args.steps, args.warmup,
-                            stream)
+            built[(n, d)] = c
+    clk = ClockSampler(_gpu_index(0))
+    clk.start()
+    cells = {}
+    for d in depths:
+        for n in ns:
+            c = built[(n, d)]
+            t = _time_steps(lambda k: G.grid_masks(spec.h, c.h, mask, status, stream), args.steps, warmup, stream)
             assert (status.cpu().numpy() == 0).all(), (n, d, status)
-            cells["%d,%d" % (n, d)] = {"p50_us": t[len(t) // 2], "p99_us": t[min(len(t) - 1, int(0.99 * len(t)))]}
+            p50 = t[len(t) // 2]
+            cells["%d,%d" % (n, d)] = {"p50_us": p50, "p99_us": t[min(len(t) - 1, int(0.99 * len(t)))],
+                                      "masks_per_s": B / (p50 * 1e-6)}
+    clocks = clk.stop()
     slopes = {}
     for d in depths:
         x = np.array(ns, dtype=np.float64)
         y = np.array([cells["%d,%d" % (n, d)]["p50_us"] for n in ns])
         slope = float(np.polyfit(x, y, 1)[0]) * 1000.0
         slopes[str(d)] = {"us_per_1k_tokens": slope, "p50_at_100": y[0], "p50_at_16k": y[-1]}
-    print(json.dumps({"metric": "grid_masks p50 us per batch-32 step vs prefix length (flatness)",
-                      "unit": "us", "higher_is_better": False, "steps": args.steps, "warmup": args.warmup,
+    worst = max(abs(v["us_per_1k_tokens"]) for v in slopes.values())
+    print(json.dumps({"metric": "per-step cost flatness: max |OLS slope| of grid_masks p50 vs prefix length",
+                      "value": worst, "unit": "us per 1k prefix tokens", "higher_is_better": False,
+                      "n_gpus": 1, "steps": args.steps, "warmup": warmup, "dtype": "u32", "data": "synthetic",
                       "config": {"workload": "sql_sweep_cell", "B": B, "V": V, "grammar": "SQL admin",
-                                 "schema": "200 x 30", "n": ns, "depth": depths},
-                      "cells": cells, "ols_slope_by_depth": slopes}), flush=True)
+                                 "schema": "200 x 30", "n": ns, "depth": depths,
+                                 "step": "grid_masks, K steps per cell with events around each"},
+                      "cells": cells, "ols_slope_by_depth": slopes, "clocks": clocks}), flush=True)
 
 
 def run_cold(args):
     """Cold-schema specialization: grid_specialize (CI classes of every
     precomputed lexer state over V=151,936) for a fresh 1,000 x 50 schema,
-    then B=256 steps (advance + masks + bf16 apply) on its configurations."""
+    then B=256 steps (advance + masks with the bf16 logits fill fused) on its
+    configurations, and the standalone bf16 mask apply at B=256."""
     import numpy as np
     import torch
     from paper_2607_11951_gb300 import grid as G
     from workloads import configs
     dev = torch.device("cuda", 0)
     stream = torch.cuda.current_stream()
+    warmup = max(3, args.warmup)
     wl = configs.sql_cold_schema()
     B, V = wl["B"], len(wl["tokens"])
     W = (V + 31) // 32
@@ -321,6 +374,8 @@ def run_cold(args):
     t2 = time.perf_counter()
     spec_ms = []
     specs = []
+    clk = ClockSampler(_gpu_index(0))
+    clk.start()
     for k in range(4):  # the first includes one-time CUDA module set-up
         torch.cuda.synchronize()
         a = time.perf_counter()
@@ -348,19 +403,24 @@ def run_cold(args):
 
     def step(k):
         G.grid_advance(spec.h, c.h, scratch.h, tok, status, stream)
-        G.grid_masks(spec.h, scratch.h, mask, status, stream)
-        G.grid_apply_mask(mask, logits[k % 2], stream)
+        G.grid_masks_apply(spec.h, scratch.h, mask, status, logits[k % 2], stream)
 
-    t = _time_steps(step, args.steps, args.warmup, stream)
+    t = _time_steps(step, args.steps, warmup, stream)
+    apply_us = _apply_alone(G, mask, logits, args.steps, stream)
+    clocks = clk.stop()
     p50 = t[len(t) // 2]
-    print(json.dumps({"metric": "cold-schema specialization ms and B=256 masks/s", "unit": "ms | masks/s",
+    print(json.dumps({"metric": "cold-schema specialization ms (fresh 1,000 x 50 schema, V=151,936)",
+                      "value": sorted(spec_ms[1:])[1], "unit": "ms", "higher_is_better": False,
+                      "n_gpus": 1, "steps": args.steps, "warmup": warmup, "dtype": "u32", "data": "synthetic",
                       "grid_specialize_ms": sorted(spec_ms[1:])[1], "grid_specialize_ms_first": spec_ms[0],
                       "grid_compile_ms": (t1 - t0) * 1e3, "grid_load_vocab_ms": (t2 - t1) * 1e3,
-                      "spec": spec.info(), "step_p50_us": p50, "masks_per_s": B / (p50 * 1e-6),
-                      "steps": args.steps, "warmup": args.warmup,
+                      "spec": spec.info(), "step_p50_us": p50, "step_p99_us": t[min(len(t) - 1, int(0.99 * len(t)))],
+                      "masks_per_s": B / (p50 * 1e-6),
+                      "roofline_apply_bf16": _roof_apply(B, V, 2, apply_us, "k_apply<bf16> (grid_apply_mask)"),
                       "config": {"workload": "sql_cold_schema", "B": B, "V": V, "schema": "1,000 x 50",
                                  "logits": "bf16 N(0,3), 2 rotating batches = 156 MB > L2",
-                                 "step": "grid_advance + grid_masks + grid_apply_mask"}}), flush=True)
+                                 "step": "grid_advance + grid_masks_apply"},
+                      "clocks": clocks}), flush=True)
 
 
 def main():
@@ -441,12 +501,9 @@ def main():
         G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
         if ev:
             ev[1].record(stream)
-        G.grid_masks(spec.h, scratch.h, mask, status, stream)
+        G.grid_masks_apply(spec.h, scratch.h, mask, status, logits[i], stream)
         if ev:
             ev[2].record(stream)
-        G.grid_apply_mask(mask, logits[i], stream)
-        if ev:
-            ev[3].record(stream)
 
     for k in range(args.warmup):
         step(k)
@@ -454,12 +511,15 @@ def main():
     if ws > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    # Three passes of K steps each, back to back:
+    # Passes of K steps each, back to back:
     #   A  the timed region of `value`: events only at its two ends
-    #   B  per-step events around the three calls (p50/p99, per-call means)
-    #   C  events recorded by the library around each kernel of grid_masks
+    #   B  per-step events around the two calls (p50/p99, per-call means)
+    #   C  events recorded by the library around each kernel of the mask step
+    #   D  the standalone grid_apply_mask (its HBM roofline)
+    #   E  one more pass with k_walk's work counters on (their counts only;
+    #      counting slows the kernel, so no time is taken from this pass)
     # Events cost the GPU a little time each, so A carries none between steps.
-    ev_b = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    ev_b = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     ev_c = [[torch.cuda.Event(enable_timing=True) for _ in range(len(MASK_KERNELS) + 1)] for _ in range(args.steps)]
     for ev in ev_b + ev_c:  # create each event by a first record, before the library sees its handle
         for e in ev:
@@ -490,13 +550,20 @@ def main():
         step(args.warmup + k)
     torch.cuda.synchronize()
     G.grid_configs_set_events(scratch.h, [])
+    apply_us = _apply_alone(G, mask, logits, args.steps, stream)  # pass D
     clocks = clk.stop()
+    work = torch.zeros(4, dtype=torch.int64, device=dev)  # pass E
+    G.grid_spec_set_work_counters(spec.h, work)
+    for k in range(N_BATCHES):
+        step(args.warmup + k)
+    torch.cuda.synchronize()
+    G.grid_spec_set_work_counters(spec.h, None)
+    work = [int(x) / N_BATCHES for x in work.cpu().tolist()]
     total_ms = max_over_ranks(total_ms, ws, dev)
-    per_step = [e[0].elapsed_time(e[3]) * 1e3 for e in ev_b]
+    per_step = [e[0].elapsed_time(e[2]) * 1e3 for e in ev_b]
     adv_us = statistics.mean(e[0].elapsed_time(e[1]) * 1e3 for e in ev_b)
     masks_us = statistics.mean(e[1].elapsed_time(e[2]) * 1e3 for e in ev_b)
-    apply_us = statistics.mean(e[2].elapsed_time(e[3]) * 1e3 for e in ev_b)
-    kern_us = {"k_advance": adv_us, "k_apply": apply_us}
+    kern_us = {"k_advance": adv_us}
     for j, name in enumerate(MASK_KERNELS):
         kern_us[name] = statistics.mean(e[j].elapsed_time(e[j + 1]) * 1e3 for e in ev_c)
     per_step.sort()
@@ -506,10 +573,10 @@ def main():
 
     # ---- end to end through the public API with host buffers ----
     # Every step copies its token ids and logits from pinned host memory and
-    # reads its mask and status back.  Three streams: a host-to-device stream
-    # brings step k+1's inputs into the second of two device buffers while
-    # step k computes, the compute stream waits for them before using them,
-    # and a device-to-host stream reads each step's mask and status (double
+    # reads its mask and status back.  Three streams: a host-to-device stream brings
+    # step k+1's inputs into the second of two device buffers while step k
+    # computes, the compute stream waits for them before using them, and a
+    # device-to-host stream reads each step's mask and status (double
     # buffered) while the next step computes.  The timed region starts before
     # the first copy and ends after the last read.
     e2e = None
@@ -524,7 +591,7 @@ def main():
         d_status = [torch.empty(B, dtype=torch.int32, device=dev) for _ in range(2)]
         h2d, d2h = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
         ev_in = [torch.cuda.Event() for _ in range(2)]    # step's inputs on the device
-        ev_used = [torch.cuda.Event() for _ in range(2)]  # step's apply done: its input buffers are free
+        ev_used = [torch.cuda.Event() for _ in range(2)]  # step's masking done: its input buffers are free
         ev_out = [torch.cuda.Event() for _ in range(2)]   # step's mask and status read back
 
         def copy_in(k):
@@ -542,8 +609,7 @@ def main():
             stream.wait_event(ev_in[j])
             stream.wait_event(ev_out[j])  # mask/status buffers of step k-2 read back
             G.grid_advance(spec.h, cfgs[i].h, scratch.h, d_tok[j], d_status[j], stream)
-            G.grid_masks(spec.h, scratch.h, d_mask[j], d_status[j], stream)
-            G.grid_apply_mask(d_mask[j], d_logits[j], stream)
+            G.grid_masks_apply(spec.h, scratch.h, d_mask[j], d_status[j], d_logits[j], stream)
             ev_used[j].record(stream)
             d2h.wait_event(ev_used[j])
             with torch.cuda.stream(d2h):
@@ -577,51 +643,55 @@ def main():
     # ---- rooflines ----
     # mask apply: HBM-bound, write-mostly; algorithmic bytes = the mask read
     # once + every logit written once (the reject fill touches every sector)
-    hbm_peak, peak_kind = _peaks()
-    apply_bytes = B * W * 4 + B * V * 4
+    roof_apply = _roof_apply(B, V, 4, apply_us, "k_apply<f32> (grid_apply_mask)")
     ac = _counters("k_apply")
-    roof_apply = {"kernel": "k_apply (grid_apply_mask)", "bound": "hbm",
-                  "achieved": apply_bytes / (apply_us * 1e-6) / 1e9, "peak": hbm_peak,
-                  "peak_kind": peak_kind + " copy bandwidth", "unit": "GB/s",
-                  "traffic": ac["dram"] if ac else None, "bytes_per_launch": apply_bytes}
-    roof_apply["frac"] = roof_apply["achieved"] / roof_apply["peak"]
-    # walk: integer work without a memory stream (tables stay in L1/L2), so
-    # its ceiling is the warp-instruction issue rate: SMs x 4 schedulers x
-    # 1 instruction per clock at the SM clock sampled during the timed region
+    roof_apply["traffic"] = ac["dram"] if ac else None
+    # walk: its algorithmic work (lexer steps of byte walks, ACTION and GOTO
+    # lookups of reduce chains, verdict-class events), each unit at least one
+    # dependent shared-memory access by one lane: the ceiling is the shared-
+    # memory pipe serving 32 lanes per clock per SM at the sampled clock.  The
+    # issue-rate fraction (ncu warp instructions, committed with a source hash)
+    # is given beside it.
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     mhz = clocks.get("sm_mhz") or 2070.0
-    issue_peak = sms * SMSP_PER_SM * mhz * 1e6 / 1e9
-    wc = _counters("k_walk")
     walk_us = kern_us["k_walk"]
-    roof_walk = {"kernel": "k_walk (grid_masks)", "bound": "alu", "unit": "G warp-inst/s",
-                 "peak": issue_peak, "peak_kind": "derived: %d SMs x %d schedulers x %.0f MHz sampled" %
-                 (sms, SMSP_PER_SM, mhz),
-                 "achieved": None, "frac": None, "traffic": None,
-                 "counters": "ncu, " + os.path.relpath(PROFILE % "k_walk", ROOT) if wc else "stale or missing"}
+    units = sum(work)
+    peak_units = sms * LANES * mhz * 1e6 / 1e9
+    roof_walk = {"kernel": "k_walk (grid_masks_apply)", "bound": "alu",
+                 "unit": "G work units/s (lexer steps + ACTION + GOTO lookups + verdict-class events)",
+                 "achieved": units / (walk_us * 1e-6) / 1e9, "peak": peak_units,
+                 "peak_kind": "derived: %d SMs x %d lanes of shared-memory pipe per clock x %.0f MHz sampled" %
+                 (sms, LANES, mhz),
+                 "work_per_launch": {"lexer_steps": work[0], "action_lookups": work[1], "goto_lookups": work[2],
+                                     "verdict_class_events": work[3]},
+                 "traffic": None}
+    roof_walk["frac"] = roof_walk["achieved"] / peak_units
+    wc = _counters("k_walk")
+    issue_peak = sms * SMSP_PER_SM * mhz * 1e6 / 1e9
+    roof_walk["issue"] = {"unit": "G warp-inst/s", "peak": issue_peak,
+                          "achieved": wc["inst"] / (walk_us * 1e-6) / 1e9 if wc else None,
+                          "frac": wc["inst"] / (walk_us * 1e-6) / 1e9 / issue_peak if wc else None,
+                          "counters": os.path.relpath(COUNTERS, ROOT) if wc else "stale or missing"}
     if wc:
-        roof_walk["achieved"] = wc["inst"] / (walk_us * 1e-6) / 1e9
-        roof_walk["frac"] = roof_walk["achieved"] / issue_peak
         roof_walk["traffic"] = wc["dram"]
-    dominant = max(kern_us, key=kern_us.get)
+    dominant = max((k for k in kern_us), key=kern_us.get)
     roof = roof_walk if dominant == "k_walk" else roof_apply
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "masks/s", "n_gpus": ws, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
-                "config": {"workload": "sql_select_only", "B": B, "V": V, "prefix_tokens": "U[50,2000]",
-                           "schema": "200 tables x 30 columns", "logits": "f32 N(0,3)",
-                           "batches": N_BATCHES, "l2": "rotating inputs: 16 logits batches = 311 MB > L2",
-                           "step": "grid_advance + grid_masks + grid_apply_mask"},
+                "config": headline_config(B, V),
                 "p50_us": p50, "p99_us": p99,
                 "token_checks_per_s": value * V,
-                "call_us": {"grid_advance": adv_us, "grid_masks": masks_us, "grid_apply_mask": apply_us},
+                "call_us": {"grid_advance": adv_us, "grid_masks_apply": masks_us},
                 "kernel_us": kern_us, "dominant_kernel": dominant,
                 "roofline": roof, "roofline_apply": roof_apply, "cpu_baseline": cpu_base, "e2e": e2e,
-                "gpu_launches": args.steps * (2 + len(MASK_KERNELS)), "clocks": clocks,
+                "gpu_launches": args.steps * (1 + len(MASK_KERNELS)), "clocks": clocks,
                 "timing": "value: K steps between two events; p50/p99 and call_us: a second pass of K "
                           "steps with events around each call; kernel_us: a third pass with events "
-                          "around each kernel of grid_masks"}
+                          "around each kernel of the mask step (k_pack includes the logits fill); "
+                          "roofline_apply: the standalone grid_apply_mask, back to back"}
         print(json.dumps(line), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()

@@ -226,6 +226,15 @@ int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask
  * they are set. */
 int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events);
 
+/* Measurement hook: with d_counters (device memory, 4 x u64, zeroed by the
+ * caller) set, every later mask step on `s` adds to it the work of its walk
+ * kernel in the units of the walk's algorithmic cost: [0] lexer steps (trie
+ * node visits of byte walks), [1] ACTION lookups (reduce-chain steps, for one
+ * terminal or a set of terminals at once), [2] GOTO lookups, [3] verdict-class
+ * events evaluated.  Counting slows that kernel down (one atomic per unit);
+ * time steps without it.  NULL stops the counting. */
+int grid_spec_set_work_counters(grid_spec* s, unsigned long long* d_counters);
+
 /* grid_masks without any allocation.  The paper has no counterpart: this is
  * an interface for callers that cannot allocate device memory when they need
  * a mask, e.g. a serving engine whose memory pool has reserved the device up

@@ -143,6 +143,15 @@ struct Tables {
   const uint32_t* acc_sym;    // S: the symbol entering each state (audit node hash)
 };
 
+// Work counters of a walk, kept in the lane's registers when the walk is
+// measured and absent (a null pointer the compiler sees) otherwise:
+// [0] lexer steps (trie node visits), [1] ACTION lookups (one per reduce
+// chain step, for a terminal or a set of terminals), [2] GOTO lookups,
+// [3] verdict-class events evaluated.
+__device__ __forceinline__ void count_work(uint32_t* ctr, int k) {
+  if (ctr) ++ctr[k];
+}
+
 // Membership test in a 4-word set stored in memory.
 __device__ __forceinline__ bool bit4(const uint32_t* m, int t) { return (m[t >> 5] >> (t & 31)) & 1u; }
 
@@ -276,12 +285,14 @@ struct LArr {
 // shift/accept, (keep_o, m_o, scr[0:ns]) is the stack under the pushed state.
 template <typename OV>
 __device__ __forceinline__ int simulate(const Tables& t, const uint16_t* base, int keep, OV ovl, int m, int tau,
-                                        LArr scr, int cap, int& keep_o, int& m_o, int& ns, int max_chain) {
+                                        LArr scr, int cap, int& keep_o, int& m_o, int& ns, int max_chain,
+                                        uint32_t* ctr = nullptr) {
   int k = keep, mm = m;
   ns = 0;
   int top = mm ? ovl[mm - 1] : base[k - 1];
   for (int it = 0; it < max_chain; ++it) {
     if (top >= t.S) return 0;
+    count_work(ctr, 1);
     const int a = t.action[top * t.T1 + tau];
     if (a == 0) return 0;
     if (a > 0) {
@@ -302,6 +313,7 @@ __device__ __forceinline__ int simulate(const Tables& t, const uint16_t* base, i
     const int top2 = ns ? scr[ns - 1] : (mm ? ovl[mm - 1] : base[k - 1]);
     if (top2 >= t.S) return 0;
     if (ns >= cap) return -1;
+    count_work(ctr, 2);
     top = t.go[top2 * t.NNT + (code & 1023)];
     scr[ns++] = (uint16_t)top;
   }
@@ -319,7 +331,8 @@ constexpr int kSetRounds = 8;
 
 template <typename OV>
 __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* base, int keep, OV ovl, int m, Bits4 G,
-                                              LArr scr, int cap, int max_chain, bool& bound) {
+                                              LArr scr, int cap, int max_chain, bool& bound,
+                                              uint32_t* ctr = nullptr) {
   Bits4 res = Bits4::zero();
   Bits4 todo = G;
   for (int round = 0; round < kSetRounds && todo.any(); ++round) {
@@ -330,6 +343,7 @@ __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* b
     int top = mm ? ovl[mm - 1] : base[k - 1];
     for (; it < max_chain && g.any(); ++it) {
       if (top >= t.S) break;
+      count_work(ctr, 1);
       const Bits4 sh = Bits4::load(t.shift_mask + top * 4);
       res = res | (g & sh);
       g = g.andnot(sh);
@@ -363,6 +377,7 @@ __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* b
         bound = true;
         return res;
       }
+      count_work(ctr, 2);
       top = t.go[top2 * t.NNT + (p & 1023)];
       scr[ns++] = (uint16_t)top;
     }
@@ -375,7 +390,7 @@ __device__ __forceinline__ Bits4 simulate_set(const Tables& t, const uint16_t* b
     const int tau = todo.lowest();
     todo.clear_lowest();
     int keep_o, m_o, ns;
-    const int a = simulate(t, base, keep, ovl, m, tau, scr, cap, keep_o, m_o, ns, max_chain);
+    const int a = simulate(t, base, keep, ovl, m, tau, scr, cap, keep_o, m_o, ns, max_chain, ctr);
     if (a < 0) {
       bound = true;
       return res;
@@ -402,11 +417,14 @@ struct Walker {
   const uint32_t* A2;
   LArr ovl, scr;  // overlay and simulation scratch, `cap` entries each
   int cap;
+  uint32_t* ctr;  // work counters (measured walks), or NULL
 };
 
 __device__ __forceinline__ void walker_init(Walker& w, LArr ovl_store, LArr scr_store, int cap, const uint16_t* base,
                                             int keep, const uint16_t* ovl, int m, int q, int lx, uint32_t pc,
-                                            uint32_t wc, const uint32_t* A, const uint32_t* A2) {
+                                            uint32_t wc, const uint32_t* A, const uint32_t* A2,
+                                            uint32_t* ctr = nullptr) {
+  w.ctr = ctr;
   w.ovl = ovl_store;
   w.scr = scr_store;
   w.cap = cap;
@@ -438,7 +456,7 @@ __device__ __forceinline__ bool commit(Walker& w, int keep_o, int m_o, int ns, i
 // allowed set of the stack it was deferred at, so it reaches SHIFT.
 __device__ __forceinline__ bool materialize(const Tables& t, Walker& w, int max_chain) {
   int keep_o, m_o, ns;
-  const int a = simulate(t, w.base, w.keep, w.ovl, w.m, w.pend, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+  const int a = simulate(t, w.base, w.keep, w.ovl, w.m, w.pend, w.scr, w.cap, keep_o, m_o, ns, max_chain, w.ctr);
   w.pend = -1;
   if (a <= 0 || a == kAccept) return false;
   return commit(w, keep_o, m_o, ns, a - 1);
@@ -470,14 +488,15 @@ __device__ __forceinline__ int emit_set(const Tables& t, Walker& w, Bits4 K, int
       bool bound = false;
       Bits4 rest = K;
       rest.set(tau);
-      const Bits4 ok = simulate_set(t, w.base, w.keep, w.ovl, w.m, rest.andnot(t.ign), w.scr, w.cap, max_chain, bound);
+      const Bits4 ok =
+          simulate_set(t, w.base, w.keep, w.ovl, w.m, rest.andnot(t.ign), w.scr, w.cap, max_chain, bound, w.ctr);
       if (bound) return -1;
       const int pick = (ok | (rest & t.ign)).lowest();
       if (pick < 0) return 0;
       if (t.ign.has(pick)) return 1;
       K = Bits4::zero();
       int keep_o, m_o, ns;
-      const int a = simulate(t, w.base, w.keep, w.ovl, w.m, pick, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+      const int a = simulate(t, w.base, w.keep, w.ovl, w.m, pick, w.scr, w.cap, keep_o, m_o, ns, max_chain, w.ctr);
       if (a <= 0 || a == kAccept || !commit(w, keep_o, m_o, ns, a - 1)) return -1;
       w.shifted = true;
       w.Acur = (w.nshift == 0 && w.A2) ? w.A2 + pick * 4 : nullptr;
@@ -485,7 +504,7 @@ __device__ __forceinline__ int emit_set(const Tables& t, Walker& w, Bits4 K, int
       return 1;
     }
     int keep_o, m_o, ns;
-    int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+    int a = simulate(t, w.base, w.keep, w.ovl, w.m, tau, w.scr, w.cap, keep_o, m_o, ns, max_chain, w.ctr);
     if (a < 0) return -1;
     if (a > 0 && a != kAccept) {
       if (!commit(w, keep_o, m_o, ns, a - 1)) return -1;
@@ -509,12 +528,13 @@ __device__ __forceinline__ int trailing_set(const Tables& t, Walker& w, Bits4 L,
   if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
   if (L.count() == 1) {
     int keep_o, m_o, ns;
-    const int a = simulate(t, w.base, w.keep, w.ovl, w.m, L.lowest(), w.scr, w.cap, keep_o, m_o, ns, max_chain);
+    const int a =
+        simulate(t, w.base, w.keep, w.ovl, w.m, L.lowest(), w.scr, w.cap, keep_o, m_o, ns, max_chain, w.ctr);
     if (a < 0) return -1;
     return a > 0 && a != kAccept ? 1 : 0;
   }
   bool bound = false;
-  const Bits4 ok = simulate_set(t, w.base, w.keep, w.ovl, w.m, L, w.scr, w.cap, max_chain, bound);
+  const Bits4 ok = simulate_set(t, w.base, w.keep, w.ovl, w.m, L, w.scr, w.cap, max_chain, bound, w.ctr);
   if (bound) return -1;
   return ok.any() ? 1 : 0;
 }
@@ -552,6 +572,7 @@ __device__ __forceinline__ Spell load_spell(const Tables& t, int s) {
 __device__ __forceinline__ int walk_bytes(const Tables& t, Walker& w, const Spell& sp, int max_chain) {
   const int len = sp.len;
   for (int i = 0; i < len; ++i) {
+    count_work(w.ctr, 0);
     const int b = sp.at(i);
     const int c = t.byte_class[b];
     int nq = t.next[w.q * t.C + c];
@@ -583,7 +604,7 @@ __device__ __forceinline__ int eos_gate(const Tables& t, Walker& w, int max_chai
   }
   if (w.pend >= 0 && !materialize(t, w, max_chain)) return -1;
   int keep_o, m_o, ns;
-  int a = simulate(t, w.base, w.keep, w.ovl, w.m, t.n_term, w.scr, w.cap, keep_o, m_o, ns, max_chain);
+  int a = simulate(t, w.base, w.keep, w.ovl, w.m, t.n_term, w.scr, w.cap, keep_o, m_o, ns, max_chain, w.ctr);
   if (a < 0) return -1;
   return a == kAccept ? 1 : 0;
 }
@@ -666,6 +687,7 @@ __device__ __forceinline__ uint16_t classify(const Tables& t, int q, int lx, con
 __device__ __forceinline__ int eval_record(const Tables& t, Walker& w, const uint16_t* rec, int max_chain) {
   const int n = rec[0];
   for (int i = 0; i < n; ++i) {
+    count_work(w.ctr, 3);
     const int e = emit_set(t, w, class_set(t, rec[2 + i]), max_chain);
     if (e <= 0) return e;
   }

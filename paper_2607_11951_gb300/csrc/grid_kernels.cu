@@ -644,6 +644,10 @@ __device__ __forceinline__ int4 row_queue(const Tables& t, const RowCtx& x) {
 // can survive): the range's items interleave, lane j of item i walking
 // spelling lo + i + j * (items of the range).  Both kinds share one call of
 // walk_bytes, one spelling per lane.
+// With COUNT, each lane also counts its work (lexer steps, ACTION and GOTO
+// lookups, verdict-class events) in registers and adds the totals to
+// work[0..3] when it is done; the plain instance has no counting code.
+template <bool COUNT>
 __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* __restrict__ ctx,
                                                              const RowRanges* __restrict__ rng, const uint16_t* stacks,
                                                              const int32_t* __restrict__ surv, int cap,
@@ -651,7 +655,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
                                                              uint32_t* __restrict__ verd0,
                                                              uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
                                                              int vcw, const int32_t* __restrict__ vsurv, int vcap,
-                                                             int words_v, int B) {
+                                                             int words_v, int B,
+                                                             unsigned long long* __restrict__ work) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ uint16_t s_ovl[kWalkWarps][kMaxOvl];
   __shared__ uint16_t s_win[kWalkWarps][kWalkWin];
@@ -665,6 +670,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   const int gw = blockIdx.x * kWalkWarps + warp;
   const int mc = max_chain_of(t);
   const LArr lo{s_lane[warp] + lane, 32}, ls{s_lane[warp] + kLaneOvl * 32 + lane, 32};
+  uint32_t cnt[4] = {0u, 0u, 0u, 0u};
+  uint32_t* const ctr = COUNT ? cnt : nullptr;
   // queue length and segment ends of every row
   const bool cached = B <= kWalkRowsCached;
   if (cached) {
@@ -770,7 +777,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
       if (k < r.nvs[cxi]) {
         v = vsurv[((size_t)row * 2 + cxi) * vcap + k];
         Walker w;
-        walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
+        walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row, ctr);
         res = eval_record(ts, w, ts.vc_rec + (size_t)(t.vc_off[tb] + v) * kRecLen, mc);
         if (res < 0 && bound_row < 0) bound_row = row;
       }
@@ -819,7 +826,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
       if (go) {
         const Spell sp = load_spell(ts, sp_i);
         Walker w;
-        walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row);
+        walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row, ctr);
         const int res = walk_bytes(ts, w, sp, mc);
         if (res < 0 && bound_row < 0) bound_row = row;
         if (res > 0)  // the verdict of every id with this spelling, in the mask's layout
@@ -828,6 +835,9 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
     }
   }
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
+  if (COUNT)
+    for (int k = 0; k < 4; ++k)
+      if (cnt[k]) atomicAdd(&work[k], (unsigned long long)cnt[k]);
 }
 
 // grid = (ceil(W / kPackWords), B), kPackWords threads: thread (b, wi) makes
@@ -1144,9 +1154,10 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
 // memory, bounds a grid of one short block per 256 sectors).  A sector whose
 // tokens are all rejected is written without being read; a mixed sector is
 // read, blended and written; a fully accepted sector is not touched.  Each
-// thread takes kApplyBatch sectors at a time, with their mask words loaded
-// together, then their mixed sectors read together, then all stored, so that
-// a thread waits on two rounds of loads per batch instead of two per sector.
+// thread takes kApplyBatch sectors at a time: their mask words loaded
+// together, then the rejected sectors stored (they wait on nothing), then the
+// mixed sectors read together and stored, so that a thread waits on two
+// rounds of loads per batch instead of two per sector.
 // Rows whose sectors are not 32-byte aligned, and the ragged end of a row,
 // are done element by element.
 constexpr int kApplyBatch = 4;
@@ -1168,11 +1179,17 @@ __global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask
       const int e0 = (s0 + u * step) * E;
       sb[u] = s0 + u * step < nsec ? (mask[(size_t)b * W + (e0 >> 5)] >> (e0 & 31)) & sfull : sfull;
     }
+#pragma unroll
+    for (int u = 0; u < kApplyBatch; ++u) {  // rejected whole sectors first: written without a read
+      const int e0 = (s0 + u * step) * E;
+      if (vec_ok && s0 + u * step < nsec && e0 + E <= V && sb[u] == 0u)
+        asm volatile("st.global.v8.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1};" ::"l"(row + e0), "r"(fill) : "memory");
+    }
     uint32_t v[kApplyBatch][8];
 #pragma unroll
     for (int u = 0; u < kApplyBatch; ++u) {  // mixed whole sectors: read
       const int e0 = (s0 + u * step) * E;
-      if (vec_ok && e0 + E <= V && sb[u] != 0u && sb[u] != sfull)
+      if (vec_ok && s0 + u * step < nsec && e0 + E <= V && sb[u] != 0u && sb[u] != sfull)
         asm volatile("ld.global.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
                      : "=r"(v[u][0]), "=r"(v[u][1]), "=r"(v[u][2]), "=r"(v[u][3]), "=r"(v[u][4]), "=r"(v[u][5]),
                        "=r"(v[u][6]), "=r"(v[u][7])
@@ -1180,17 +1197,15 @@ __global__ void __launch_bounds__(256) k_apply(const uint32_t* __restrict__ mask
                      : "memory");
     }
 #pragma unroll
-    for (int u = 0; u < kApplyBatch; ++u) {  // blend and store
+    for (int u = 0; u < kApplyBatch; ++u) {  // mixed sectors: blend and store; partial sectors one by one
       const int e0 = (s0 + u * step) * E;
       if (s0 + u * step >= nsec || sb[u] == sfull) continue;
       T* p = row + e0;
       const int n = min(E, V - e0);
       if (vec_ok && n == E) {
+        if (sb[u] == 0u) continue;  // written above
         uint32_t w[8];
-        if (sb[u] == 0u) {
-#pragma unroll
-          for (int k = 0; k < 8; ++k) w[k] = fill;
-        } else if (sizeof(T) == 4) {
+        if (sizeof(T) == 4) {
 #pragma unroll
           for (int k = 0; k < 8; ++k) w[k] = ((sb[u] >> k) & 1u) ? v[u][k] : fill;
         } else {
@@ -1257,7 +1272,8 @@ static int set_smem_limits() {
   GRID_CUDA(cudaFuncSetAttribute(k_pack<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_pack<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
-  GRID_CUDA(cudaFuncSetAttribute(k_walk, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_walk<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_walk<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   return GRID_OK;
 }
@@ -1625,7 +1641,7 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   s->n1 = (counts[0] + kSpan - 1) / kSpan;
   s->max_cd = *std::max_element(counts.begin(), counts.end());
   int per_sm = 0;
-  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk, kWalkWarps * 32, t.blob_bytes));
+  GRID_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_walk<false>, kWalkWarps * 32, t.blob_bytes));
   s->walk_blocks = std::max(1, per_sm) * s->sms;
   if ((rc = build_reserve_tables(s))) return fail(rc);
   *out = s;
@@ -1743,10 +1759,16 @@ int grid::launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratc
   GRID_CUDA(launch_pdl(k_filter, dim3(std::max(1, cd_blocks + vc_blocks), B, 2), dim3(256), 0, st, t, m.ctx,
                        (const uint32_t*)m.sel, m.surv, m.cap, m.vsurv, m.vcap, cd_blocks));
   if (ev) GRID_CUDA(cudaEventRecord(ev[2], st));
-  GRID_CUDA(launch_pdl(k_walk, dim3(s->walk_blocks), dim3(kWalkWarps * 32), t.blob_bytes, st, t, m.ctx,
-                       (const RowRanges*)m.rng, (const uint16_t*)c.stack, (const int32_t*)m.surv, m.cap,
-                       (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
-                       m.words_v, B));
+  if (s->walk_work)  // the measured instance, which counts its work
+    GRID_CUDA(launch_pdl(k_walk<true>, dim3(s->walk_blocks), dim3(kWalkWarps * 32), t.blob_bytes, st, t, m.ctx,
+                         (const RowRanges*)m.rng, (const uint16_t*)c.stack, (const int32_t*)m.surv, m.cap,
+                         (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
+                         m.words_v, B, s->walk_work));
+  else
+    GRID_CUDA(launch_pdl(k_walk<false>, dim3(s->walk_blocks), dim3(kWalkWarps * 32), t.blob_bytes, st, t, m.ctx,
+                         (const RowRanges*)m.rng, (const uint16_t*)c.stack, (const int32_t*)m.surv, m.cap,
+                         (const uint32_t*)m.A2, m.verd0, m.verd1, m.vcbits, vcw, (const int32_t*)m.vsurv, m.vcap,
+                         m.words_v, B, (unsigned long long*)nullptr));
   if (ev) GRID_CUDA(cudaEventRecord(ev[3], st));
   const dim3 pgrid((t.W + kPackWords - 1) / kPackWords, B);
   const size_t psmem = (size_t)(2 * std::max(1, t.nselw) + 2 * vcw) * 4;
@@ -1789,6 +1811,12 @@ extern "C" int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint3
   lg.dtype = dtype;
   lg.stride = row_stride;
   return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr, lg);
+}
+
+extern "C" int grid_spec_set_work_counters(grid_spec* s, unsigned long long* d_counters) {
+  if (!s) return set_error(GRID_E_INVALID_ARG, "grid_spec_set_work_counters: bad arguments");
+  s->walk_work = d_counters;
+  return GRID_OK;
 }
 
 extern "C" int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events) {

@@ -140,6 +140,7 @@ struct grid_spec {
   int max_vc = 0;       // verdict classes of the largest table
   uint8_t fingerprint[16] = {};  // BLAKE2b-128 of the grammar and vocabulary fingerprints
   ReserveTables rt;
+  unsigned long long* walk_work = nullptr;  // measurement hook: k_walk's work counters (4), or NULL
 };
 
 struct grid_configs {

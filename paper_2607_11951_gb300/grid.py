@@ -24,7 +24,7 @@ GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
-            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_masks_static", "grid_forced_span",
+            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_spec_set_work_counters", "grid_masks_static", "grid_forced_span",
             "grid_reserve", "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
             "grid_audit_genesis", "grid_blake2b", "grid_fingerprint", "grid_apply_mask", "grid_configs_export"]
 
@@ -89,6 +89,7 @@ def lib():
         "grid_blake2b": (I32, [P, SZ, P, I32]),
         "grid_fingerprint": (I32, [P, P, P, P]),
         "grid_configs_set_events": (I32, [P, P, I32]),
+        "grid_spec_set_work_counters": (I32, [P, P]),
         "grid_masks_static": (I32, [P, P, P, P, P, P, I32, I32, P, P, P]),
         "grid_apply_mask": (I32, [P, P, I32, I32, I32, I64, P]),
         "grid_configs_export": (I32, [P, I32, P, I32, P, P, P, P]),
@@ -326,6 +327,11 @@ def grid_configs_set_events(cfg, events):
     kernels of every later grid_masks on cfg; an empty list stops it."""
     arr = (ctypes.c_void_p * max(1, len(events)))(*[e.cuda_event for e in events])
     _check(lib().grid_configs_set_events(cfg, ctypes.cast(arr, ctypes.c_void_p), len(events)))
+
+
+def grid_spec_set_work_counters(spec, counters):
+    """counters: int64 CUDA tensor [4] (zeroed by the caller), or None to stop."""
+    _check(lib().grid_spec_set_work_counters(spec, ctypes.c_void_p(None) if counters is None else _ptr(counters)))
 
 
 def grid_masks_static(spec, stack, depth, dfa_state, lex_node, flags, mask, status, stream=None):
