@@ -226,6 +226,45 @@ int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask
  * they are set. */
 int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_events);
 
+/* ---- configuration-keyed mask cache (Sec. 4.3, Def. T1 key, Prop. OBL-KEY1) ----
+ * A cache holds, per key, the context-independent part of a mask: the bits
+ * of the token ids whose verdict the CI classes decide, and which ids are
+ * the stack-dependent residue.  The key is (kind, lexer state, whether the
+ * pending lexeme's forced emission succeeds, A(sigma), A(sigma')): kind 1
+ * marks identifier positions (a lexer state where a lexicon category is
+ * live), a distinct key type, whose continuing ids are always residue, so a
+ * generic entry is never consulted at an identifier position; the spec (its
+ * grammar, role and schema) scopes the whole cache.  The residue (verdict
+ * classes and byte walks) and the EOS gate are never cached and are computed
+ * on every step, so a hit changes no bit of any mask (OBL-KEY1; the tests
+ * compare cache-on with cache-off over randomized replays).  Entries are
+ * filled by the step that first meets a key (an empty slot is claimed; the
+ * slot is the key's hash modulo n_entries, no eviction) and read from the
+ * next step on; the content is a function of the key, so concurrent fills of
+ * one key write identical words. */
+typedef struct grid_cache grid_cache;
+
+/* Allocate a cache of n_entries (a power of two, <= 2^20) entries of
+ * 64 + 8 * ceil(V/32) bytes for spec `s` (which must outlive it).
+ * Synchronizes.  Free with grid_cache_free. */
+int grid_cache_create(const grid_spec* s, int32_t n_entries, grid_cache** out);
+void grid_cache_free(grid_cache* c);
+
+/* Empty every entry and zero the counters (enqueued on `stream`). */
+int grid_cache_clear(grid_cache* c, void* stream);
+
+/* Counters (synchronous): out[0] lookups, out[1] hits, out[2] entries
+ * claimed for filling, out[3] entries ready. */
+int grid_cache_stats(const grid_cache* c, int64_t out[4]);
+
+/* grid_masks (d_logits == NULL) or grid_masks_apply (d_logits of `dtype`,
+ * row_stride >= V) reading and filling `cache`: the same masks, statuses and
+ * logits bit for bit, with the context-independent part of each row taken
+ * from the cache on a hit.  Calls that use one cache must not overlap on the
+ * GPU.  Enqueue only. */
+int grid_masks_cached(const grid_spec* s, const grid_configs* c, grid_cache* cache, uint32_t* d_mask,
+                      int32_t* d_status, void* d_logits, int32_t dtype, int64_t row_stride, void* stream);
+
 /* Measurement hook: with d_counters (device memory, 4 x u64, zeroed by the
  * caller) set, every later mask step on `s` adds to it the work of its walk
  * kernel in the units of the walk's algorithmic cost: [0] lexer steps (trie

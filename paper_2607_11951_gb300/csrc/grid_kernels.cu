@@ -248,7 +248,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
                                                         RowRanges* __restrict__ rng, uint32_t* __restrict__ A2,
                                                         uint32_t* __restrict__ sel, uint32_t* __restrict__ verd0,
                                                         uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
-                                                        int n_vcbits, int B, int words_v) {
+                                                        int n_vcbits, int B, int words_v, CacheDev cache) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   __shared__ uint16_t s_stk[kStackWin];
@@ -494,6 +494,44 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   __syncthreads();
   // ---- the row's context for the later kernels
   if (threadIdx.x == 0) {
+    // configuration-keyed cache of the context-independent part (Sec. 4.3):
+    // key = (kind, lexer state, emit_ok, A(sigma), A(sigma')); the CD residue
+    // is never cached.  A ready entry with this key is read; an empty slot is
+    // claimed and filled by k_pack; any other slot is left alone.
+    int chit = -1, cfill = -1;
+    if (cache.n && !complete) {
+      uint32_t key[11];
+      key[0] = (q != kStart && tbl0 < 0) ? 1u : 0u;
+      key[1] = (uint32_t)q;
+      key[2] = (uint32_t)emit_ok;
+      for (int k = 0; k < 4; ++k) {
+        key[3 + k] = s_A0[k];
+        key[7 + k] = emit_ok ? s_A1[k] : 0u;
+      }
+      unsigned long long hsh = 1469598103934665603ull;  // FNV-1a over the key words
+      for (int k = 0; k < 11; ++k) {
+        hsh ^= key[k];
+        hsh *= 1099511628211ull;
+      }
+      const int slot = (int)(hsh & (unsigned long long)(cache.n - 1));
+      uint32_t* h = cache.hdr + (size_t)slot * 16;
+      atomicAdd(&cache.stats[0], 1ull);
+      const uint32_t state = *(volatile uint32_t*)h;
+      if (state == 2u) {
+        bool same = true;
+        for (int k = 0; k < 11; ++k) same &= ((volatile uint32_t*)h)[1 + k] == key[k];
+        if (same) {
+          chit = slot;
+          atomicAdd(&cache.stats[1], 1ull);
+        }
+      } else if (state == 0u && atomicCAS(h, 0u, 1u) == 0u) {
+        for (int k = 0; k < 11; ++k) h[1 + k] = key[k];
+        cfill = slot;
+        atomicAdd(&cache.stats[2], 1ull);
+      }
+    }
+    r.chit = chit;
+    r.cfill = cfill;
     for (int k = 0; k < 4; ++k) {
       r.A0[k] = s_A0[k];
       r.A1[k] = emit_ok ? s_A1[k] : 0u;
@@ -863,9 +901,10 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
                                                      const uint32_t* __restrict__ verd0,
                                                      const uint32_t* __restrict__ verd1, int words_v,
                                                      uint32_t* __restrict__ mask, int32_t* __restrict__ d_status,
-                                                     void* __restrict__ logits, long long stride, int vec_ok) {
+                                                     void* __restrict__ logits, long long stride, int vec_ok,
+                                                     CacheDev cache) {
   extern __shared__ __align__(16) uint32_t s_dyn[];  // class selections (2 nselw) | verdict-class bits (2 vcw)
-  __shared__ int s_fl, s_tb, s_any;
+  __shared__ int s_fl, s_tb, s_any, s_hit, s_fill;
   __shared__ uint32_t s_kill[8];
   const int b = blockIdx.y;
   const int wi = blockIdx.x * kPackWords + threadIdx.x;
@@ -891,10 +930,12 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
     s_tb = rc.tbl0;
     s_fl = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
     s_any = 0;
+    s_hit = cache.n ? rc.chit : -1;
+    s_fill = cache.n ? rc.cfill : -1;
   }
   if (threadIdx.x < 8) s_kill[threadIdx.x] = rc.kill[threadIdx.x];
   __syncthreads();
-  const int fl = s_fl, tb = s_tb;
+  const int fl = s_fl, tb = s_tb, hit = s_hit, fill = s_fill;
   // a context that k_row did not select for (a completed row, sigma' without
   // a forced emission, sigma without a table) reads zeros
   {
@@ -913,8 +954,16 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
   if (have && !(fl & 4)) {
     const uint32_t wv0 = verd0[(size_t)b * words_v + wi];
     const uint32_t wv1 = (fl & 1) ? verd1[(size_t)b * words_v + wi] : 0u;
+    // a cache hit gives the context-independent bits; only the residue ids
+    // (verdict-class and walked) are decided here
+    uint32_t todo = valid;
+    if (hit >= 0) {
+      m = cache.ci[(size_t)hit * t.W + wi];
+      todo = cache.sel[(size_t)hit * t.W + wi];
+    }
+    uint32_t ci_bits = 0u, sel_bits = 0u;  // what a filling row stores
     uint4 ct4[4];
-    if (tb >= 0) {
+    if (tb >= 0 && todo) {
       const uint4* c = reinterpret_cast<const uint4*>(t.cls_by_id + (size_t)tb * t.Vp) + 4 * wi;
 #pragma unroll
       for (int k = 0; k < 4; ++k) ct4[k] = c[k];
@@ -925,7 +974,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
     uint32_t ctw[16];
 #pragma unroll
     for (int k = 0; k < 16; ++k) ctw[k] = code_walk | ((uint32_t)code_walk << 16);
-    if (tb >= 0) {
+    if (tb >= 0 && todo) {
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         ctw[4 * k] = ct4[k].x;
@@ -936,7 +985,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
     }
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
-      if (!((valid >> j) & 1u)) continue;
+      if (!((todo >> j) & 1u)) continue;
       const int by = (fbw[j >> 2] >> ((j & 3) * 8)) & 0xFF;
       const int cx = (s_kill[by >> 5] >> (by & 31)) & 1u;
       const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
@@ -948,11 +997,18 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
         } else {
           bit = ((cx ? wv1 : wv0) >> j) & 1u;
         }
+        sel_bits |= 1u << j;
+      } else {
+        ci_bits |= bit << j;
       }
       m |= bit << j;
     }
+    if (fill >= 0) {
+      cache.ci[(size_t)fill * t.W + wi] = ci_bits;
+      cache.sel[(size_t)fill * t.W + wi] = sel_bits;
+    }
     const int ej = t.eos - 32 * wi;
-    if (ej >= 0 && ej < 32 && (fl & 2)) m |= 1u << ej;
+    if (ej >= 0 && ej < 32 && (fl & 2)) m |= 1u << ej;  // the EOS gate is stack-dependent: never cached
   }
   if (have) {
     mask[(size_t)b * t.W + wi] = m;
@@ -1004,15 +1060,21 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
       }
     }
   }
+  if (fill >= 0) __threadfence();  // the entry's words before its readiness
   __syncthreads();
   // one atomic per block counts the block for its row and carries whether it
-  // set a bit; the row's last block writes the status
+  // set a bit; the row's last block writes the status (and marks a cache
+  // entry the row filled ready: all blocks have written their words)
   if (threadIdx.x == 0) {
     const unsigned long long old = atomicAdd(&ctx[b].pack_done, 1ull + (s_any ? (1ull << 32) : 0ull));
     if ((uint32_t)old == gridDim.x - 1) {
       int st = atomicAdd(&ctx[b].status, 0);
       if (st == GRID_ST_OK && (old >> 32) == 0ull && !s_any) st = GRID_ST_EMPTY_MASK;
       d_status[b] = st;
+      if (fill >= 0) {
+        __threadfence();
+        atomicExch(cache.hdr + (size_t)fill * 16, 2u);
+      }
     }
   }
 }
@@ -1752,7 +1814,7 @@ int grid::launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratc
   const int zero_blocks = std::min(128, (int)((zero_words / 8 + kRowWarps * 32 * 4 - 1) / (kRowWarps * 32 * 4)) + 1);
   if (ev) GRID_CUDA(cudaEventRecord(ev[0], st));
   GRID_CUDA(launch_pdl(k_row, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx, m.rng,
-                       m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v));
+                       m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v, m.cache));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
   const int cd_blocks = (s->max_cd + 256 * kFilterPer - 1) / (256 * kFilterPer);
   const int vc_blocks = (s->max_vc + 256 * kFilterPer - 1) / (256 * kFilterPer);
@@ -1777,15 +1839,15 @@ int grid::launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratc
   if (!lg.p)
     GRID_CUDA(launch_pdl(k_pack<0>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
                          (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                         m.words_v, d_mask, d_status, (void*)nullptr, 0ll, 0));
+                         m.words_v, d_mask, d_status, (void*)nullptr, 0ll, 0, m.cache));
   else if (lg.dtype == GRID_DTYPE_F32)
     GRID_CUDA(launch_pdl(k_pack<1>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
                          (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok));
+                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok, m.cache));
   else
     GRID_CUDA(launch_pdl(k_pack<2>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
                          (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok));
+                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok, m.cache));
   if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
@@ -1806,6 +1868,86 @@ extern "C" int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint3
     return set_error(GRID_E_INVALID_ARG, "grid_masks_apply: bad arguments");
   const MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
                       c->surv, c->vsurv, c->cap, c->vcap, c->words_v};
+  FusedLogits lg;
+  lg.p = d_logits;
+  lg.dtype = dtype;
+  lg.stride = row_stride;
+  return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr, lg);
+}
+
+// ---------------------------------------------------------------------------
+// Configuration-keyed mask cache (Sec. 4.3, Def. T1 key, Prop. OBL-KEY1).
+struct grid_cache {
+  const grid_spec* s = nullptr;
+  CacheDev d;
+  Arena mem;
+};
+
+extern "C" int grid_cache_create(const grid_spec* s, int32_t n_entries, grid_cache** out) {
+  if (!s || !out || n_entries <= 0 || (n_entries & (n_entries - 1)) || n_entries > (1 << 20))
+    return set_error(GRID_E_INVALID_ARG, "grid_cache_create: n_entries must be a power of two in 1 .. 2^20");
+  *out = nullptr;
+  auto* c = new grid_cache();
+  c->s = s;
+  c->d.n = n_entries;
+  const size_t W = s->t.W;
+  int rc;
+  if ((rc = c->mem.alloc((size_t)n_entries * 16 * 4, (void**)&c->d.hdr)) ||
+      (rc = c->mem.alloc((size_t)n_entries * W * 4, (void**)&c->d.ci)) ||
+      (rc = c->mem.alloc((size_t)n_entries * W * 4, (void**)&c->d.sel)) ||
+      (rc = c->mem.alloc(4 * 8, (void**)&c->d.stats))) {
+    c->mem.release();
+    delete c;
+    return rc;
+  }
+  cudaError_t e = cudaMemset(c->d.hdr, 0, (size_t)n_entries * 16 * 4);
+  if (e == cudaSuccess) e = cudaMemset(c->d.stats, 0, 4 * 8);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    c->mem.release();
+    delete c;
+    return set_error(GRID_E_CUDA, std::string("grid_cache_create: ") + cudaGetErrorString(e));
+  }
+  *out = c;
+  return GRID_OK;
+}
+
+extern "C" void grid_cache_free(grid_cache* c) {
+  if (!c) return;
+  c->mem.release();
+  delete c;
+}
+
+extern "C" int grid_cache_clear(grid_cache* c, void* stream) {
+  if (!c) return set_error(GRID_E_INVALID_ARG, "grid_cache_clear: bad arguments");
+  GRID_CUDA(cudaMemsetAsync(c->d.hdr, 0, (size_t)c->d.n * 16 * 4, (cudaStream_t)stream));
+  GRID_CUDA(cudaMemsetAsync(c->d.stats, 0, 4 * 8, (cudaStream_t)stream));
+  return GRID_OK;
+}
+
+extern "C" int grid_cache_stats(const grid_cache* c, int64_t out[4]) {
+  if (!c || !out) return set_error(GRID_E_INVALID_ARG, "grid_cache_stats: bad arguments");
+  unsigned long long st[3];
+  std::vector<uint32_t> hdr((size_t)c->d.n * 16);
+  GRID_CUDA(cudaMemcpy(st, c->d.stats, 3 * 8, cudaMemcpyDeviceToHost));
+  GRID_CUDA(cudaMemcpy(hdr.data(), c->d.hdr, hdr.size() * 4, cudaMemcpyDeviceToHost));
+  int64_t ready = 0;
+  for (int i = 0; i < c->d.n; ++i) ready += hdr[(size_t)i * 16] == 2u;
+  out[0] = (int64_t)st[0];
+  out[1] = (int64_t)st[1];
+  out[2] = (int64_t)st[2];
+  out[3] = ready;
+  return GRID_OK;
+}
+
+extern "C" int grid_masks_cached(const grid_spec* s, const grid_configs* c, grid_cache* cache, uint32_t* d_mask,
+                                 int32_t* d_status, void* d_logits, int32_t dtype, int64_t row_stride, void* stream) {
+  if (!s || !c || !cache || !d_mask || !d_status || cache->s != s ||
+      (d_logits && (row_stride < s->t.V || (dtype != GRID_DTYPE_F32 && dtype != GRID_DTYPE_BF16))))
+    return set_error(GRID_E_INVALID_ARG, "grid_masks_cached: bad arguments (the cache must belong to the spec)");
+  MaskScratch m{c->ctx, c->rng, c->sel, c->verd0, c->verd1, c->A2, c->vcbits,
+                c->surv, c->vsurv, c->cap, c->vcap, c->words_v};
+  m.cache = cache->d;
   FusedLogits lg;
   lg.p = d_logits;
   lg.dtype = dtype;

@@ -35,6 +35,7 @@ struct RowCtx {
   int32_t nsurv[2];       // CD spellings that survived k_filter, per context (0: sigma, 1: sigma')
   int32_t nvs[2];         // verdict classes that survived k_filter, per context
   int32_t nrng;
+  int32_t chit, cfill;  // mask-cache entry this row reads (hit) or fills (miss), or -1
   uint32_t kill[8];  // bit b: first byte b ends the pending lexeme
   uint16_t ovl1[kMaxOvl];
 };
@@ -80,12 +81,27 @@ struct Arena {
 
 // Buffers of one mask step (owned by a grid_configs, or carved out of the
 // static area of grid_masks_static).
+// Device view of a configuration-keyed mask cache (grid_cache): per entry a
+// 16-word header -- [0] state (0 empty, 1 being filled, 2 ready), [1] kind
+// (1 = identifier position: a lexer state without a CI table), [2] lexer
+// state, [3] emit_ok, [4..7] A(sigma), [8..11] A(sigma') -- and W words of
+// the values of the context-independent bits (ci) and W words marking the
+// ids whose bits are the stack-dependent residue (sel).  n == 0: no cache.
+struct CacheDev {
+  uint32_t* hdr = nullptr;
+  uint32_t* ci = nullptr;
+  uint32_t* sel = nullptr;
+  unsigned long long* stats = nullptr;  // [0] lookups, [1] hits, [2] fills claimed
+  int n = 0;                            // entries, a power of two
+};
+
 struct MaskScratch {
   RowCtx* ctx;
   RowRanges* rng;
   uint32_t *sel, *verd0, *verd1, *A2, *vcbits;
   int32_t *surv, *vsurv;
   int cap, vcap, words_v;
+  CacheDev cache;
 };
 
 // Logits to mask in the same pass as the mask (grid_masks_apply), or none.

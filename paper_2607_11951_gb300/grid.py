@@ -25,7 +25,8 @@ EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_gramma
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
             "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_spec_set_work_counters", "grid_masks_static", "grid_forced_span",
-            "grid_reserve", "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
+            "grid_reserve", "grid_cache_create", "grid_cache_free", "grid_cache_clear", "grid_cache_stats",
+            "grid_masks_cached", "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
             "grid_audit_genesis", "grid_blake2b", "grid_fingerprint", "grid_apply_mask", "grid_configs_export"]
 
 
@@ -80,6 +81,11 @@ def lib():
         "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
         "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P, P]),
         "grid_reserve": (I32, [P, P, P, P, I32, P, P, I32, P, P]),
+        "grid_cache_create": (I32, [P, I32, ctypes.POINTER(P)]),
+        "grid_cache_free": (None, [P]),
+        "grid_cache_clear": (I32, [P, P]),
+        "grid_cache_stats": (I32, [P, ctypes.POINTER(I64)]),
+        "grid_masks_cached": (I32, [P, P, P, P, P, P, I32, I64, P]),
         "grid_configs_enable_audit": (I32, [P, P, P]),
         "grid_audit_append": (I32, [P, P, P, P, I32, P, P]),
         "grid_audit_seal": (I32, [P, P, P, ctypes.c_uint32, P, P]),
@@ -267,6 +273,43 @@ def grid_reserve(spec, cfg, cost, tokens, status, budget=None, safety=0, fire=No
     _check(lib().grid_reserve(spec, cfg, _ptr(cost), _ptr(tokens), tokens.shape[1], _ptr(status),
                               nul if budget is None else _ptr(budget), safety, nul if fire is None else _ptr(fire),
                               _stream(stream)))
+
+
+def grid_masks_cached(spec, cfg, cache, mask, status, logits=None, stream=None):
+    """grid_masks (logits None) or grid_masks_apply through a mask cache."""
+    assert mask.is_contiguous() and status.is_contiguous()
+    if logits is None:
+        lp, dt, stride = ctypes.c_void_p(None), GRID_DTYPE_F32, 0
+    else:
+        import torch
+        assert logits.stride(1) == 1
+        lp, stride = _ptr(logits), logits.stride(0)
+        dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
+    _check(lib().grid_masks_cached(getattr(spec, "h", spec), getattr(cfg, "h", cfg), getattr(cache, "h", cache),
+                                   _ptr(mask), _ptr(status), lp, dt, stride, _stream(stream)))
+
+
+class Cache:
+    """A configuration-keyed mask cache of a spec (n_entries a power of two)."""
+
+    def __init__(self, spec, n_entries=1024):
+        self.spec = spec
+        out = ctypes.c_void_p()
+        _check(lib().grid_cache_create(spec.h, n_entries, ctypes.byref(out)))
+        self.h = out
+
+    def clear(self, stream=None):
+        _check(lib().grid_cache_clear(self.h, _stream(stream)))
+
+    def stats(self):
+        out = (ctypes.c_int64 * 4)()
+        _check(lib().grid_cache_stats(self.h, out))
+        return dict(zip(["lookups", "hits", "fills", "ready"], list(out)))
+
+    def __del__(self):
+        if getattr(self, "h", None) and _lib is not None:
+            _lib.grid_cache_free(self.h)
+            self.h = None
 
 
 def grid_configs_enable_audit(spec, cfg, stream=None):

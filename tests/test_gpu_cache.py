@@ -1,0 +1,68 @@
+"""The configuration-keyed mask cache (Sec. 4.3, Prop. OBL-KEY1): cache-on
+equals cache-off, bit for bit, over randomized replays -- the same
+configurations masked through a cache that fills on first sight of a key and
+is read on every later step, rows sharing keys within a batch and across
+steps, identifier and generic positions -- for masks, statuses and the fused
+logits fill; and the cache is really used (hits)."""
+import numpy as np
+import pytest
+
+from tests.harness import GpuRun, unpack
+from workloads import configs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("name", ["tiny_expr", "sql_admin", "sql_select_only", "sql_shared"])
+def test_cache_on_equals_cache_off_over_replays(name):
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl = getattr(configs, name)()
+    run = GpuRun(wl)
+    assert (run.build_configs() == 0).all()
+    cache = G.Cache(run.spec, 256)
+    B, V = run.B, run.V
+    rng = np.random.default_rng(17)
+    m_on = torch.zeros_like(run.mask)
+    st_on = torch.zeros_like(run.status)
+    for step in range(5):
+        for rep in range(2):  # the second pass meets every key of the batch again
+            words, status = run.masks()
+            G.grid_masks_cached(run.spec, run.cfg, cache, m_on, st_on)
+            torch.cuda.synchronize()
+            assert (m_on.cpu().numpy().view(np.uint32) == words).all(), (name, step, rep)
+            assert (st_on.cpu().numpy() == status).all()
+        bits = unpack(words, V)
+        tok = np.full(B, -1, np.int32)
+        for b in range(B):
+            if status[b] == 0:
+                adm = np.flatnonzero(bits[b])
+                adm = adm[adm != wl["eos"]] if adm.size > 1 else adm
+                tok[b] = int(rng.choice(adm))
+        G.grid_advance(run.spec.h, run.cfg.h, run.cfg.h, torch.from_numpy(tok).cuda(), run.status)
+        torch.cuda.synchronize()
+    st = cache.stats()
+    assert st["hits"] >= B and st["ready"] > 0, st
+
+
+def test_cache_fused_logits_and_clear():
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl = configs.sql_select_only()
+    run = GpuRun(wl)
+    assert (run.build_configs() == 0).all()
+    cache = G.Cache(run.spec, 1024)
+    lg = torch.from_numpy(configs.logits(3, run.B, run.V)).cuda()
+    for rep in range(3):
+        a, b = lg.clone(), lg.clone()
+        m1, s1 = torch.zeros_like(run.mask), torch.zeros_like(run.status)
+        m2, s2 = torch.zeros_like(run.mask), torch.zeros_like(run.status)
+        G.grid_masks_apply(run.spec.h, run.cfg.h, m1, s1, a)
+        G.grid_masks_cached(run.spec, run.cfg, cache, m2, s2, b)
+        torch.cuda.synchronize()
+        assert torch.equal(m1, m2) and torch.equal(s1, s2) and torch.equal(a.view(torch.int32), b.view(torch.int32))
+        if rep == 1:
+            assert cache.stats()["hits"] > 0
+            cache.clear()
+            torch.cuda.synchronize()
+            assert cache.stats() == {"lookups": 0, "hits": 0, "fills": 0, "ready": 0}
