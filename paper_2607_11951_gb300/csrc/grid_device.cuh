@@ -122,6 +122,7 @@ struct Tables {
   const int32_t* first_of_byte;
   const uint8_t* first_byte_by_id;
   const uint32_t* id_valid;    // W words: bit set for the ids with a spelling (not EOS, special or padding)
+  const uint32_t* killw;       // Q * W: bit j of word (q, wi): id 32 wi + j's first byte ends a lexeme at q
   // CI tables (one per lexer state in the precomputed set; table 0 = start state)
   int ci_on;
   int n_tbl;

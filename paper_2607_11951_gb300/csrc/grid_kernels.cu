@@ -148,6 +148,22 @@ __global__ void k_events(Tables t, const uint16_t* __restrict__ cls_sp, const in
   }
 }
 
+// Per lexer state q and mask word wi, the ids whose first byte ends a pending
+// lexeme in state q (every id at the start state): the split of a row's ids
+// between sigma' and sigma that k_pack applies one word at a time.
+__global__ void k_killw(Tables t, uint32_t* __restrict__ out) {
+  const int wi = blockIdx.x * blockDim.x + threadIdx.x;
+  const int q = blockIdx.y;
+  if (wi >= t.W) return;
+  uint32_t w = 0u;
+  for (int j = 0; j < 32; ++j) {
+    const int id = 32 * wi + j;
+    const int by = id < t.Vp ? t.first_byte_by_id[id] : 0;
+    if (q == kStart || q == kDead || t.next[q * t.C + t.byte_class[by]] == kDead) w |= 1u << j;
+  }
+  out[(size_t)q * t.W + wi] = w;
+}
+
 // Terminal set of every class id (events and final tests of the verdict
 // classes use nothing else of a class).
 __global__ void k_class_sets(Tables t, uint4* __restrict__ out) {
@@ -895,7 +911,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
 // whose ids are all rejected is written with -inf without being read, a mixed
 // sector is read, blended and written, an accepted sector is not touched.
 constexpr int kPackWords = 256;
-template <int APPLY>
+template <int APPLY, bool CACHE>
 __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restrict__ ctx, const uint32_t* __restrict__ sel,
                                                      const uint32_t* __restrict__ vcbits, int vcw,
                                                      const uint32_t* __restrict__ verd0,
@@ -904,21 +920,17 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
                                                      void* __restrict__ logits, long long stride, int vec_ok,
                                                      CacheDev cache) {
   extern __shared__ __align__(16) uint32_t s_dyn[];  // class selections (2 nselw) | verdict-class bits (2 vcw)
-  __shared__ int s_fl, s_tb, s_any, s_hit, s_fill;
-  __shared__ uint32_t s_kill[8];
+  __shared__ int s_fl, s_tb, s_any, s_hit, s_fill, s_q;
   const int b = blockIdx.y;
   const int wi = blockIdx.x * kPackWords + threadIdx.x;
   const bool have = wi < t.W;
   const int nw = t.nselw;
   const int code_vc = t.ncls + 3, code_walk = t.ncls + 4;
-  // spec tables only, read before the wait on the walks: the ids' first
-  // bytes, which ids have a spelling, the start state's class codes
-  uint4 fb4[2], c04[4];
+  // spec tables only, read before the wait on the walks: which ids have a
+  // spelling, the start state's class codes
+  uint4 c04[4];
   uint32_t valid = 0u;
   if (have) {
-    const uint4* f = reinterpret_cast<const uint4*>(t.first_byte_by_id) + 2 * wi;
-    fb4[0] = f[0];
-    fb4[1] = f[1];
     const uint4* c = reinterpret_cast<const uint4*>(t.cls_by_id) + 4 * wi;
 #pragma unroll
     for (int k = 0; k < 4; ++k) c04[k] = c[k];
@@ -930,12 +942,12 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
     s_tb = rc.tbl0;
     s_fl = (rc.emit_ok ? 1 : 0) | (rc.eos_ok ? 2 : 0) | (rc.complete ? 4 : 0);
     s_any = 0;
-    s_hit = cache.n ? rc.chit : -1;
-    s_fill = cache.n ? rc.cfill : -1;
+    s_hit = CACHE ? rc.chit : -1;
+    s_fill = CACHE ? rc.cfill : -1;
+    s_q = rc.q;
   }
-  if (threadIdx.x < 8) s_kill[threadIdx.x] = rc.kill[threadIdx.x];
   __syncthreads();
-  const int fl = s_fl, tb = s_tb, hit = s_hit, fill = s_fill;
+  const int fl = s_fl, tb = s_tb, hit = CACHE ? s_hit : -1, fill = CACHE ? s_fill : -1;
   // a context that k_row did not select for (a completed row, sigma' without
   // a forced emission, sigma without a table) reads zeros
   {
@@ -957,7 +969,9 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
     // a cache hit gives the context-independent bits; only the residue ids
     // (verdict-class and walked) are decided here
     uint32_t todo = valid;
-    if (hit >= 0) {
+    // bit j: id 32 wi + j's first byte ends the pending lexeme (context sigma')
+    const uint32_t killw = t.killw[(size_t)s_q * t.W + wi];
+    if (CACHE && hit >= 0) {
       m = cache.ci[(size_t)hit * t.W + wi];
       todo = cache.sel[(size_t)hit * t.W + wi];
     }
@@ -968,7 +982,6 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
 #pragma unroll
       for (int k = 0; k < 4; ++k) ct4[k] = c[k];
     }
-    const uint32_t fbw[8] = {fb4[0].x, fb4[0].y, fb4[0].z, fb4[0].w, fb4[1].x, fb4[1].y, fb4[1].z, fb4[1].w};
     const uint32_t c0w[16] = {c04[0].x, c04[0].y, c04[0].z, c04[0].w, c04[1].x, c04[1].y, c04[1].z, c04[1].w,
                               c04[2].x, c04[2].y, c04[2].z, c04[2].w, c04[3].x, c04[3].y, c04[3].z, c04[3].w};
     uint32_t ctw[16];
@@ -986,8 +999,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
       if (!((todo >> j) & 1u)) continue;
-      const int by = (fbw[j >> 2] >> ((j & 3) * 8)) & 0xFF;
-      const int cx = (s_kill[by >> 5] >> (by & 31)) & 1u;
+      const int cx = (killw >> j) & 1u;
       const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
       uint32_t bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
       if (code >= code_vc && (!cx || (fl & 1))) {
@@ -997,13 +1009,13 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
         } else {
           bit = ((cx ? wv1 : wv0) >> j) & 1u;
         }
-        sel_bits |= 1u << j;
-      } else {
+        if (CACHE) sel_bits |= 1u << j;
+      } else if (CACHE) {
         ci_bits |= bit << j;
       }
       m |= bit << j;
     }
-    if (fill >= 0) {
+    if (CACHE && fill >= 0) {
       cache.ci[(size_t)fill * t.W + wi] = ci_bits;
       cache.sel[(size_t)fill * t.W + wi] = sel_bits;
     }
@@ -1060,7 +1072,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
       }
     }
   }
-  if (fill >= 0) __threadfence();  // the entry's words before its readiness
+  if (CACHE && fill >= 0) __threadfence();  // the entry's words before its readiness
   __syncthreads();
   // one atomic per block counts the block for its row and carries whether it
   // set a bit; the row's last block writes the status (and marks a cache
@@ -1071,7 +1083,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
       int st = atomicAdd(&ctx[b].status, 0);
       if (st == GRID_ST_OK && (old >> 32) == 0ull && !s_any) st = GRID_ST_EMPTY_MASK;
       d_status[b] = st;
-      if (fill >= 0) {
+      if (CACHE && fill >= 0) {
         __threadfence();
         atomicExch(cache.hdr + (size_t)fill * 16, 2u);
       }
@@ -1330,9 +1342,12 @@ static int set_smem_limits() {
   GRID_CUDA(cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_events, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   // k_pack: one row's class selections and verdict-class bits, two contexts
-  GRID_CUDA(cudaFuncSetAttribute(k_pack<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
-  GRID_CUDA(cudaFuncSetAttribute(k_pack<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
-  GRID_CUDA(cudaFuncSetAttribute(k_pack<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<0, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<0, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_pack<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
@@ -1693,6 +1708,12 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   if (nslot > 0)
     k_scatter_vc<<<(nslot + 255) / 256, 256, 0, st>>>(slot_tbl, slot_sp, slot_vc_c, nslot, t.NS, vc_sp);
   k_permute<<<(t.Vp + 255) / 256, 256, 0, st>>>(t, cls_sp, vc_sp, cls_by_id, vc_by_id, fb);
+  {
+    uint32_t* killw = nullptr;
+    if ((rc = a.alloc((size_t)t.Q * t.W * 4, (void**)&killw))) return fail_tmp(rc);
+    k_killw<<<dim3((t.W + 255) / 256, t.Q), 256, 0, st>>>(t, killw);
+    t.killw = killw;
+  }
   GRID_CUDA(cudaGetLastError());
   GRID_CUDA(cudaStreamSynchronize(st));
   tmp.release();
@@ -1836,18 +1857,21 @@ int grid::launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratc
   const size_t psmem = (size_t)(2 * std::max(1, t.nselw) + 2 * vcw) * 4;
   const int esz = lg.dtype == GRID_DTYPE_F32 ? 4 : 2;
   const int vec_ok = lg.p && ((uintptr_t)lg.p % 32 == 0) && ((lg.stride * esz) % 32 == 0);  // 32-byte sectors
-  if (!lg.p)
-    GRID_CUDA(launch_pdl(k_pack<0>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
-                         (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                         m.words_v, d_mask, d_status, (void*)nullptr, 0ll, 0, m.cache));
-  else if (lg.dtype == GRID_DTYPE_F32)
-    GRID_CUDA(launch_pdl(k_pack<1>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
-                         (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok, m.cache));
+  auto pack = [&](auto kern) {
+    return launch_pdl(kern, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
+                      (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1, m.words_v,
+                      d_mask, d_status, lg.p, (long long)lg.stride, lg.p ? vec_ok : 0, m.cache);
+  };
+  const bool cached = m.cache.n > 0;
+  const int mode = !lg.p ? 0 : (lg.dtype == GRID_DTYPE_F32 ? 1 : 2);
+  cudaError_t pe;
+  if (mode == 0)
+    pe = cached ? pack(k_pack<0, true>) : pack(k_pack<0, false>);
+  else if (mode == 1)
+    pe = cached ? pack(k_pack<1, true>) : pack(k_pack<1, false>);
   else
-    GRID_CUDA(launch_pdl(k_pack<2>, pgrid, dim3(kPackWords), psmem, st, t, m.ctx, (const uint32_t*)m.sel,
-                         (const uint32_t*)m.vcbits, vcw, (const uint32_t*)m.verd0, (const uint32_t*)m.verd1,
-                         m.words_v, d_mask, d_status, lg.p, lg.stride, vec_ok, m.cache));
+    pe = cached ? pack(k_pack<2, true>) : pack(k_pack<2, false>);
+  GRID_CUDA(pe);
   if (ev) GRID_CUDA(cudaEventRecord(ev[4], st));
   GRID_CUDA(cudaGetLastError());
   return GRID_OK;
