@@ -578,6 +578,41 @@ def main():
                   "entries_ready": c1["ready"],
                   "step": "grid_advance + grid_masks_cached (fused fp32 fill), cache warmed by one pass "
                           "over the 16 batches"}
+    # pass G: independent batch-32 steps on 4 streams at once (each stream
+    # with its own scratch, mask and status; no two streams on one batch at a
+    # time): how much of the GPU one step leaves idle, beside the sequential
+    # value above
+    NS_ = 4
+    strs = [torch.cuda.Stream(device=dev) for _ in range(NS_)]
+    scr = [G.Configs(spec, B) for _ in range(NS_)]
+    msk = [torch.zeros((B, W), dtype=torch.int32, device=dev) for _ in range(NS_)]
+    sts = [torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(NS_)]
+
+    def conc_run(n):
+        start = torch.cuda.Event(enable_timing=True)
+        done = [torch.cuda.Event() for _ in range(NS_)]
+        start.record(stream)
+        for x in strs:
+            x.wait_event(start)
+        for k in range(n):
+            j, i = k % NS_, k % N_BATCHES
+            G.grid_advance(spec.h, cfgs[i].h, scr[j].h, toks[i], sts[j], strs[j])
+            G.grid_masks_apply(spec.h, scr[j].h, msk[j], sts[j], logits[i], strs[j])
+        for j in range(NS_):
+            done[j].record(strs[j])
+            stream.wait_event(done[j])
+        end = torch.cuda.Event(enable_timing=True)
+        end.record(stream)
+        return start, end
+
+    conc_run(N_BATCHES)
+    torch.cuda.synchronize()
+    ca, cb = conc_run(args.steps)
+    torch.cuda.synchronize()
+    conc_ms = ca.elapsed_time(cb)
+    concurrent = {"streams": NS_, "masks_per_s": B * args.steps / (conc_ms * 1e-3),
+                  "ms_per_step": conc_ms / args.steps,
+                  "step": "grid_advance + grid_masks_apply, K steps dealt round-robin to the streams"}
     clocks = clk.stop()
     work = torch.zeros(4, dtype=torch.int64, device=dev)  # pass E
     G.grid_spec_set_work_counters(spec.h, work)
@@ -714,7 +749,7 @@ def main():
                 "call_us": {"grid_advance": adv_us, "grid_masks_apply": masks_us},
                 "kernel_us": kern_us, "dominant_kernel": dominant,
                 "roofline": roof, "roofline_apply": roof_apply, "cpu_baseline": cpu_base, "e2e": e2e,
-                "mask_cache": cache_line,
+                "mask_cache": cache_line, "concurrent_batches": concurrent,
                 "gpu_launches": args.steps * (1 + len(MASK_KERNELS)), "clocks": clocks,
                 "timing": "value: K steps between two events; p50/p99 and call_us: a second pass of K "
                           "steps with events around each call; kernel_us: a third pass with events "
