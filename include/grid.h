@@ -137,6 +137,17 @@ void grid_grammar_free(grid_grammar* g);
  * out[5]=byte classes, out[6]=lexicon-trie nodes, out[7]=categories. */
 int grid_grammar_info(const grid_grammar* g, int64_t out[8]);
 
+/* Debug/test view of the identifier trie over the union of the L3 lexicons
+ * (host memory, n_nodes = out[6] of grid_grammar_info): nodes in BFS order
+ * with each node's children in increasing byte order, node 0 the root (the
+ * empty prefix); the children of node n are the edges cstart[n] ..
+ * cstart[n+1]-1 (cstart: n_nodes + 1 entries), edge e spelling byte
+ * cbyte[e] and leading to node cnode[e] (n_nodes - 1 edges); pcats[n] has
+ * bit c set when node n's string is a prefix of a word of category c,
+ * wcats[n] when it is a word of category c. */
+int grid_grammar_lexicon_trie(const grid_grammar* g, int32_t* cstart, uint8_t* cbyte, int32_t* cnode,
+                              uint32_t* pcats, uint32_t* wcats, int64_t n_nodes);
+
 /* Def. 3: build the DFS-ordered byte trie of the vocabulary.  Token t has the
  * spelling bytes[offsets[t] .. offsets[t+1]) (host memory, read during the call).
  * `eos_id` and the `n_special` ids in `special_ids` are excluded from the trie

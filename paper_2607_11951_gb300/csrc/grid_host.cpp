@@ -1350,6 +1350,19 @@ extern "C" int grid_grammar_info(const grid_grammar* g, int64_t out[8]) {
   return GRID_OK;
 }
 
+extern "C" int grid_grammar_lexicon_trie(const grid_grammar* g, int32_t* cstart, uint8_t* cbyte, int32_t* cnode,
+                                        uint32_t* pcats, uint32_t* wcats, int64_t n_nodes) {
+  if (!g || !cstart || !pcats || !wcats || n_nodes != g->h.LN || (n_nodes > 1 && (!cbyte || !cnode)))
+    return set_error(GRID_E_INVALID_ARG, "grid_grammar_lexicon_trie: bad arguments (n_nodes must be the node count)");
+  const HostGrammar& h = g->h;
+  std::copy(h.lx_cstart.begin(), h.lx_cstart.end(), cstart);
+  std::copy(h.lx_cbyte.begin(), h.lx_cbyte.end(), cbyte);
+  std::copy(h.lx_cnode.begin(), h.lx_cnode.end(), cnode);
+  std::copy(h.lx_pcats.begin(), h.lx_pcats.end(), pcats);
+  std::copy(h.lx_wcats.begin(), h.lx_wcats.end(), wcats);
+  return GRID_OK;
+}
+
 extern "C" int grid_load_vocab(const uint8_t* bytes, const int64_t* offsets, int32_t V, int32_t eos_id,
                                const int32_t* special_ids, int32_t n_special, grid_vocab** out) {
   if (!out || !offsets || V <= 0 || n_special < 0 || (n_special > 0 && !special_ids))

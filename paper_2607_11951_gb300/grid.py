@@ -21,7 +21,7 @@ GRID_ST_OK, GRID_ST_NONVIABLE, GRID_ST_STACK_OVERFLOW, GRID_ST_TOKEN_NOT_ALLOWED
 GRID_ST_EMPTY_MASK, GRID_ST_BOUND, GRID_ST_COMPLETE = 4, 5, 6
 GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 
-EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info",
+EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info", "grid_grammar_lexicon_trie",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
             "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_spec_set_work_counters", "grid_masks_static", "grid_forced_span",
@@ -67,6 +67,7 @@ def lib():
         "grid_compile": (I32, [ctypes.c_char_p, SZ, ctypes.c_char_p, P, I32, P, ctypes.POINTER(P)]),
         "grid_grammar_free": (None, [P]),
         "grid_grammar_info": (I32, [P, ctypes.POINTER(I64)]),
+        "grid_grammar_lexicon_trie": (I32, [P, P, P, P, P, P, I64]),
         "grid_load_vocab": (I32, [P, P, I32, I32, P, I32, ctypes.POINTER(P)]),
         "grid_vocab_free": (None, [P]),
         "grid_vocab_info": (I32, [P, ctypes.POINTER(I64)]),
@@ -176,6 +177,20 @@ def grid_grammar_info(g):
     keys = ["terminals", "lalr_states", "nonterminals", "productions", "dfa_states",
             "byte_classes", "lexicon_nodes", "categories"]
     return dict(zip(keys, list(out)))
+
+
+def grid_grammar_lexicon_trie(g):
+    """The identifier trie's arrays (numpy): cstart, cbyte, cnode, pcats, wcats."""
+    import numpy as np
+    n = grid_grammar_info(g)["lexicon_nodes"]
+    cstart = np.zeros(n + 1, np.int32)
+    cbyte = np.zeros(max(1, n - 1), np.uint8)
+    cnode = np.zeros(max(1, n - 1), np.int32)
+    pc = np.zeros(n, np.uint32)
+    wc = np.zeros(n, np.uint32)
+    p = lambda a: a.ctypes.data_as(ctypes.c_void_p)
+    _check(lib().grid_grammar_lexicon_trie(g, p(cstart), p(cbyte), p(cnode), p(pc), p(wc), n))
+    return cstart, cbyte[:max(0, n - 1)], cnode[:max(0, n - 1)], pc, wc
 
 
 def grid_load_vocab(tokens, eos: int, specials=()):

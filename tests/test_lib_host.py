@@ -143,3 +143,44 @@ def test_lexicon_trie_and_vocab_sizes_against_python():
     info = v.info()
     assert info["spellings"] == len(kept)
     assert info["bytes"] == sum(len(t) for t in kept)
+
+
+def test_lexicon_trie_arrays_against_python_bfs():
+    """The identifier trie's arrays equal a trie built here by breadth-first
+    numbering with children in byte order: child ranges, edge bytes, child
+    ids, and the prefix / word category masks, for a random lexicon with
+    shared prefixes, words in both categories and one-letter words."""
+    rng = np.random.default_rng(9)
+    alpha = b"abcdefghij_0123"
+    def word():
+        n = int(rng.integers(1, 7))
+        return bytes([alpha[int(rng.integers(0, 10))]]) + bytes(alpha[int(i)] for i in rng.integers(0, len(alpha), n - 1))
+    tables = sorted({word() for _ in range(120)})
+    cols = sorted({word() for _ in range(200)} | set(tables[:30]) | {b"a", b"b"})
+    g = G.Grammar(grammar_text("sql"), [], {"TABLE_NAME": tables, "COLUMN_NAME": cols})
+    cstart, cbyte, cnode, pc, wc = G.grid_grammar_lexicon_trie(g.h)
+    # reference trie: BFS from the root, children by byte
+    cats = {0: tables, 1: cols}
+    strings = sorted({w[:k] for c in cats.values() for w in c for k in range(len(w) + 1)}, key=lambda x: (len(x), x))
+    children = {}
+    for x in strings[1:]:
+        children.setdefault(x[:-1], []).append(x)
+    order, seen = [b""], 0
+    while seen < len(order):
+        x = order[seen]
+        seen += 1
+        order.extend(sorted(children.get(x, []), key=lambda y: y[-1]))
+    idx = {x: i for i, x in enumerate(order)}
+    assert len(order) == len(pc)
+    want_start, want_byte, want_node = [0], [], []
+    for x in order:
+        for y in sorted(children.get(x, []), key=lambda y: y[-1]):
+            want_byte.append(y[-1])
+            want_node.append(idx[y])
+        want_start.append(len(want_byte))
+    assert cstart.tolist() == want_start
+    assert cbyte.tolist() == want_byte and cnode.tolist() == want_node
+    for x in order:
+        p = sum(1 << c for c, ws in cats.items() if any(w.startswith(x) for w in ws))
+        w = sum(1 << c for c, ws in cats.items() if x in set(ws))
+        assert pc[idx[x]] == p and wc[idx[x]] == w, x
