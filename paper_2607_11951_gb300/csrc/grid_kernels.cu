@@ -230,21 +230,30 @@ __global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const u
 }
 
 // ---------------- mask step ----------------
-// Class selection for allowed set A: bit c = set(c) meets A u I, the OR of
-// the class masks of the terminals in A u I (lanes take the words).
-__device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, int lane) {
-  const Bits4 AI = A | t.ign;
-  for (int w0 = lane; w0 < t.nselw; w0 += 32) {
-    uint32_t acc = 0u;
-    Bits4 r = AI;
-    while (r.any()) {
+// Class selection for allowed set A, word w0: bit c = set(c) meets A u I,
+// the OR of the class masks of the terminals in A u I.  The terminals' words
+// are loaded kSelBatch at a time, so that a word costs |A u I| / kSelBatch
+// memory round trips instead of |A u I|.
+constexpr int kSelBatch = 16;
+__device__ __forceinline__ uint32_t select_word(const Tables& t, const Bits4 AI, int w0) {
+  uint32_t acc = 0u;
+  Bits4 r = AI;
+  while (r.any()) {
+    uint32_t v[kSelBatch];
+#pragma unroll
+    for (int k = 0; k < kSelBatch; ++k) {
       const int tau = r.lowest();
-      r.clear_lowest();
-      acc |= __ldg(&t.cls_mask[(size_t)tau * t.nselw + w0]);
+      v[k] = 0u;
+      if (tau >= 0) {
+        r.clear_lowest();
+        v[k] = __ldg(&t.cls_mask[(size_t)tau * t.nselw + w0]);
+      }
     }
-    if (w0 == (t.ncls >> 5)) acc |= 1u << (t.ncls & 31);  // the code "always"
-    out[w0] = acc;
+#pragma unroll
+    for (int k = 0; k < kSelBatch; ++k) acc |= v[k];
   }
+  if (w0 == (t.ncls >> 5)) acc |= 1u << (t.ncls & 31);  // the code "always"
+  return acc;
 }
 
 // One block per row (kRowWarps warps), plus clearing blocks after the rows.
@@ -258,7 +267,7 @@ __device__ void select_classes(const Tables& t, const Bits4 A, uint32_t* out, in
 // ballots), and then the allowed set after that shift is A2 (walks and verdict
 // classes simulate nothing before their second shift).  Phase 2: warp 0 lays
 // out the live first-byte ranges that continue the lexeme (rows without a CI
-// table; they need A0), warps 1 and 2 select the contexts' CI classes.
+// table; they need A0), warps 1 .. 5 select the contexts' CI classes.
 // Clearing blocks zero both verdict bitmaps and the verdict-class bits.
 __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
                                                         RowRanges* __restrict__ rng, uint32_t* __restrict__ A2,
@@ -267,7 +276,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
                                                         int n_vcbits, int B, int words_v, CacheDev cache) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
-  __shared__ uint16_t s_stk[kStackWin];
+  __shared__ __align__(16) uint16_t s_stk[kStackWin];
   __shared__ uint16_t s_ovl1[kMaxOvl];
   __shared__ uint16_t s_ovl2[kRowJobWarps][kMaxOvl * 32];
   __shared__ uint16_t s_scr[kRowJobWarps][kMaxOvl * 32];
@@ -299,6 +308,13 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x;
   RowCtx& r = ctx[b];
+  // the stack window is read before the depth is known (one 16-byte access
+  // per thread), in parallel with the configuration
+  const uint16_t* base = c.stack + (size_t)b * t.D;
+  const bool vec = t.D % 8 == 0 && kStackWin / 8 <= kRowWarps * 32;
+  uint4 sv = make_uint4(0u, 0u, 0u, 0u);
+  if (vec && (int)threadIdx.x < kStackWin / 8 && (int)threadIdx.x * 8 < t.D)
+    sv = reinterpret_cast<const uint4*>(base)[threadIdx.x];
   if (threadIdx.x == 0) {
     const int lx = c.lx[b];
     s_row[0] = c.flags[b] & 1;
@@ -314,9 +330,12 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   __syncthreads();
   const int complete = s_row[0], depth = s_row[1], q = s_row[2], lx = s_row[3];
   const uint32_t pc0 = s_pc[0], wc0 = s_pc[1];
-  const uint16_t* base = c.stack + (size_t)b * t.D;
   if (depth <= kStackWin) {  // the reduce chains below read the stack top repeatedly
-    for (int i = threadIdx.x; i < depth; i += blockDim.x) s_stk[i] = base[i];
+    if (vec) {
+      if ((int)threadIdx.x < ((depth + 7) >> 3)) reinterpret_cast<uint4*>(s_stk)[threadIdx.x] = sv;
+    } else {
+      for (int i = threadIdx.x; i < depth; i += blockDim.x) s_stk[i] = base[i];
+    }
     base = s_stk;
   }
   __syncthreads();
@@ -501,10 +520,15 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
         s_total0 = total0;
         s_nrng = nrng;
       }
-    } else if (warp == 1 && t.ci_on && tbl0 >= 0) {
-      select_classes(ts, A0, sel + ((size_t)b * 2) * t.nselw, lane);
-    } else if (warp == 2 && t.ci_on && emit_ok) {
-      select_classes(ts, A1, sel + ((size_t)b * 2 + 1) * t.nselw, lane);
+    } else if (warp >= 1 && t.ci_on) {
+      // both contexts' selection words, one per lane of warps 1 ..
+      const Bits4 AI0 = A0 | ts.ign, AI1 = A1 | ts.ign;
+      const int nw = t.nselw;
+      for (int i = (warp - 1) * 32 + lane; i < 2 * nw; i += (kRowWarps - 1) * 32) {
+        const int cx = i >= nw ? 1 : 0, w0 = i - cx * nw;
+        if (cx ? !emit_ok : tbl0 < 0) continue;
+        sel[((size_t)b * 2 + cx) * nw + w0] = select_word(ts, cx ? AI1 : AI0, w0);
+      }
     }
   }
   __syncthreads();
@@ -1094,7 +1118,11 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
 // One warp per row.  The lanes copy the row's stack for an out-of-place
 // advance and mirror it in shared memory (16-byte accesses when the row
 // stride allows them); lane 0 then feeds the tokens, with its overlay and
-// simulation scratch in shared memory.
+// simulation scratch in shared memory.  The loads that start a row are issued
+// as two independent chains: the configuration and then its stack (the first
+// 256 entries are read before the depth is known), and the first token with
+// its spelling.
+constexpr int kAdvSpec = 32;  // 16-byte stack accesses issued per lane before the depth is known
 __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs cin, DevConfigs cout,
                                                              const int32_t* __restrict__ tokens, int n_steps,
                                                              int32_t* __restrict__ d_status, int B, int copy) {
@@ -1107,19 +1135,48 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x * kAdvWarps + warp;
   if (b >= B) return;
-  const DevConfigs& from = copy ? cin : cout;
-  const int depth0 = from.depth[b];
-  const uint16_t* src = from.stack + (size_t)b * t.D;
+  // chain 1: the row's configuration (lanes 0-3), the speculative stack read
+  const uint16_t* src = (copy ? cin.stack : cout.stack) + (size_t)b * t.D;
   uint16_t* stack = cout.stack + (size_t)b * t.D;
-  // the row's stack is mirrored in shared memory while it fits; the global
-  // copy is always written and stays authoritative
+  int cf = 0;
+  if (lane < 4) {
+    const int32_t* f = lane == 0 ? (copy ? cin.depth : cout.depth)
+                     : lane == 1 ? (copy ? cin.q : cout.q)
+                     : lane == 2 ? (copy ? cin.lx : cout.lx)
+                                 : (copy ? cin.flags : cout.flags);
+    cf = f[b];
+  }
+  uint32_t cpc = 0u, cwc = 0u;  // category bits of the pending lexeme's trie node (lane 2)
+  if (lane == 2 && cf >= 0) {
+    cpc = t.lx_pcats[cf];
+    cwc = t.lx_wcats[cf];
+  }
+  const bool vec = t.D % 8 == 0;  // rows start on 16-byte boundaries: 8 entries per access
+  const uint4* s4 = reinterpret_cast<const uint4*>(src);
+  uint4 sv = make_uint4(0u, 0u, 0u, 0u);
+  if (vec && lane < kAdvSpec && lane * 8 < t.D) sv = s4[lane];
+  // chain 2: the first token and its spelling (lane 0)
+  int tok0 = -1, sp0 = -1;
+  Spell spl0;
+  spl0.len = 0;
+  if (lane == 0 && n_steps > 0) {
+    tok0 = tokens[(size_t)b * n_steps];
+    if (tok0 >= 0 && tok0 < t.V && tok0 != t.eos) {
+      sp0 = t.spell_of_id[tok0];
+      if (sp0 >= 0) spl0 = load_spell(t, sp0);
+    }
+  }
+  const int depth0 = __shfl_sync(0xffffffffu, cf, 0);
   bool use_win = depth0 <= kStackWin;
-  if (t.D % 8 == 0) {  // rows start on 16-byte boundaries: 8 entries per access
+  if (vec) {
     const int n8 = (depth0 + 7) >> 3;  // (n8 * 8 <= D: the last access stays inside the row)
-    const uint4* s4 = reinterpret_cast<const uint4*>(src);
     uint4* d4 = reinterpret_cast<uint4*>(stack);
     uint4* w4 = reinterpret_cast<uint4*>(s_stk[warp]);
-    for (int i = lane; i < n8; i += 32) {
+    if (lane < n8) {
+      if (copy) d4[lane] = sv;
+      if (use_win) w4[lane] = sv;
+    }
+    for (int i = lane + kAdvSpec; i < n8; i += 32) {
       const uint4 v = s4[i];
       if (copy) d4[i] = v;
       if (use_win) w4[i] = v;
@@ -1136,16 +1193,14 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
     uint64_t* hdst = cout.hs + (size_t)b * t.D;
     for (int i = lane; i < depth0; i += 32) hdst[i] = hsrc[i];
   }
-  if (copy && lane == 0) {
-    cout.depth[b] = depth0;
-    cout.q[b] = cin.q[b];
-    cout.lx[b] = cin.lx[b];
-    cout.flags[b] = cin.flags[b];
-  }
+  const int q0 = __shfl_sync(0xffffffffu, cf, 1);
+  const int lx0 = __shfl_sync(0xffffffffu, cf, 2);
+  const int flags0 = __shfl_sync(0xffffffffu, cf, 3);
+  const uint32_t pc0 = __shfl_sync(0xffffffffu, cpc, 2), wc0 = __shfl_sync(0xffffffffu, cwc, 2);
   __syncwarp();
   if (lane != 0) return;
-  int depth = depth0, q = cout.q[b], lx = cout.lx[b], flags = cout.flags[b];
-  uint32_t pc = lx >= 0 ? t.lx_pcats[lx] : 0u, wcat = lx >= 0 ? t.lx_wcats[lx] : 0u;
+  int depth = depth0, q = q0, lx = lx0, flags = flags0;
+  uint32_t pc = pc0, wcat = wc0;
   int status = GRID_ST_OK;
   const int mc = max_chain_of(t);
   Walker w;
@@ -1176,12 +1231,12 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
       flags |= 1;
       continue;
     }
-    const int s = t.spell_of_id[tok];
+    const int s = k == 0 ? sp0 : t.spell_of_id[tok];
     if (s < 0) {
       status = GRID_ST_TOKEN_NOT_ALLOWED;
       break;
     }
-    const int r = walk_bytes(ts, w, load_spell(t, s), mc);
+    const int r = walk_bytes(ts, w, k == 0 ? spl0 : load_spell(t, s), mc);
     if (r < 0) {
       status = GRID_ST_BOUND;
       break;
