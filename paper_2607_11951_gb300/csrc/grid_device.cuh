@@ -138,7 +138,9 @@ struct Tables {
   const int32_t* vc_off;
   const uint16_t* vc_rec;     // kRecLen per verdict class
   const uint16_t* vc_first;   // class id of each verdict class's first event
-  const uint32_t* vc_by_id;   // n_tbl * V: verdict class (within its table) of kClsVC spellings
+  const uint32_t* vc_by_id;   // n_tbl * V: verdict class (within its table) of kClsVC spellings, or NULL
+                              // when the class codes carry it (vc_inline)
+  int vc_inline;              // 1: a verdict-class id's code is ncls + kPackCodes + its class index
   const uint32_t* cls_sets;   // ncls * 4: terminal set of every class id
   const uint32_t* cls_mask;   // T1 * nselw: bit c of row tau = tau is in class c's set
   const uint32_t* acc_sym;    // S: the symbol entering each state (audit node hash)

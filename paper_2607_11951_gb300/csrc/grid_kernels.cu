@@ -70,7 +70,8 @@ constexpr int kRowJobWarps = 4;  // k_row: warps 2 .. 5 compute the allowed sets
 // Class codes as k_pack reads them: CI class ids 0..ncls-1, then these five
 // (so that one bit test of the row's class selection covers CI, always and
 // never, and only verdict-class and walked tokens need a second lookup).
-constexpr int kPackCodes = 5;  // ncls + 0 always, +1 never, +2 n/a, +3 verdict class, +4 walked
+constexpr int kPackCodes = 5;  // ncls + 0 always, +1 never, +2 n/a, +3 verdict class, +4 walked;
+                               // with vc_inline, ncls + 5 + v: verdict class v of the code's table
 constexpr int kWalkRowsCached = 256;  // rows whose queue bounds k_walk keeps in shared memory
 constexpr int kLaneOvl = 32;     // overlay / scratch entries per walk lane (shared memory)
 constexpr int kMaxStage = 96 * 1024;
@@ -224,8 +225,9 @@ __global__ void k_permute(Tables t, const uint16_t* __restrict__ cls_sp, const u
     uint16_t code = c;  // the k_pack code of c
     if (c >= kClsFirstCode)
       code = (uint16_t)(t.ncls + (c == kClsAcc ? 0 : c == kClsRej ? 1 : c == kClsNA ? 2 : c == kClsVC ? 3 : 4));
+    if (c == kClsVC && t.vc_inline) code = (uint16_t)(t.ncls + kPackCodes + vc_sp[(size_t)k * t.NS + s]);
     cls_by_id[(size_t)k * t.Vp + id] = code;
-    vc_by_id[(size_t)k * t.Vp + id] = c == kClsVC ? vc_sp[(size_t)k * t.NS + s] : 0xFFFFFFFFu;
+    if (vc_by_id) vc_by_id[(size_t)k * t.Vp + id] = c == kClsVC ? vc_sp[(size_t)k * t.NS + s] : 0xFFFFFFFFu;
   }
 }
 
@@ -949,7 +951,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
   const int wi = blockIdx.x * kPackWords + threadIdx.x;
   const bool have = wi < t.W;
   const int nw = t.nselw;
-  const int code_vc = t.ncls + 3, code_walk = t.ncls + 4;
+  const int code_vc = t.ncls + 3, code_walk = t.ncls + 4, code_vc0 = t.ncls + kPackCodes;
   // spec tables only, read before the wait on the walks: which ids have a
   // spelling, the start state's class codes
   uint4 c04[4];
@@ -1025,13 +1027,15 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
       if (!((todo >> j) & 1u)) continue;
       const int cx = (killw >> j) & 1u;
       const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
-      uint32_t bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
+      uint32_t bit = 0u;  // codes of verdict classes and walks in a context k_row left out: rejected
+      if (code < code_vc) bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
       if (code >= code_vc && (!cx || (fl & 1))) {
-        if (code == code_vc) {
-          const uint32_t v = t.vc_by_id[(size_t)(cx ? 0 : tb) * t.Vp + 32 * wi + j];
-          bit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
-        } else {
+        if (code == code_walk) {
           bit = ((cx ? wv1 : wv0) >> j) & 1u;
+        } else {  // the verdict class: in the code, or looked up
+          const uint32_t v = code >= code_vc0 ? (uint32_t)(code - code_vc0)
+                                              : t.vc_by_id[(size_t)(cx ? 0 : tb) * t.Vp + 32 * wi + j];
+          bit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
         }
         if (CACHE) sel_bits |= 1u << j;
       } else if (CACHE) {
@@ -1630,11 +1634,9 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
   if ((rc = tmp.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&cls_sp)) ||
       (rc = tmp.alloc((size_t)t.n_tbl * t.NS * 2, (void**)&key_sp)) ||
       (rc = tmp.alloc((size_t)t.n_tbl * 8, (void**)&counts_d)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.Vp * 2, (void**)&cls_by_id)) ||
-      (rc = a.alloc((size_t)t.n_tbl * t.Vp * 4, (void**)&vc_by_id)) || (rc = a.alloc((size_t)t.Vp, (void**)&fb)))
+      (rc = a.alloc((size_t)t.n_tbl * t.Vp * 2, (void**)&cls_by_id)) || (rc = a.alloc((size_t)t.Vp, (void**)&fb)))
     return fail_tmp(rc);
   t.cls_by_id = cls_by_id;
-  t.vc_by_id = vc_by_id;
   t.first_byte_by_id = fb;
   GRID_CUDA(cudaMemsetAsync(counts_d, 0, (size_t)t.n_tbl * 8, st));
   const dim3 cgrid(std::max(1, std::min((t.NS + 255) / 256, 4 * s->sms)), t.n_tbl);
@@ -1762,6 +1764,11 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
     return fail_tmp(rc);
   if (nslot > 0)
     k_scatter_vc<<<(nslot + 255) / 256, 256, 0, st>>>(slot_tbl, slot_sp, slot_vc_c, nslot, t.NS, vc_sp);
+  // verdict-class indices ride in the 16-bit class codes when they fit;
+  // otherwise k_pack looks them up per id
+  t.vc_inline = t.ncls + kPackCodes + s->max_vc <= 0xFFFF ? 1 : 0;
+  if (!t.vc_inline && (rc = a.alloc((size_t)t.n_tbl * t.Vp * 4, (void**)&vc_by_id))) return fail_tmp(rc);
+  t.vc_by_id = vc_by_id;
   k_permute<<<(t.Vp + 255) / 256, 256, 0, st>>>(t, cls_sp, vc_sp, cls_by_id, vc_by_id, fb);
   {
     uint32_t* killw = nullptr;
