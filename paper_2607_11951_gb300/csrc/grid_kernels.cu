@@ -1727,15 +1727,24 @@ extern "C" int grid_specialize(const grid_grammar* g, const grid_vocab* v, void*
       }
       h_vc[i] = it->second;
     }
-    // order each table's records by event count, so that the 32 records of a
-    // walk item tend to cost alike
+    // order each table's records by their event sequences (then the event
+    // count and the final class): a walk item evaluates 32 neighbouring
+    // records on one row's stack, and records that share their first events
+    // take the same path through them, so the warp's lanes stay together
     for (int k = 0; k < t.n_tbl; ++k) {
       const int n = (int)(per[k].size() / kRecLen);
       std::vector<int32_t> ord(n), pos(n);
       for (int i = 0; i < n; ++i) ord[i] = i;
       const uint16_t* R = per[k].data();
-      std::stable_sort(ord.begin(), ord.end(), [&](int x, int y) {
-        return R[(size_t)x * kRecLen] < R[(size_t)y * kRecLen];
+      std::sort(ord.begin(), ord.end(), [&](int x, int y) {
+        const uint16_t* a = R + (size_t)x * kRecLen;
+        const uint16_t* b = R + (size_t)y * kRecLen;
+        const int m = std::min<int>(a[0], b[0]);
+        for (int e = 0; e < m; ++e)
+          if (a[2 + e] != b[2 + e]) return a[2 + e] < b[2 + e];
+        if (a[0] != b[0]) return a[0] < b[0];
+        if (a[1] != b[1]) return a[1] < b[1];
+        return x < y;
       });
       std::vector<uint16_t> sorted(per[k].size());
       for (int i = 0; i < n; ++i) {
