@@ -5,9 +5,11 @@ V = 151,936 (seeded, BPE-like, ~3% multi-word tokens), batch B = 32 parser
 configurations at prefixes of U[50, 2000] tokens, fp32 logits N(0, 3).
 
 One step = the whole per-token hot path for one batch, through the C ABI:
-  grid_advance (out-of-place, one admitted token per row)
-  -> grid_masks_apply (allowed sets + EOS gate, trie walk, id-order packing,
-     with the in-place -inf fill of the fp32 logits fused into the packing).
+  grid_advance_masks: the advance (out-of-place, one admitted token per row)
+  fed inside the mask step's first kernel, then the mask step (allowed sets +
+  EOS gate, trie walk, id-order packing, with the in-place -inf fill of the
+  fp32 logits fused into the packing).  The same step as two calls
+  (grid_advance, then grid_masks_apply) is timed beside it.
 The standalone grid_apply_mask kernel is timed on its own for its HBM
 roofline (fp32 headline batch; bf16 B=256 in the cold-schema line).
 Steps rotate over 16 distinct pre-built batches (512 prefixes); their logits
@@ -194,7 +196,7 @@ def headline_config(B, V):
     return {"workload": "sql_select_only", "B": B, "V": V, "prefix_tokens": "U[50,2000]",
             "schema": "200 tables x 30 columns", "logits": "f32 N(0,3)",
             "batches": N_BATCHES, "l2": "rotating inputs: 16 logits batches = 311 MB > L2",
-            "step": "grid_advance + grid_masks_apply (mask step with the logits fill fused)"}
+            "step": "grid_advance_masks (the advance inside the mask step, the logits fill fused)"}
 
 
 def run_reference(args):
@@ -402,8 +404,7 @@ def run_cold(args):
     logits = [torch.from_numpy(configs.logits(200 + k, B, V)).to(dev).to(torch.bfloat16) for k in range(2)]
 
     def step(k):
-        G.grid_advance(spec.h, c.h, scratch.h, tok, status, stream)
-        G.grid_masks_apply(spec.h, scratch.h, mask, status, logits[k % 2], stream)
+        G.grid_advance_masks(spec.h, c.h, scratch.h, tok, mask, status, logits[k % 2], stream)
 
     t = _time_steps(step, args.steps, warmup, stream)
     apply_us = _apply_alone(G, mask, logits, args.steps, stream)
@@ -419,7 +420,7 @@ def run_cold(args):
                       "roofline_apply_bf16": _roof_apply(B, V, 2, apply_us, "k_apply<bf16> (grid_apply_mask)"),
                       "config": {"workload": "sql_cold_schema", "B": B, "V": V, "schema": "1,000 x 50",
                                  "logits": "bf16 N(0,3), 2 rotating batches = 156 MB > L2",
-                                 "step": "grid_advance + grid_masks_apply"},
+                                 "step": "grid_advance_masks"},
                       "clocks": clocks}), flush=True)
 
 
@@ -498,12 +499,14 @@ def main():
         i = k % N_BATCHES
         if ev:
             ev[0].record(stream)
-        G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
+        G.grid_advance_masks(spec.h, cfgs[i].h, scratch.h, toks[i], mask, status, logits[i], stream)
         if ev:
             ev[1].record(stream)
+
+    def step2(k):  # the same step as two calls
+        i = k % N_BATCHES
+        G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
         G.grid_masks_apply(spec.h, scratch.h, mask, status, logits[i], stream)
-        if ev:
-            ev[2].record(stream)
 
     for k in range(args.warmup):
         step(k)
@@ -513,13 +516,13 @@ def main():
     torch.cuda.synchronize()
     # Passes of K steps each, back to back:
     #   A  the timed region of `value`: events only at its two ends
-    #   B  per-step events around the two calls (p50/p99, per-call means)
+    #   B  per-step events around the call (p50/p99)
     #   C  events recorded by the library around each kernel of the mask step
     #   D  the standalone grid_apply_mask (its HBM roofline)
     #   E  one more pass with k_walk's work counters on (their counts only;
     #      counting slows the kernel, so no time is taken from this pass)
     # Events cost the GPU a little time each, so A carries none between steps.
-    ev_b = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    ev_b = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     ev_c = [[torch.cuda.Event(enable_timing=True) for _ in range(len(MASK_KERNELS) + 1)] for _ in range(args.steps)]
     for ev in ev_b + ev_c:  # create each event by a first record, before the library sees its handle
         for e in ev:
@@ -550,6 +553,23 @@ def main():
         step(args.warmup + k)
     torch.cuda.synchronize()
     G.grid_configs_set_events(scratch.h, [])
+    # the two-call step (grid_advance, then grid_masks_apply), and the advance
+    # alone, back to back
+    sa_, sb_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sa_.record(stream)
+    for k in range(args.steps):
+        step2(args.warmup + k)
+    sb_.record(stream)
+    sa_.synchronize()
+    sb_.synchronize()
+    two_call_ms = sa_.elapsed_time(sb_) / args.steps
+    sa_.record(stream)
+    for k in range(args.steps):
+        i = (args.warmup + k) % N_BATCHES
+        G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
+    sb_.record(stream)
+    torch.cuda.synchronize()
+    adv_alone_us = sa_.elapsed_time(sb_) * 1e3 / args.steps
     apply_us = _apply_alone(G, mask, logits, args.steps, stream)  # pass D
     # pass F: the same steps through the configuration-keyed mask cache (its
     # context-independent part read from entries filled by earlier steps; the
@@ -596,8 +616,7 @@ def main():
             x.wait_event(start)
         for k in range(n):
             j, i = k % NS_, k % N_BATCHES
-            G.grid_advance(spec.h, cfgs[i].h, scr[j].h, toks[i], sts[j], strs[j])
-            G.grid_masks_apply(spec.h, scr[j].h, msk[j], sts[j], logits[i], strs[j])
+            G.grid_advance_masks(spec.h, cfgs[i].h, scr[j].h, toks[i], msk[j], sts[j], logits[i], strs[j])
         for j in range(NS_):
             done[j].record(strs[j])
             stream.wait_event(done[j])
@@ -612,7 +631,7 @@ def main():
     conc_ms = ca.elapsed_time(cb)
     concurrent = {"streams": NS_, "masks_per_s": B * args.steps / (conc_ms * 1e-3),
                   "ms_per_step": conc_ms / args.steps,
-                  "step": "grid_advance + grid_masks_apply, K steps dealt round-robin to the streams"}
+                  "step": "grid_advance_masks, K steps dealt round-robin to the streams"}
     clocks = clk.stop()
     work = torch.zeros(4, dtype=torch.int64, device=dev)  # pass E
     G.grid_spec_set_work_counters(spec.h, work)
@@ -622,10 +641,9 @@ def main():
     G.grid_spec_set_work_counters(spec.h, None)
     work = [int(x) / N_BATCHES for x in work.cpu().tolist()]
     total_ms = max_over_ranks(total_ms, ws, dev)
-    per_step = [e[0].elapsed_time(e[2]) * 1e3 for e in ev_b]
-    adv_us = statistics.mean(e[0].elapsed_time(e[1]) * 1e3 for e in ev_b)
-    masks_us = statistics.mean(e[1].elapsed_time(e[2]) * 1e3 for e in ev_b)
-    kern_us = {"k_advance": adv_us}
+    per_step = [e[0].elapsed_time(e[1]) * 1e3 for e in ev_b]
+    call_us = statistics.mean(per_step)
+    kern_us = {}
     for j, name in enumerate(MASK_KERNELS):
         kern_us[name] = statistics.mean(e[j].elapsed_time(e[j + 1]) * 1e3 for e in ev_c)
     per_step.sort()
@@ -670,8 +688,8 @@ def main():
                 copy_in(k + 1)
             stream.wait_event(ev_in[j])
             stream.wait_event(ev_out[j])  # mask/status buffers of step k-2 read back
-            G.grid_advance(spec.h, cfgs[i].h, scratch.h, d_tok[j], d_status[j], stream)
-            G.grid_masks_apply(spec.h, scratch.h, d_mask[j], d_status[j], d_logits[j], stream)
+            G.grid_advance_masks(spec.h, cfgs[i].h, scratch.h, d_tok[j], d_mask[j], d_status[j], d_logits[j],
+                                 stream)
             ev_used[j].record(stream)
             d2h.wait_event(ev_used[j])
             with torch.cuda.stream(d2h):
@@ -719,7 +737,7 @@ def main():
     walk_us = kern_us["k_walk"]
     units = sum(work)
     peak_units = sms * LANES * mhz * 1e6 / 1e9
-    roof_walk = {"kernel": "k_walk (grid_masks_apply)", "bound": "alu",
+    roof_walk = {"kernel": "k_walk (grid_advance_masks)", "bound": "alu",
                  "unit": "G work units/s (lexer steps + ACTION + GOTO lookups + verdict-class events)",
                  "achieved": units / (walk_us * 1e-6) / 1e9, "peak": peak_units,
                  "peak_kind": "derived: %d SMs x %d lanes of shared-memory pipe per clock x %.0f MHz sampled" %
@@ -746,15 +764,18 @@ def main():
                 "config": headline_config(B, V),
                 "p50_us": p50, "p99_us": p99,
                 "token_checks_per_s": value * V,
-                "call_us": {"grid_advance": adv_us, "grid_masks_apply": masks_us},
+                "call_us": {"grid_advance_masks": call_us},
+                "two_call_step": {"ms_per_step": two_call_ms, "masks_per_s": B / (two_call_ms * 1e-3),
+                                  "grid_advance_alone_us": adv_alone_us,
+                                  "step": "grid_advance, then grid_masks_apply (the advance in its own kernel)"},
                 "kernel_us": kern_us, "dominant_kernel": dominant,
                 "roofline": roof, "roofline_apply": roof_apply, "cpu_baseline": cpu_base, "e2e": e2e,
                 "mask_cache": cache_line, "concurrent_batches": concurrent,
-                "gpu_launches": args.steps * (1 + len(MASK_KERNELS)), "clocks": clocks,
+                "gpu_launches": args.steps * len(MASK_KERNELS), "clocks": clocks,
                 "timing": "value: K steps between two events; p50/p99 and call_us: a second pass of K "
                           "steps with events around each call; kernel_us: a third pass with events "
-                          "around each kernel of the mask step (k_pack includes the logits fill); "
-                          "roofline_apply: the standalone grid_apply_mask, back to back"}
+                          "around each kernel of the step (k_row includes the advance, k_pack the logits "
+                          "fill); roofline_apply: the standalone grid_apply_mask, back to back"}
         print(json.dumps(line), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()

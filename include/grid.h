@@ -227,6 +227,24 @@ int grid_masks(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int3
 int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask, int32_t* d_status,
                      void* d_logits, int32_t dtype, int64_t row_stride, void* stream);
 
+/* One decoding step in one launch sequence (Sec. 6.1 steps 7 then 1-5):
+ * grid_advance of d_tokens (n_steps per row) from `in` into `out`, then
+ * grid_masks of `out` -- or grid_masks_apply when d_logits is not NULL
+ * (dtype and row_stride as there; d_logits NULL: no fill, dtype and
+ * row_stride unused).  The advance runs inside the mask step's first kernel,
+ * one row per block, so that a row's mask preparation starts as soon as its
+ * own token is fed.  The configurations and masks are those of grid_advance
+ * followed by grid_masks(_apply); d_status[b] is the advance's status when
+ * row b's token was refused (GRID_ST_TOKEN_NOT_ALLOWED, GRID_ST_STACK_OVERFLOW,
+ * GRID_ST_BOUND, GRID_ST_COMPLETE: the row keeps its configuration as of the
+ * last accepted token and is masked there), else the mask step's.  `in` and
+ * `out` follow grid_advance's rules (same B and D, audit on both or neither;
+ * in == out advances in place); the scratch and overlap rule of grid_masks
+ * apply to `out`.  Enqueue only. */
+int grid_advance_masks(const grid_spec* s, const grid_configs* in, grid_configs* out, const int32_t* d_tokens,
+                       int32_t n_steps, uint32_t* d_mask, int32_t* d_status, void* d_logits, int32_t dtype,
+                       int64_t row_stride, void* stream);
+
 /* Measurement hook: with n_events == 5, every later grid_masks on `c` records
  * events[0..4] (cudaEvent_t, created by the caller) on its stream before its
  * first kernel and after each of its four kernels (per-row allowed sets, EOS

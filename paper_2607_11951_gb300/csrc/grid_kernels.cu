@@ -258,6 +258,177 @@ __device__ __forceinline__ uint32_t select_word(const Tables& t, const Bits4 AI,
   return acc;
 }
 
+// The configuration one warp leaves after feeding its row's tokens (lane 0's
+// values; `win`: the warp's shared-memory window holds the row's stack).
+struct AdvOut {
+  int depth, q, lx, flags, status;
+  uint32_t pc, wc;
+  bool win;
+};
+
+// Advance of row b by one warp (Sec. 3.1 parser step, Sec. 4.1 byte walk).
+// The lanes copy the row's stack for an out-of-place advance and mirror it in
+// `win` (kStackWin entries, 16-byte accesses when the row stride allows them);
+// lane 0 then feeds the tokens, with its overlay and simulation scratch in
+// `lo` / `ls`, and writes the configuration it leaves (and the row's status
+// when d_status is given).  The loads that start a row are issued as two
+// independent chains: the configuration and then its stack (the first 256
+// entries are read before the depth is known), and the first token with its
+// spelling.  Returns in lane 0 only; the other lanes return once the copy is
+// done.
+constexpr int kAdvSpec = 32;  // 16-byte stack accesses issued per lane before the depth is known
+__device__ __forceinline__ bool advance_warp(const Tables& t, const Tables& ts, const DevConfigs& cin,
+                                             const DevConfigs& cout, const int32_t* __restrict__ tokens,
+                                             int n_steps, int32_t* __restrict__ d_status, int b, int copy,
+                                             int lane, uint16_t* win, LArr lo, LArr ls, AdvOut& out) {
+  // chain 1: the row's configuration (lanes 0-3), the speculative stack read
+  const uint16_t* src = (copy ? cin.stack : cout.stack) + (size_t)b * t.D;
+  uint16_t* stack = cout.stack + (size_t)b * t.D;
+  int cf = 0;
+  if (lane < 4) {
+    const int32_t* f = lane == 0 ? (copy ? cin.depth : cout.depth)
+                     : lane == 1 ? (copy ? cin.q : cout.q)
+                     : lane == 2 ? (copy ? cin.lx : cout.lx)
+                                 : (copy ? cin.flags : cout.flags);
+    cf = f[b];
+  }
+  uint32_t cpc = 0u, cwc = 0u;  // category bits of the pending lexeme's trie node (lane 2)
+  if (lane == 2 && cf >= 0) {
+    cpc = t.lx_pcats[cf];
+    cwc = t.lx_wcats[cf];
+  }
+  const bool vec = t.D % 8 == 0;  // rows start on 16-byte boundaries: 8 entries per access
+  const uint4* s4 = reinterpret_cast<const uint4*>(src);
+  uint4 sv = make_uint4(0u, 0u, 0u, 0u);
+  if (vec && lane < kAdvSpec && lane * 8 < t.D) sv = s4[lane];
+  // chain 2: the first token and its spelling (lane 0)
+  int tok0 = -1, sp0 = -1;
+  Spell spl0;
+  spl0.len = 0;
+  if (lane == 0 && n_steps > 0) {
+    tok0 = tokens[(size_t)b * n_steps];
+    if (tok0 >= 0 && tok0 < t.V && tok0 != t.eos) {
+      sp0 = t.spell_of_id[tok0];
+      if (sp0 >= 0) spl0 = load_spell(t, sp0);
+    }
+  }
+  const int depth0 = __shfl_sync(0xffffffffu, cf, 0);
+  bool use_win = depth0 <= kStackWin;
+  if (vec) {
+    const int n8 = (depth0 + 7) >> 3;  // (n8 * 8 <= D: the last access stays inside the row)
+    uint4* d4 = reinterpret_cast<uint4*>(stack);
+    uint4* w4 = reinterpret_cast<uint4*>(win);
+    if (lane < n8) {
+      if (copy) d4[lane] = sv;
+      if (use_win) w4[lane] = sv;
+    }
+    for (int i = lane + kAdvSpec; i < n8; i += 32) {
+      const uint4 v = s4[i];
+      if (copy) d4[i] = v;
+      if (use_win) w4[i] = v;
+    }
+  } else {
+    for (int i = lane; i < depth0; i += 32) {
+      const uint16_t v = src[i];
+      if (copy) stack[i] = v;
+      if (use_win) win[i] = v;
+    }
+  }
+  if (copy && cout.hs) {  // the node hashes travel with the stack
+    const uint64_t* hsrc = cin.hs + (size_t)b * t.D;
+    uint64_t* hdst = cout.hs + (size_t)b * t.D;
+    for (int i = lane; i < depth0; i += 32) hdst[i] = hsrc[i];
+  }
+  const int q0 = __shfl_sync(0xffffffffu, cf, 1);
+  const int lx0 = __shfl_sync(0xffffffffu, cf, 2);
+  const int flags0 = __shfl_sync(0xffffffffu, cf, 3);
+  const uint32_t pc0 = __shfl_sync(0xffffffffu, cpc, 2), wc0 = __shfl_sync(0xffffffffu, cwc, 2);
+  __syncwarp();
+  if (lane != 0) return false;
+  int depth = depth0, q = q0, lx = lx0, flags = flags0;
+  uint32_t pc = pc0, wcat = wc0;
+  int status = GRID_ST_OK;
+  const int mc = max_chain_of(t);
+  Walker w;
+  for (int k = 0; k < n_steps; ++k) {
+    const int tok = tokens[(size_t)b * n_steps + k];
+    if (tok < 0) continue;
+    if (flags & 1) {
+      status = GRID_ST_COMPLETE;
+      break;
+    }
+    if (tok >= t.V) {
+      status = GRID_ST_TOKEN_NOT_ALLOWED;
+      break;
+    }
+    walker_init(w, lo, ls, kMaxOvl, use_win ? win : stack, depth, nullptr, 0, q, lx, pc, wcat, nullptr, nullptr);
+    if (tok == t.eos) {
+      const int e = eos_gate(ts, w, mc);
+      if (e < 0) {
+        status = GRID_ST_BOUND;
+        break;
+      }
+      if (e == 0) {
+        status = GRID_ST_TOKEN_NOT_ALLOWED;
+        break;
+      }
+      flags |= 1;
+      continue;
+    }
+    const int s = k == 0 ? sp0 : t.spell_of_id[tok];
+    if (s < 0) {
+      status = GRID_ST_TOKEN_NOT_ALLOWED;
+      break;
+    }
+    const int r = walk_bytes(ts, w, k == 0 ? spl0 : load_spell(t, s), mc);
+    if (r < 0) {
+      status = GRID_ST_BOUND;
+      break;
+    }
+    if (r == 0) {
+      status = GRID_ST_TOKEN_NOT_ALLOWED;
+      break;
+    }
+    if (w.keep + w.m > t.D) {
+      status = GRID_ST_STACK_OVERFLOW;
+      break;
+    }
+    for (int i = 0; i < w.m; ++i) stack[w.keep + i] = w.ovl[i];
+    if (cout.hs) {  // rolling hash of every pushed node: O(1) per push
+      uint64_t* hrow = cout.hs + (size_t)b * t.D;
+      uint64_t hp = hrow[w.keep - 1];
+      for (int i = 0; i < w.m; ++i) {
+        hp = node_hash(hp, t.acc_sym[w.ovl[i]]);
+        hrow[w.keep + i] = hp;
+      }
+    }
+    if (use_win && w.keep + w.m <= kStackWin) {
+      for (int i = 0; i < w.m; ++i) win[w.keep + i] = w.ovl[i];
+    } else {
+      use_win = false;
+    }
+    depth = w.keep + w.m;
+    q = w.q;
+    lx = w.lx;
+    pc = w.pc;
+    wcat = w.wc;
+  }
+  cout.depth[b] = depth;
+  cout.q[b] = q;
+  cout.lx[b] = lx;
+  cout.flags[b] = flags;
+  if (d_status) d_status[b] = status;
+  out.depth = depth;
+  out.q = q;
+  out.lx = lx;
+  out.flags = flags;
+  out.status = status;
+  out.pc = pc;
+  out.wc = wcat;
+  out.win = use_win;
+  return true;
+}
+
 // One block per row (kRowWarps warps), plus clearing blocks after the rows.
 // Phase 1, every warp at once: warp 0 finds the first bytes that end the
 // pending lexeme; warp 1 makes the forced emission of the pending lexeme
@@ -271,11 +442,18 @@ __device__ __forceinline__ uint32_t select_word(const Tables& t, const Bits4 AI,
 // out the live first-byte ranges that continue the lexeme (rows without a CI
 // table; they need A0), warps 1 .. 5 select the contexts' CI classes.
 // Clearing blocks zero both verdict bitmaps and the verdict-class bits.
+// With ADV the row's tokens are fed first (advance_warp on warp 0, from
+// adv.cin into c), and the row is masked in the configuration that leaves:
+// the advance of one row and the mask preparation of another overlap, and
+// the stack window is taken from the advance.  The row's status is then the
+// advance's error, if its token was refused, else the mask step's.
+template <bool ADV>
 __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, RowCtx* __restrict__ ctx,
                                                         RowRanges* __restrict__ rng, uint32_t* __restrict__ A2,
                                                         uint32_t* __restrict__ sel, uint32_t* __restrict__ verd0,
                                                         uint32_t* __restrict__ verd1, uint32_t* __restrict__ vcbits,
-                                                        int n_vcbits, int B, int words_v, CacheDev cache) {
+                                                        int n_vcbits, int B, int words_v, CacheDev cache,
+                                                        AdvArgs adv) {
   extern __shared__ __align__(16) uint8_t smem[];
   __shared__ Tables ts;
   __shared__ __align__(16) uint16_t s_stk[kStackWin];
@@ -285,7 +463,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   __shared__ uint32_t s_A0[4], s_A1[4], s_keep[8], s_kill[8];
   __shared__ int s_row[8];  // complete, depth, q, lx, emit_ok, keep1, m1, eos_ok
   __shared__ uint32_t s_pc[2];
-  __shared__ int s_status, s_total0, s_nrng;
+  __shared__ int s_status, s_total0, s_nrng, s_adv[2];
   if ((int)blockIdx.x >= B) {
     // clearing blocks: zero both verdict bitmaps and the verdict-class bits of every row
     pdl_wait();
@@ -310,30 +488,54 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x;
   RowCtx& r = ctx[b];
-  // the stack window is read before the depth is known (one 16-byte access
-  // per thread), in parallel with the configuration
   const uint16_t* base = c.stack + (size_t)b * t.D;
-  const bool vec = t.D % 8 == 0 && kStackWin / 8 <= kRowWarps * 32;
+  const bool vec = !ADV && t.D % 8 == 0 && kStackWin / 8 <= kRowWarps * 32;
   uint4 sv = make_uint4(0u, 0u, 0u, 0u);
-  if (vec && (int)threadIdx.x < kStackWin / 8 && (int)threadIdx.x * 8 < t.D)
-    sv = reinterpret_cast<const uint4*>(base)[threadIdx.x];
-  if (threadIdx.x == 0) {
-    const int lx = c.lx[b];
-    s_row[0] = c.flags[b] & 1;
-    s_row[1] = c.depth[b];
-    s_row[2] = c.q[b];
-    s_row[3] = lx;
-    s_pc[0] = lx >= 0 ? t.lx_pcats[lx] : 0u;
-    s_pc[1] = lx >= 0 ? t.lx_wcats[lx] : 0u;
-    s_status = GRID_ST_OK;
-    s_total0 = 0;
-    s_nrng = 0;
+  if (ADV) {
+    // the row's tokens, on warp 0 (overlay and scratch in job warp 0's area,
+    // which phase 1 uses only after the barrier below)
+    AdvOut o;
+    if (warp == 0 && advance_warp(t, ts, adv.cin, c, adv.tokens, adv.n_steps, nullptr, b, adv.copy, lane, s_stk,
+                                  LArr{s_scr[0], 1}, LArr{s_scr[0] + kMaxOvl, 1}, o)) {
+      s_row[0] = o.flags & 1;
+      s_row[1] = o.depth;
+      s_row[2] = o.q;
+      s_row[3] = o.lx;
+      s_pc[0] = o.pc;
+      s_pc[1] = o.wc;
+      s_adv[0] = o.status;
+      s_adv[1] = o.win ? 1 : 0;
+      s_status = GRID_ST_OK;
+      s_total0 = 0;
+      s_nrng = 0;
+    }
+  } else {
+    // the stack window is read before the depth is known (one 16-byte access
+    // per thread), in parallel with the configuration
+    if (vec && (int)threadIdx.x < kStackWin / 8 && (int)threadIdx.x * 8 < t.D)
+      sv = reinterpret_cast<const uint4*>(base)[threadIdx.x];
+    if (threadIdx.x == 0) {
+      const int lx = c.lx[b];
+      s_row[0] = c.flags[b] & 1;
+      s_row[1] = c.depth[b];
+      s_row[2] = c.q[b];
+      s_row[3] = lx;
+      s_pc[0] = lx >= 0 ? t.lx_pcats[lx] : 0u;
+      s_pc[1] = lx >= 0 ? t.lx_wcats[lx] : 0u;
+      s_adv[0] = GRID_ST_OK;
+      s_adv[1] = 0;
+      s_status = GRID_ST_OK;
+      s_total0 = 0;
+      s_nrng = 0;
+    }
   }
   __syncthreads();
   const int complete = s_row[0], depth = s_row[1], q = s_row[2], lx = s_row[3];
   const uint32_t pc0 = s_pc[0], wc0 = s_pc[1];
   if (depth <= kStackWin) {  // the reduce chains below read the stack top repeatedly
-    if (vec) {
+    if (ADV && s_adv[1]) {
+      // the advance left the row's stack in the window
+    } else if (vec) {
       if ((int)threadIdx.x < ((depth + 7) >> 3)) reinterpret_cast<uint4*>(s_stk)[threadIdx.x] = sv;
     } else {
       for (int i = threadIdx.x; i < depth; i += blockDim.x) s_stk[i] = base[i];
@@ -600,7 +802,7 @@ __global__ void __launch_bounds__(kRowWarps * 32) k_row(Tables t, DevConfigs c, 
     r.nrng = s_nrng;
   }
   for (int i = threadIdx.x; i < m1; i += blockDim.x) r.ovl1[i] = s_ovl1[i];
-  if (threadIdx.x == 0) r.status = complete ? GRID_ST_COMPLETE : s_status;
+  if (threadIdx.x == 0) r.status = s_adv[0] != GRID_ST_OK ? s_adv[0] : (complete ? GRID_ST_COMPLETE : s_status);
 }
 
 // grid = (cd_blocks + vc_blocks, B, 2), 256 threads, kFilterPer records per
@@ -1119,14 +1321,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
   }
 }
 
-// One warp per row.  The lanes copy the row's stack for an out-of-place
-// advance and mirror it in shared memory (16-byte accesses when the row
-// stride allows them); lane 0 then feeds the tokens, with its overlay and
-// simulation scratch in shared memory.  The loads that start a row are issued
-// as two independent chains: the configuration and then its stack (the first
-// 256 entries are read before the depth is known), and the first token with
-// its spelling.
-constexpr int kAdvSpec = 32;  // 16-byte stack accesses issued per lane before the depth is known
+// One warp per row (advance_warp).
 __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs cin, DevConfigs cout,
                                                              const int32_t* __restrict__ tokens, int n_steps,
                                                              int32_t* __restrict__ d_status, int B, int copy) {
@@ -1139,145 +1334,9 @@ __global__ void __launch_bounds__(kAdvWarps * 32) k_advance(Tables t, DevConfigs
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x * kAdvWarps + warp;
   if (b >= B) return;
-  // chain 1: the row's configuration (lanes 0-3), the speculative stack read
-  const uint16_t* src = (copy ? cin.stack : cout.stack) + (size_t)b * t.D;
-  uint16_t* stack = cout.stack + (size_t)b * t.D;
-  int cf = 0;
-  if (lane < 4) {
-    const int32_t* f = lane == 0 ? (copy ? cin.depth : cout.depth)
-                     : lane == 1 ? (copy ? cin.q : cout.q)
-                     : lane == 2 ? (copy ? cin.lx : cout.lx)
-                                 : (copy ? cin.flags : cout.flags);
-    cf = f[b];
-  }
-  uint32_t cpc = 0u, cwc = 0u;  // category bits of the pending lexeme's trie node (lane 2)
-  if (lane == 2 && cf >= 0) {
-    cpc = t.lx_pcats[cf];
-    cwc = t.lx_wcats[cf];
-  }
-  const bool vec = t.D % 8 == 0;  // rows start on 16-byte boundaries: 8 entries per access
-  const uint4* s4 = reinterpret_cast<const uint4*>(src);
-  uint4 sv = make_uint4(0u, 0u, 0u, 0u);
-  if (vec && lane < kAdvSpec && lane * 8 < t.D) sv = s4[lane];
-  // chain 2: the first token and its spelling (lane 0)
-  int tok0 = -1, sp0 = -1;
-  Spell spl0;
-  spl0.len = 0;
-  if (lane == 0 && n_steps > 0) {
-    tok0 = tokens[(size_t)b * n_steps];
-    if (tok0 >= 0 && tok0 < t.V && tok0 != t.eos) {
-      sp0 = t.spell_of_id[tok0];
-      if (sp0 >= 0) spl0 = load_spell(t, sp0);
-    }
-  }
-  const int depth0 = __shfl_sync(0xffffffffu, cf, 0);
-  bool use_win = depth0 <= kStackWin;
-  if (vec) {
-    const int n8 = (depth0 + 7) >> 3;  // (n8 * 8 <= D: the last access stays inside the row)
-    uint4* d4 = reinterpret_cast<uint4*>(stack);
-    uint4* w4 = reinterpret_cast<uint4*>(s_stk[warp]);
-    if (lane < n8) {
-      if (copy) d4[lane] = sv;
-      if (use_win) w4[lane] = sv;
-    }
-    for (int i = lane + kAdvSpec; i < n8; i += 32) {
-      const uint4 v = s4[i];
-      if (copy) d4[i] = v;
-      if (use_win) w4[i] = v;
-    }
-  } else {
-    for (int i = lane; i < depth0; i += 32) {
-      const uint16_t v = src[i];
-      if (copy) stack[i] = v;
-      if (use_win) s_stk[warp][i] = v;
-    }
-  }
-  if (copy && cout.hs) {  // the node hashes travel with the stack
-    const uint64_t* hsrc = cin.hs + (size_t)b * t.D;
-    uint64_t* hdst = cout.hs + (size_t)b * t.D;
-    for (int i = lane; i < depth0; i += 32) hdst[i] = hsrc[i];
-  }
-  const int q0 = __shfl_sync(0xffffffffu, cf, 1);
-  const int lx0 = __shfl_sync(0xffffffffu, cf, 2);
-  const int flags0 = __shfl_sync(0xffffffffu, cf, 3);
-  const uint32_t pc0 = __shfl_sync(0xffffffffu, cpc, 2), wc0 = __shfl_sync(0xffffffffu, cwc, 2);
-  __syncwarp();
-  if (lane != 0) return;
-  int depth = depth0, q = q0, lx = lx0, flags = flags0;
-  uint32_t pc = pc0, wcat = wc0;
-  int status = GRID_ST_OK;
-  const int mc = max_chain_of(t);
-  Walker w;
-  const LArr lo{s_lo[warp], 1}, ls{s_ls[warp], 1};
-  for (int k = 0; k < n_steps; ++k) {
-    const int tok = tokens[(size_t)b * n_steps + k];
-    if (tok < 0) continue;
-    if (flags & 1) {
-      status = GRID_ST_COMPLETE;
-      break;
-    }
-    if (tok >= t.V) {
-      status = GRID_ST_TOKEN_NOT_ALLOWED;
-      break;
-    }
-    walker_init(w, lo, ls, kMaxOvl, use_win ? s_stk[warp] : stack, depth, nullptr, 0, q, lx, pc, wcat, nullptr,
-                nullptr);
-    if (tok == t.eos) {
-      const int e = eos_gate(ts, w, mc);
-      if (e < 0) {
-        status = GRID_ST_BOUND;
-        break;
-      }
-      if (e == 0) {
-        status = GRID_ST_TOKEN_NOT_ALLOWED;
-        break;
-      }
-      flags |= 1;
-      continue;
-    }
-    const int s = k == 0 ? sp0 : t.spell_of_id[tok];
-    if (s < 0) {
-      status = GRID_ST_TOKEN_NOT_ALLOWED;
-      break;
-    }
-    const int r = walk_bytes(ts, w, k == 0 ? spl0 : load_spell(t, s), mc);
-    if (r < 0) {
-      status = GRID_ST_BOUND;
-      break;
-    }
-    if (r == 0) {
-      status = GRID_ST_TOKEN_NOT_ALLOWED;
-      break;
-    }
-    if (w.keep + w.m > t.D) {
-      status = GRID_ST_STACK_OVERFLOW;
-      break;
-    }
-    for (int i = 0; i < w.m; ++i) stack[w.keep + i] = w.ovl[i];
-    if (cout.hs) {  // rolling hash of every pushed node: O(1) per push
-      uint64_t* hrow = cout.hs + (size_t)b * t.D;
-      uint64_t hp = hrow[w.keep - 1];
-      for (int i = 0; i < w.m; ++i) {
-        hp = node_hash(hp, t.acc_sym[w.ovl[i]]);
-        hrow[w.keep + i] = hp;
-      }
-    }
-    if (use_win && w.keep + w.m <= kStackWin) {
-      for (int i = 0; i < w.m; ++i) s_stk[warp][w.keep + i] = w.ovl[i];
-    } else {
-      use_win = false;
-    }
-    depth = w.keep + w.m;
-    q = w.q;
-    lx = w.lx;
-    pc = w.pc;
-    wcat = w.wc;
-  }
-  cout.depth[b] = depth;
-  cout.q[b] = q;
-  cout.lx[b] = lx;
-  cout.flags[b] = flags;
-  d_status[b] = status;
+  AdvOut out;
+  advance_warp(t, ts, cin, cout, tokens, n_steps, d_status, b, copy, lane, s_stk[warp], LArr{s_lo[warp], 1},
+               LArr{s_ls[warp], 1}, out);
 }
 
 // In-place -inf fill, grid = (blocks per row, B): threads stride over a row's
@@ -1407,7 +1466,8 @@ static int set_smem_limits() {
   GRID_CUDA(cudaFuncSetAttribute(k_pack<0, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_pack<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_pack<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
-  GRID_CUDA(cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_row<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
+  GRID_CUDA(cudaFuncSetAttribute(k_row<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_walk<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
   GRID_CUDA(cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn));
@@ -1898,15 +1958,21 @@ extern "C" int grid_advance(const grid_spec* s, const grid_configs* in, grid_con
 // The four kernels of one mask step on `st`; `ev` (5 events or NULL) is
 // recorded before the first kernel and after each.
 int grid::launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, int B, uint32_t* d_mask,
-                       int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg) {
+                       int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg,
+                       const AdvArgs* adv) {
   const Tables& t = s->t;
   const int vcw = std::max(1, s->vcw);
   const int n_vcbits = B * 2 * vcw;
   const size_t zero_words = (size_t)B * m.words_v * 2 + n_vcbits;
   const int zero_blocks = std::min(128, (int)((zero_words / 8 + kRowWarps * 32 * 4 - 1) / (kRowWarps * 32 * 4)) + 1);
   if (ev) GRID_CUDA(cudaEventRecord(ev[0], st));
-  GRID_CUDA(launch_pdl(k_row, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx, m.rng,
-                       m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v, m.cache));
+  if (adv)
+    GRID_CUDA(launch_pdl(k_row<true>, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx,
+                         m.rng, m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v, m.cache, *adv));
+  else
+    GRID_CUDA(launch_pdl(k_row<false>, dim3(B + zero_blocks), dim3(kRowWarps * 32), t.blob_bytes, st, t, c, m.ctx,
+                         m.rng, m.A2, m.sel, m.verd0, m.verd1, m.vcbits, n_vcbits, B, m.words_v, m.cache,
+                         AdvArgs{}));
   if (ev) GRID_CUDA(cudaEventRecord(ev[1], st));
   const int cd_blocks = (s->max_cd + 256 * kFilterPer - 1) / (256 * kFilterPer);
   const int vc_blocks = (s->max_vc + 256 * kFilterPer - 1) / (256 * kFilterPer);
@@ -1968,6 +2034,27 @@ extern "C" int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint3
   lg.dtype = dtype;
   lg.stride = row_stride;
   return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr, lg);
+}
+
+extern "C" int grid_advance_masks(const grid_spec* s, const grid_configs* in, grid_configs* out,
+                                  const int32_t* d_tokens, int32_t n_steps, uint32_t* d_mask, int32_t* d_status,
+                                  void* d_logits, int32_t dtype, int64_t row_stride, void* stream) {
+  if (!s || !in || !out || !d_tokens || !d_mask || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
+    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: bad arguments");
+  if (d_logits && (row_stride < s->t.V || (dtype != GRID_DTYPE_F32 && dtype != GRID_DTYPE_BF16)))
+    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: bad logits arguments");
+  if ((in->c.hs != nullptr) != (out->c.hs != nullptr))
+    return set_error(GRID_E_INVALID_ARG,
+                     "grid_advance_masks: audit must be enabled on both configurations or on neither");
+  const MaskScratch m{out->ctx, out->rng, out->sel, out->verd0, out->verd1, out->A2, out->vcbits,
+                      out->surv, out->vsurv, out->cap, out->vcap, out->words_v};
+  FusedLogits lg;
+  lg.p = d_logits;
+  lg.dtype = dtype;
+  lg.stride = row_stride;
+  const AdvArgs adv{in->c, d_tokens, n_steps, in != out ? 1 : 0};
+  return launch_masks(s, out->c, m, out->B, d_mask, d_status, (cudaStream_t)stream, out->ev[0] ? out->ev : nullptr,
+                      lg, &adv);
 }
 
 // ---------------------------------------------------------------------------

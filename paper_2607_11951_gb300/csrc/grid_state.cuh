@@ -111,6 +111,15 @@ struct FusedLogits {
   long long stride = 0;
 };
 
+// Tokens to feed before the mask step, in its first kernel
+// (grid_advance_masks): from cin into the configurations being masked.
+struct AdvArgs {
+  DevConfigs cin;
+  const int32_t* tokens;
+  int n_steps;
+  int copy;  // 1: cin and the masked configurations are distinct (out of place)
+};
+
 constexpr int kMaskKernels = 4;  // k_row, k_filter, k_walk, k_pack
 
 extern int g_sms;  // SM count of the current device, set by grid_specialize
@@ -186,9 +195,11 @@ namespace grid {
 
 // The four kernels of one mask step (k_row, k_filter, k_walk, k_pack) on
 // `st`; `ev` (5 events or NULL) is recorded before the first kernel and after
-// each.  With lg.p set, k_pack also masks the logits.
+// each.  With lg.p set, k_pack also masks the logits; with adv set, k_row
+// first feeds adv's tokens into c.
 int launch_masks(const grid_spec* s, const DevConfigs& c, const MaskScratch& m, int B, uint32_t* d_mask,
-                 int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg = FusedLogits());
+                 int32_t* d_status, cudaStream_t st, const cudaEvent_t* ev, const FusedLogits& lg = FusedLogits(),
+                 const AdvArgs* adv = nullptr);
 
 // The parser step (k_advance) of B rows from `in` into `out` (copy = 1: out
 // of place) on `st`.

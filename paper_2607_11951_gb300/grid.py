@@ -24,7 +24,7 @@ GRID_DTYPE_F32, GRID_DTYPE_BF16 = 0, 1
 EXPORTED = ["grid_last_error", "grid_compile", "grid_grammar_free", "grid_grammar_info", "grid_grammar_lexicon_trie",
             "grid_load_vocab", "grid_vocab_free", "grid_vocab_info", "grid_specialize",
             "grid_spec_free", "grid_spec_info", "grid_configs_create", "grid_configs_free", "grid_configs_reset",
-            "grid_advance", "grid_masks", "grid_masks_apply", "grid_configs_set_events", "grid_spec_set_work_counters", "grid_masks_static", "grid_forced_span",
+            "grid_advance", "grid_masks", "grid_masks_apply", "grid_advance_masks", "grid_configs_set_events", "grid_spec_set_work_counters", "grid_masks_static", "grid_forced_span",
             "grid_reserve", "grid_cache_create", "grid_cache_free", "grid_cache_clear", "grid_cache_stats",
             "grid_masks_cached", "grid_configs_enable_audit", "grid_audit_append", "grid_audit_seal", "grid_audit_head", "grid_audit_verify",
             "grid_audit_genesis", "grid_blake2b", "grid_fingerprint", "grid_apply_mask", "grid_configs_export"]
@@ -80,6 +80,7 @@ def lib():
         "grid_advance": (I32, [P, P, P, P, I32, P, P]),
         "grid_masks": (I32, [P, P, P, P, P]),
         "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
+        "grid_advance_masks": (I32, [P, P, P, P, I32, P, P, P, I32, I64, P]),
         "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P, P]),
         "grid_reserve": (I32, [P, P, P, P, I32, P, P, I32, P, P]),
         "grid_cache_create": (I32, [P, I32, ctypes.POINTER(P)]),
@@ -263,6 +264,24 @@ def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
     assert mask.is_contiguous() and status.is_contiguous() and logits.stride(1) == 1
     _check(lib().grid_masks_apply(spec, cfg, _ptr(mask), _ptr(status), _ptr(logits), dt, logits.stride(0),
                                   _stream(stream)))
+
+
+def grid_advance_masks(spec, cin, cout, tokens, mask, status, logits=None, stream=None):
+    """grid_advance of ``tokens`` (int32 CUDA tensor [B] or [B, n_steps]) from
+    cin into cout, then the masks of cout (and, with ``logits``, their -inf
+    fill) in one launch sequence; status: the advance's error for a row whose
+    token was refused, else the mask step's."""
+    import torch
+    n = 1 if tokens.dim() == 1 else tokens.shape[1]
+    assert tokens.is_contiguous() and tokens.dtype == torch.int32
+    assert mask.is_contiguous() and status.is_contiguous() and mask.dtype == torch.int32
+    lp, dt, stride = ctypes.c_void_p(None), GRID_DTYPE_F32, 0
+    if logits is not None:
+        dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
+        assert logits.stride(1) == 1
+        lp, stride = _ptr(logits), logits.stride(0)
+    _check(lib().grid_advance_masks(spec, cin, cout, _ptr(tokens), n, _ptr(mask), _ptr(status), lp, dt, stride,
+                                    _stream(stream)))
 
 
 def grid_forced_span(spec, cfg, max_span, mask, span, span_len, status, records=None, stream=None):
