@@ -179,8 +179,12 @@ void grid_spec_free(grid_spec* s);
  * byte by byte at mask time (more stack-dependent events than one record
  * holds), out[3]=such entries over all tables, out[4]=bytes of the tables
  * staged in shared memory (0 = not staged), out[5]=verdict classes (distinct
- * event records of stack-dependent spellings) over all tables, out[6]=1 if CI
- * classes are enabled, out[7]=distinct spellings. */
+ * event records of stack-dependent spellings) over all tables, out[6]=flags:
+ * bit 0 = CI classes enabled (off when the 16-bit class codes cannot hold
+ * every class id: 2 x DFA states x 2^categories >= 65531), bit 1 = a verdict
+ * class's index rides in its id's class code (off when class ids, 5 special
+ * codes and the largest table's verdict classes exceed 65535; then a per-id
+ * index table is read), out[7]=distinct spellings. */
 int grid_spec_info(const grid_spec* s, int64_t out[8]);
 
 /* Create B configurations, all at the start configuration (empty output),

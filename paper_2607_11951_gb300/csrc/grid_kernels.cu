@@ -1224,26 +1224,53 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
         ctw[4 * k + 3] = ct4[k].w;
       }
     }
+    if (t.vc_inline) {
+      // every id takes the same instructions (selects, no branches): its
+      // class selection bit, its verdict-class bit and its walked bit are all
+      // read (indices clamped into range) and the code picks one, so that the
+      // warp's threads never split over the kinds of their ids
+      const uint32_t ok1 = (fl & 1) ? 0xFFFFFFFFu : 0u;  // sigma' exists
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      if (!((todo >> j) & 1u)) continue;
-      const int cx = (killw >> j) & 1u;
-      const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
-      uint32_t bit = 0u;  // codes of verdict classes and walks in a context k_row left out: rejected
-      if (code < code_vc) bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
-      if (code >= code_vc && (!cx || (fl & 1))) {
-        if (code == code_walk) {
-          bit = ((cx ? wv1 : wv0) >> j) & 1u;
-        } else {  // the verdict class: in the code, or looked up
-          const uint32_t v = code >= code_vc0 ? (uint32_t)(code - code_vc0)
-                                              : t.vc_by_id[(size_t)(cx ? 0 : tb) * t.Vp + 32 * wi + j];
-          bit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
+      for (int j = 0; j < 32; ++j) {
+        const uint32_t cx = (killw >> j) & 1u;
+        const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
+        const int ci = min(code, code_vc - 1);
+        const uint32_t cbit = ((cx ? sel1 : sel0)[ci >> 5] >> (ci & 31)) & 1u;
+        const int v = max(code - code_vc0, 0);
+        const uint32_t vbit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
+        const uint32_t wbit = ((cx ? wv1 : wv0) >> j) & 1u;
+        const bool dep = code >= code_vc;  // verdict class or walked: decided per row
+        const bool live = !cx || ok1;      // a context k_row left out rejects its residue ids
+        const uint32_t bit = dep ? (live ? (code == code_walk ? wbit : vbit) : 0u) : cbit;
+        if (CACHE) {
+          if (dep && live)
+            sel_bits |= 1u << j;
+          else
+            ci_bits |= bit << j;
         }
-        if (CACHE) sel_bits |= 1u << j;
-      } else if (CACHE) {
-        ci_bits |= bit << j;
+        m |= (bit & (todo >> j)) << j;
       }
-      m |= bit << j;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        if (!((todo >> j) & 1u)) continue;
+        const int cx = (killw >> j) & 1u;
+        const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
+        uint32_t bit = 0u;  // codes of verdict classes and walks in a context k_row left out: rejected
+        if (code < code_vc) bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
+        if (code >= code_vc && (!cx || (fl & 1))) {
+          if (code == code_walk) {
+            bit = ((cx ? wv1 : wv0) >> j) & 1u;
+          } else {  // the verdict class, looked up
+            const uint32_t v = t.vc_by_id[(size_t)(cx ? 0 : tb) * t.Vp + 32 * wi + j];
+            bit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
+          }
+          if (CACHE) sel_bits |= 1u << j;
+        } else if (CACHE) {
+          ci_bits |= bit << j;
+        }
+        m |= bit << j;
+      }
     }
     if (CACHE && fill >= 0) {
       cache.ci[(size_t)fill * t.W + wi] = ci_bits;
@@ -1873,7 +1900,7 @@ extern "C" int grid_spec_info(const grid_spec* s, int64_t out[8]) {
   out[3] = off[t.n_tbl];
   out[4] = t.blob_bytes;
   out[5] = s->n_vc;
-  out[6] = t.ci_on;
+  out[6] = (t.ci_on ? 1 : 0) | (t.vc_inline ? 2 : 0);
   out[7] = t.NS;
   return GRID_OK;
 }

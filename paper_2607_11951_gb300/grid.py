@@ -221,8 +221,11 @@ def grid_spec_info(spec):
     out = (ctypes.c_int64 * 8)()
     _check(lib().grid_spec_info(spec, out))
     keys = ["ci_tables", "ci_classes", "cd_start", "cd_total", "staged_bytes", "verdict_classes",
-            "ci_on", "spellings"]
-    return dict(zip(keys, list(out)))
+            "flags", "spellings"]
+    d = dict(zip(keys, list(out)))
+    d["ci_on"] = d["flags"] & 1
+    d["vc_in_codes"] = (d["flags"] >> 1) & 1
+    return d
 
 
 def grid_configs_create(spec, B: int):

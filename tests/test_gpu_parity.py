@@ -144,6 +144,36 @@ def test_cold_schema_full_parity():
     _compare_full(wl, run)
 
 
+@pytest.mark.parametrize("n_cat,n_kw,ci_on,in_codes", [(10, 9, 0, 1), (9, 20, 1, 0)])
+def test_manycat_code_space_edges_full_parity(n_cat, n_kw, ci_on, in_codes):
+    """The two edges of the 16-bit class-code space.  Ten categories over 36
+    lexer states: 2 x 36 x 2^10 class ids do not fit, CI classes are off and
+    every spelling of every row is decided by a walk.  Nine categories over
+    62 lexer states: the 63,488 class ids fit but the largest table's verdict
+    classes do not fit beside them, so the packing reads each verdict-class
+    id's index from the per-id table.  Both bit-exact against the oracle on
+    every row, and the fused decoding step equal to the two calls."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl, run = _run("manycat%d" % n_cat, lambda: configs.manycat(n_cat, n_kw))
+    info = run.spec.info()
+    assert info["ci_on"] == ci_on and info["vc_in_codes"] == in_codes, info
+    bits = _compare_full(wl, run)
+    rng = np.random.default_rng(n_cat)
+    tok = np.array([rng.choice(np.flatnonzero(bits[b])) for b in range(run.B)], dtype=np.int32)
+    t = torch.from_numpy(tok).cuda()
+    a, c = G.Configs(run.spec, run.B), G.Configs(run.spec, run.B)
+    st_a = torch.zeros(run.B, dtype=torch.int32, device="cuda")
+    st_c = torch.zeros(run.B, dtype=torch.int32, device="cuda")
+    m_a = torch.zeros_like(run.mask)
+    m_c = torch.zeros_like(run.mask)
+    G.grid_advance(run.spec.h, run.cfg.h, a.h, t, st_a)
+    G.grid_masks(run.spec.h, a.h, m_a, st_a)
+    G.grid_advance_masks(run.spec.h, run.cfg.h, c.h, t, m_c, st_c)
+    torch.cuda.synchronize()
+    assert torch.equal(m_a, m_c) and torch.equal(st_a, st_c)
+
+
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_masked_logits_bit_exact(dtype):
     """grid_apply_mask: rejected -> -inf, accepted values bit-identical (incl.

@@ -242,3 +242,114 @@ def logits(seed: int, B: int, V: int, std: float = 3.0):
     """fp32 logits ~ N(0, std^2), shape [B, V], as a numpy array."""
     rng = np.random.default_rng(seed + 99)
     return (rng.standard_normal((B, V), dtype=np.float32) * np.float32(std)).astype(np.float32)
+
+
+# --------------------------------------------------------------------------
+# many lexicon categories: the edges of the 16-bit class-code space
+# --------------------------------------------------------------------------
+MANYCAT_KEYWORDS = ["ab", "bad", "cab", "dace", "ebb", "deed", "aced", "bead", "cede", "dab", "beaded",
+                    "decade", "acceded", "abed", "ace", "ebbed", "added", "adde", "cabbed", "dabbed"]
+
+
+def manycat_grammar(n_cat: int, n_kw: int) -> str:
+    """A list language whose items are n_cat lexicon categories C0.. sharing the
+    identifier regex /[a-e]+/, qualified pairs C(2k) "." C(2k+1), a call
+    C0 "(" args ")" and keyword-led items; the n_kw keywords are words over the
+    same letters, each adding lexer states.  A CI class id ranges over
+    2 x lexer states x 2^n_cat values, so the number of categories and
+    keywords moves the spec across the edges of the 16-bit code space."""
+    kws = MANYCAT_KEYWORDS[:n_kw]
+    out = ["# %d lexicon categories over one regex, %d keywords (generated)" % (n_cat, n_kw)]
+    out += ['%%token K%d "%s"' % (i, k) for i, k in enumerate(kws)]
+    out += ["%%token C%d /[a-e]+/" % c for c in range(n_cat)]
+    out += ['%token COMMA ","', '%token SEMI ";"', '%token DOT "."', '%token LP "("', '%token RP ")"',
+            "%ignore WS /[ ]+/"]
+    out += ["%%category C%d" % c for c in range(n_cat)]
+    out += ["%start prog", "", "prog -> items SEMI", "items -> items COMMA item", "items -> item"]
+    out += ["item -> C%d" % c for c in range(n_cat)]
+    out += ["item -> C%d DOT C%d" % (c, c + 1) for c in range(0, n_cat - 1, 2)]
+    out += ["item -> C0 LP args RP"]
+    out += ["item -> K%d C%d" % (i, i % n_cat) for i in range(len(kws))]
+    out += ["args -> args COMMA C1", "args -> C2"]
+    return "\n".join(out) + "\n"
+
+
+def manycat(n_cat: int, n_kw: int, seed: int = 1008, B: int = 16, n_multi: int = 6000):
+    """Many-category workload.  Lexicons: 12 words over a-e of length 2-5 per
+    category (keywords excluded), pairwise disjoint, plus 6 words shared by
+    several categories that sentences never use.  Vocabulary: every string of
+    length 1-2 over [abcde,;.() ], then ``n_multi`` distinct random strings of
+    2-4 pieces (letter runs, keywords, punctuation, blanks), EOS last.
+    Prefixes: random sentences (items from single-lexicon words, blanks
+    between lexemes) tokenized greedily and cut at a random byte offset."""
+    rng = np.random.default_rng(seed)
+    letters = "abcde"
+    kws = MANYCAT_KEYWORDS[:n_kw]
+    taken = set(MANYCAT_KEYWORDS)
+
+    def rand_word(lo=2, hi=5):
+        return "".join(letters[int(i)] for i in rng.integers(0, 5, size=int(rng.integers(lo, hi + 1))))
+
+    own = []
+    for _ in range(n_cat):
+        ws = []
+        while len(ws) < 12:
+            w = rand_word()
+            if w not in taken:
+                taken.add(w)
+                ws.append(w)
+        own.append(ws)
+    shared = []
+    while len(shared) < 6:
+        w = rand_word()
+        if w not in taken:
+            taken.add(w)
+            shared.append(w)
+    lexicons = {}
+    for c in range(n_cat):
+        extra = [shared[k] for k in range(6) if (c + k) % 3 == 0]
+        lexicons["C%d" % c] = sorted(own[c] + extra)
+    alpha = "abcde,;.() "
+    toks = [a for a in alpha] + [a + b for a in alpha for b in alpha]
+    seen = set(toks)
+    pieces = [lambda: rand_word(1, 4), lambda: kws[int(rng.integers(len(kws)))] if kws else "a",
+              lambda: ",;.()"[int(rng.integers(5))], lambda: " "]
+    while len(toks) < len(alpha) * (len(alpha) + 1) + n_multi:
+        s = "".join(pieces[int(rng.choice(4, p=[0.45, 0.1, 0.3, 0.15]))]() for _ in range(int(rng.integers(2, 5))))
+        if s not in seen:
+            seen.add(s)
+            toks.append(s)
+    tokens = [t.encode() for t in toks]
+    eos = len(tokens)
+    tokens.append(b"<eos>")
+
+    def item():
+        k = int(rng.integers(4))
+        if k == 0:
+            c = int(rng.integers(n_cat))
+            return [own[c][int(rng.integers(12))]]
+        if k == 1:
+            c = 2 * int(rng.integers(n_cat // 2))
+            return [own[c][int(rng.integers(12))], ".", own[c + 1][int(rng.integers(12))]]
+        if k == 2:
+            args = [own[2][int(rng.integers(12))]] + [own[1][int(rng.integers(12))]
+                                                     for _ in range(int(rng.integers(0, 3)))]
+            return [own[0][int(rng.integers(12))], "("] + sum(([a, ","] for a in args), [])[:-1] + [")"]
+        i = int(rng.integers(len(kws)))
+        return [kws[i], own[i % n_cat][int(rng.integers(12))]]
+
+    tk = GreedyTokenizer(tokens, [eos])
+    prefixes, texts = [], []
+    for _ in range(B):
+        lexemes = []
+        for j in range(int(rng.integers(1, 6))):
+            if j:
+                lexemes.append(",")
+            lexemes += item()
+        lexemes.append(";")
+        s = " ".join(lexemes).encode()
+        cut = int(rng.integers(0, len(s) + 1))
+        texts.append(s[:cut])
+        prefixes.append(tk.encode(s[:cut]))
+    return dict(name="manycat%d" % n_cat, grammar=manycat_grammar(n_cat, n_kw), role=None, lexicons=lexicons,
+                tokens=tokens, eos=eos, specials=[], prefixes=prefixes, texts=texts, B=B, seed=seed)
