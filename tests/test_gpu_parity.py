@@ -144,12 +144,12 @@ def test_cold_schema_full_parity():
     _compare_full(wl, run)
 
 
-@pytest.mark.parametrize("n_cat,n_kw,ci_on,in_codes", [(10, 9, 0, 1), (9, 20, 1, 0)])
+@pytest.mark.parametrize("n_cat,n_kw,ci_on,in_codes", [(10, 9, 0, 1), (9, 21, 1, 0)])
 def test_manycat_code_space_edges_full_parity(n_cat, n_kw, ci_on, in_codes):
     """The two edges of the 16-bit class-code space.  Ten categories over 36
     lexer states: 2 x 36 x 2^10 class ids do not fit, CI classes are off and
     every spelling of every row is decided by a walk.  Nine categories over
-    62 lexer states: the 63,488 class ids fit but the largest table's verdict
+    63 lexer states: the 64,512 class ids fit but the largest table's verdict
     classes do not fit beside them, so the packing reads each verdict-class
     id's index from the per-id table.  Both bit-exact against the oracle on
     every row, and the fused decoding step equal to the two calls."""

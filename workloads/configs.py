@@ -248,7 +248,7 @@ def logits(seed: int, B: int, V: int, std: float = 3.0):
 # many lexicon categories: the edges of the 16-bit class-code space
 # --------------------------------------------------------------------------
 MANYCAT_KEYWORDS = ["ab", "bad", "cab", "dace", "ebb", "deed", "aced", "bead", "cede", "dab", "beaded",
-                    "decade", "acceded", "abed", "ace", "ebbed", "added", "adde", "cabbed", "dabbed"]
+                    "decade", "acceded", "abed", "ace", "ebbed", "added", "adde", "cabbed", "dabbed", "bade"]
 
 
 def manycat_grammar(n_cat: int, n_kw: int) -> str:
@@ -274,7 +274,7 @@ def manycat_grammar(n_cat: int, n_kw: int) -> str:
     return "\n".join(out) + "\n"
 
 
-def manycat(n_cat: int, n_kw: int, seed: int = 1008, B: int = 16, n_multi: int = 6000):
+def manycat(n_cat: int, n_kw: int, seed: int = 1008, B: int = 16, n_multi: int = 10000):
     """Many-category workload.  Lexicons: 12 words over a-e of length 2-5 per
     category (keywords excluded), pairwise disjoint, plus 6 words shared by
     several categories that sentences never use.  Vocabulary: every string of
