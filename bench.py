@@ -633,7 +633,7 @@ def main():
                   "ms_per_step": conc_ms / args.steps,
                   "step": "grid_advance_masks, K steps dealt round-robin to the streams"}
     clocks = clk.stop()
-    work = torch.zeros(4, dtype=torch.int64, device=dev)  # pass E
+    work = torch.zeros(6, dtype=torch.int64, device=dev)  # pass E
     G.grid_spec_set_work_counters(spec.h, work)
     for k in range(N_BATCHES):
         step(args.warmup + k)
@@ -735,7 +735,7 @@ def main():
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     mhz = clocks.get("sm_mhz") or 2070.0
     walk_us = kern_us["k_walk"]
-    units = sum(work)
+    units = sum(work[:4])
     peak_units = sms * LANES * mhz * 1e6 / 1e9
     roof_walk = {"kernel": "k_walk (grid_advance_masks)", "bound": "alu",
                  "unit": "G work units/s (lexer steps + ACTION + GOTO lookups + verdict-class events)",
@@ -744,6 +744,10 @@ def main():
                  (sms, LANES, mhz),
                  "work_per_launch": {"lexer_steps": work[0], "action_lookups": work[1], "goto_lookups": work[2],
                                      "verdict_class_events": work[3]},
+                 "evaluated_per_launch": {"verdict_class_records": work[4], "byte_walked_spellings": work[5],
+                                          "verdict_class_records_per_row": work[4] / B,
+                                          "paper_class_verdicts_per_step": "143-150 (its own SQL bench and "
+                                                                           "tokenizer, Sec. 4.2 / Sec. 8.2)"},
                  "traffic": None}
     roof_walk["frac"] = roof_walk["achieved"] / peak_units
     wc = _counters("k_walk")

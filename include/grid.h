@@ -298,13 +298,15 @@ int grid_cache_stats(const grid_cache* c, int64_t out[4]);
 int grid_masks_cached(const grid_spec* s, const grid_configs* c, grid_cache* cache, uint32_t* d_mask,
                       int32_t* d_status, void* d_logits, int32_t dtype, int64_t row_stride, void* stream);
 
-/* Measurement hook: with d_counters (device memory, 4 x u64, zeroed by the
+/* Measurement hook: with d_counters (device memory, 6 x u64, zeroed by the
  * caller) set, every later mask step on `s` adds to it the work of its walk
  * kernel in the units of the walk's algorithmic cost: [0] lexer steps (trie
  * node visits of byte walks), [1] ACTION lookups (reduce-chain steps, for one
  * terminal or a set of terminals at once), [2] GOTO lookups, [3] verdict-class
- * events evaluated.  Counting slows that kernel down (one atomic per unit);
- * time steps without it.  NULL stops the counting. */
+ * events evaluated; and what it evaluated: [4] verdict-class records (one per
+ * row, context and surviving class: the verdict classes of Sec. 4.2 decided by
+ * the step), [5] spellings walked byte by byte.  Counting slows that kernel
+ * down; time steps without it.  NULL stops the counting. */
 int grid_spec_set_work_counters(grid_spec* s, unsigned long long* d_counters);
 
 /* grid_masks without any allocation.  The paper has no counterpart: this is

@@ -928,7 +928,8 @@ __device__ __forceinline__ int4 row_queue(const Tables& t, const RowCtx& x) {
 // walk_bytes, one spelling per lane.
 // With COUNT, each lane also counts its work (lexer steps, ACTION and GOTO
 // lookups, verdict-class events) in registers and adds the totals to
-// work[0..3] when it is done; the plain instance has no counting code.
+// work[0..3] when it is done (and the records and spellings it evaluated to
+// work[4..5]); the plain instance has no counting code.
 template <bool COUNT>
 __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* __restrict__ ctx,
                                                              const RowRanges* __restrict__ rng, const uint16_t* stacks,
@@ -952,7 +953,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   const int gw = blockIdx.x * kWalkWarps + warp;
   const int mc = max_chain_of(t);
   const LArr lo{s_lane[warp] + lane, 32}, ls{s_lane[warp] + kLaneOvl * 32 + lane, 32};
-  uint32_t cnt[4] = {0u, 0u, 0u, 0u};
+  uint32_t cnt[6] = {0u, 0u, 0u, 0u, 0u, 0u};  // the walk's work units, then records and spellings evaluated
   uint32_t* const ctr = COUNT ? cnt : nullptr;
   // queue length and segment ends of every row
   const bool cached = B <= kWalkRowsCached;
@@ -1057,6 +1058,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
       const int k = item * 32 + lane;
       int res = 0, v = 0;
       if (k < r.nvs[cxi]) {
+        if (COUNT) ++cnt[4];
         v = vsurv[((size_t)row * 2 + cxi) * vcap + k];
         Walker w;
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row, ctr);
@@ -1106,6 +1108,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
         go = sp_i < p1;
       }
       if (go) {
+        if (COUNT) ++cnt[5];
         const Spell sp = load_spell(ts, sp_i);
         Walker w;
         walker_init(w, lo, ls, kLaneOvl, base, ckeep, s_ovl[warp], cm, cq, clx, cpc, cwc, Ac, A2row, ctr);
@@ -1118,7 +1121,7 @@ __global__ void __launch_bounds__(kWalkWarps * 32, 2) k_walk(Tables t, RowCtx* _
   }
   if (lane == 0 && bound_row >= 0) atomicCAS(&ctx[bound_row].status, GRID_ST_OK, GRID_ST_BOUND);
   if (COUNT)
-    for (int k = 0; k < 4; ++k)
+    for (int k = 0; k < 6; ++k)
       if (cnt[k]) atomicAdd(&work[k], (unsigned long long)cnt[k]);
 }
 

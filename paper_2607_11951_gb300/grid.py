@@ -410,7 +410,9 @@ def grid_configs_set_events(cfg, events):
 
 
 def grid_spec_set_work_counters(spec, counters):
-    """counters: int64 CUDA tensor [4] (zeroed by the caller), or None to stop."""
+    """counters: int64 CUDA tensor [6] (zeroed by the caller), or None to stop."""
+    if counters is not None:
+        assert counters.is_cuda and counters.numel() >= 6 and counters.element_size() == 8
     _check(lib().grid_spec_set_work_counters(spec, ctypes.c_void_p(None) if counters is None else _ptr(counters)))
 
 

@@ -157,3 +157,27 @@ def test_fused_step_with_audit_keeps_node_hashes():
     # the records carry the rolling hash of each row's stack: equal records,
     # equal node hashes
     assert torch.equal(rec_a, rec_b)
+
+
+def test_fused_step_refuses_bad_arguments():
+    """Mismatched batch sizes, a row stride below V and an unknown logits
+    type are refused with an error before anything is enqueued."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl = configs.tiny_expr(B=4)
+    run = GpuRun(wl)
+    run.build_configs()
+    other = G.Configs(run.spec, 5)
+    tok = torch.zeros(4, dtype=torch.int32, device="cuda")
+    st = torch.zeros(4, dtype=torch.int32, device="cuda")
+    with pytest.raises(G.GridError):
+        G.grid_advance_masks(run.spec.h, run.cfg.h, other.h, tok, run.mask, st)
+    lib = G.lib()
+    logits = torch.zeros((4, run.V), device="cuda")
+    out = G.Configs(run.spec, 4)
+    rc = lib.grid_advance_masks(run.spec.h, run.cfg.h, out.h, G._ptr(tok), 1, G._ptr(run.mask), G._ptr(st),
+                                G._ptr(logits), G.GRID_DTYPE_F32, run.V - 1, None)
+    assert rc == -1  # GRID_E_INVALID_ARG
+    rc = lib.grid_advance_masks(run.spec.h, run.cfg.h, out.h, G._ptr(tok), 1, G._ptr(run.mask), G._ptr(st),
+                                G._ptr(logits), 7, run.V, None)
+    assert rc == -1  # GRID_E_INVALID_ARG

@@ -315,3 +315,27 @@ def test_ragged_vocab_tail_and_single_row():
     run = GpuRun(wl)
     assert (run.build_configs() == 0).all()
     _compare_full(wl, run)
+
+
+def test_walk_work_counters():
+    """The measurement hook counts without changing the masks: with counters
+    on, the masks equal those without; lexer steps, ACTION lookups and the
+    records and spellings evaluated are all counted on the headline batch, and
+    a step evaluates no more records per row and context than the tables
+    hold."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl, run = _run("headline", configs.sql_select_only)
+    words0, st0 = run.masks()
+    work = torch.zeros(6, dtype=torch.int64, device="cuda")
+    G.grid_spec_set_work_counters(run.spec.h, work)
+    words1, st1 = run.masks()
+    G.grid_spec_set_work_counters(run.spec.h, None)
+    torch.cuda.synchronize()
+    assert (words1 == words0).all() and (st1 == st0).all()
+    w = work.cpu().tolist()
+    assert all(x > 0 for x in w), w
+    assert w[4] <= 2 * run.B * run.spec.info()["verdict_classes"]
+    words2, _ = run.masks()  # counting off again: the counters stay as they were
+    torch.cuda.synchronize()
+    assert work.cpu().tolist() == w and (words2 == words0).all()
