@@ -1177,18 +1177,18 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
     s_fill = CACHE ? rc.cfill : -1;
     s_q = rc.q;
   }
-  __syncthreads();
-  const int fl = s_fl, tb = s_tb, hit = CACHE ? s_hit : -1, fill = CACHE ? s_fill : -1;
-  // a context that k_row did not select for (a completed row, sigma' without
-  // a forced emission, sigma without a table) reads zeros
+  // the row's class selections and verdict-class bits, staged alongside its
+  // context (a selection k_row did not write is masked off at use)
   {
-    const bool v0 = t.ci_on && !(fl & 4) && tb >= 0, v1 = t.ci_on && !(fl & 4) && (fl & 1);
-    for (int i = threadIdx.x; i < 2 * nw; i += kPackWords)
-      s_dyn[i] = (i < nw ? v0 : v1) ? sel[(size_t)b * 2 * nw + i] : 0u;
+    for (int i = threadIdx.x; i < 2 * nw; i += kPackWords) s_dyn[i] = sel[(size_t)b * 2 * nw + i];
     const uint32_t* vb = vcbits + (size_t)b * 2 * vcw;
     for (int i = threadIdx.x; i < 2 * vcw; i += kPackWords) s_dyn[2 * nw + i] = vb[i];
   }
   __syncthreads();
+  const int fl = s_fl, tb = s_tb, hit = CACHE ? s_hit : -1, fill = CACHE ? s_fill : -1;
+  // a context that k_row did not select for (a completed row, sigma' without
+  // a forced emission, sigma without a table) selects no class
+  const uint32_t v0 = (t.ci_on && !(fl & 4) && tb >= 0) ? 1u : 0u, v1 = (t.ci_on && !(fl & 4) && (fl & 1)) ? 1u : 0u;
   const uint32_t* sel0 = s_dyn;
   const uint32_t* sel1 = s_dyn + nw;
   const uint32_t* vcb0 = s_dyn + 2 * nw;
@@ -1238,7 +1238,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
         const uint32_t cx = (killw >> j) & 1u;
         const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
         const int ci = min(code, code_vc - 1);
-        const uint32_t cbit = ((cx ? sel1 : sel0)[ci >> 5] >> (ci & 31)) & 1u;
+        const uint32_t cbit = ((cx ? sel1 : sel0)[ci >> 5] >> (ci & 31)) & (cx ? v1 : v0);
         const int v = max(code - code_vc0, 0);
         const uint32_t vbit = ((cx ? vcb1 : vcb0)[v >> 5] >> (v & 31)) & 1u;
         const uint32_t wbit = ((cx ? wv1 : wv0) >> j) & 1u;
@@ -1260,7 +1260,7 @@ __global__ void __launch_bounds__(kPackWords) k_pack(Tables t, RowCtx* __restric
         const int cx = (killw >> j) & 1u;
         const int code = (int)(((cx ? c0w[j >> 1] : ctw[j >> 1]) >> ((j & 1) * 16)) & 0xFFFFu);
         uint32_t bit = 0u;  // codes of verdict classes and walks in a context k_row left out: rejected
-        if (code < code_vc) bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & 1u;
+        if (code < code_vc) bit = ((cx ? sel1 : sel0)[code >> 5] >> (code & 31)) & (cx ? v1 : v0);
         if (code >= code_vc && (!cx || (fl & 1))) {
           if (code == code_walk) {
             bit = ((cx ? wv1 : wv0) >> j) & 1u;
