@@ -578,8 +578,7 @@ def main():
 
     def warm_step(k):
         i = k % N_BATCHES
-        G.grid_advance(spec.h, cfgs[i].h, scratch.h, toks[i], status, stream)
-        G.grid_masks_cached(spec, scratch.h, cache, mask, status, logits[i], stream)
+        G.grid_advance_masks(spec.h, cfgs[i].h, scratch.h, toks[i], mask, status, logits[i], stream, cache=cache)
 
     for k in range(N_BATCHES + args.warmup):
         warm_step(k)
@@ -596,7 +595,7 @@ def main():
     cache_line = {"ms_per_step": warm_ms, "masks_per_s": B / (warm_ms * 1e-3),
                   "hit_rate": (c1["hits"] - c0["hits"]) / max(1, c1["lookups"] - c0["lookups"]),
                   "entries_ready": c1["ready"],
-                  "step": "grid_advance + grid_masks_cached (fused fp32 fill), cache warmed by one pass "
+                  "step": "grid_advance_masks through the cache (fused fp32 fill), cache warmed by one pass "
                           "over the 16 batches"}
     # pass G: independent batch-32 steps on 4 streams at once (each stream
     # with its own scratch, mask and status; no two streams on one batch at a

@@ -97,6 +97,7 @@ typedef struct grid_grammar grid_grammar;
 typedef struct grid_vocab grid_vocab;
 typedef struct grid_spec grid_spec;
 typedef struct grid_configs grid_configs;
+typedef struct grid_cache grid_cache;
 
 /* One L3 lexicon: the allowed words W_c of category terminal `category`
  * (Sec. 2, L3).  Word i is words[offsets[i] .. offsets[i+1]); host memory,
@@ -235,7 +236,8 @@ int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask
  * grid_advance of d_tokens (n_steps per row) from `in` into `out`, then
  * grid_masks of `out` -- or grid_masks_apply when d_logits is not NULL
  * (dtype and row_stride as there; d_logits NULL: no fill, dtype and
- * row_stride unused).  The advance runs inside the mask step's first kernel,
+ * row_stride unused); with `cache` (a cache of `s`, or NULL) through the
+ * mask cache as grid_masks_cached.  The advance runs inside the mask step's first kernel,
  * one row per block, so that a row's mask preparation starts as soon as its
  * own token is fed.  The configurations and masks are those of grid_advance
  * followed by grid_masks(_apply); d_status[b] is the advance's status when
@@ -245,9 +247,9 @@ int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint32_t* d_mask
  * `out` follow grid_advance's rules (same B and D, audit on both or neither;
  * in == out advances in place); the scratch and overlap rule of grid_masks
  * apply to `out`.  Enqueue only. */
-int grid_advance_masks(const grid_spec* s, const grid_configs* in, grid_configs* out, const int32_t* d_tokens,
-                       int32_t n_steps, uint32_t* d_mask, int32_t* d_status, void* d_logits, int32_t dtype,
-                       int64_t row_stride, void* stream);
+int grid_advance_masks(const grid_spec* s, const grid_configs* in, grid_configs* out, grid_cache* cache,
+                       const int32_t* d_tokens, int32_t n_steps, uint32_t* d_mask, int32_t* d_status,
+                       void* d_logits, int32_t dtype, int64_t row_stride, void* stream);
 
 /* Measurement hook: with n_events == 5, every later grid_masks on `c` records
  * events[0..4] (cudaEvent_t, created by the caller) on its stream before its
@@ -275,7 +277,6 @@ int grid_configs_set_events(grid_configs* c, void* const* events, int32_t n_even
  * slot is the key's hash modulo n_entries, no eviction) and read from the
  * next step on; the content is a function of the key, so concurrent fills of
  * one key write identical words. */
-typedef struct grid_cache grid_cache;
 
 /* Allocate a cache of n_entries (a power of two, <= 2^20) entries of
  * 64 + 8 * ceil(V/32) bytes for spec `s` (which must outlive it).

@@ -2066,27 +2066,6 @@ extern "C" int grid_masks_apply(const grid_spec* s, const grid_configs* c, uint3
   return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr, lg);
 }
 
-extern "C" int grid_advance_masks(const grid_spec* s, const grid_configs* in, grid_configs* out,
-                                  const int32_t* d_tokens, int32_t n_steps, uint32_t* d_mask, int32_t* d_status,
-                                  void* d_logits, int32_t dtype, int64_t row_stride, void* stream) {
-  if (!s || !in || !out || !d_tokens || !d_mask || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
-    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: bad arguments");
-  if (d_logits && (row_stride < s->t.V || (dtype != GRID_DTYPE_F32 && dtype != GRID_DTYPE_BF16)))
-    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: bad logits arguments");
-  if ((in->c.hs != nullptr) != (out->c.hs != nullptr))
-    return set_error(GRID_E_INVALID_ARG,
-                     "grid_advance_masks: audit must be enabled on both configurations or on neither");
-  const MaskScratch m{out->ctx, out->rng, out->sel, out->verd0, out->verd1, out->A2, out->vcbits,
-                      out->surv, out->vsurv, out->cap, out->vcap, out->words_v};
-  FusedLogits lg;
-  lg.p = d_logits;
-  lg.dtype = dtype;
-  lg.stride = row_stride;
-  const AdvArgs adv{in->c, d_tokens, n_steps, in != out ? 1 : 0};
-  return launch_masks(s, out->c, m, out->B, d_mask, d_status, (cudaStream_t)stream, out->ev[0] ? out->ev : nullptr,
-                      lg, &adv);
-}
-
 // ---------------------------------------------------------------------------
 // Configuration-keyed mask cache (Sec. 4.3, Def. T1 key, Prop. OBL-KEY1).
 struct grid_cache {
@@ -2165,6 +2144,30 @@ extern "C" int grid_masks_cached(const grid_spec* s, const grid_configs* c, grid
   lg.dtype = dtype;
   lg.stride = row_stride;
   return launch_masks(s, c->c, m, c->B, d_mask, d_status, (cudaStream_t)stream, c->ev[0] ? c->ev : nullptr, lg);
+}
+
+extern "C" int grid_advance_masks(const grid_spec* s, const grid_configs* in, grid_configs* out, grid_cache* cache,
+                                  const int32_t* d_tokens, int32_t n_steps, uint32_t* d_mask, int32_t* d_status,
+                                  void* d_logits, int32_t dtype, int64_t row_stride, void* stream) {
+  if (!s || !in || !out || !d_tokens || !d_mask || !d_status || n_steps < 0 || in->B != out->B || in->D != out->D)
+    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: bad arguments");
+  if (cache && cache->s != s)
+    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: the cache must belong to the spec");
+  if (d_logits && (row_stride < s->t.V || (dtype != GRID_DTYPE_F32 && dtype != GRID_DTYPE_BF16)))
+    return set_error(GRID_E_INVALID_ARG, "grid_advance_masks: bad logits arguments");
+  if ((in->c.hs != nullptr) != (out->c.hs != nullptr))
+    return set_error(GRID_E_INVALID_ARG,
+                     "grid_advance_masks: audit must be enabled on both configurations or on neither");
+  MaskScratch m{out->ctx, out->rng, out->sel, out->verd0, out->verd1, out->A2, out->vcbits,
+                out->surv, out->vsurv, out->cap, out->vcap, out->words_v};
+  if (cache) m.cache = cache->d;
+  FusedLogits lg;
+  lg.p = d_logits;
+  lg.dtype = dtype;
+  lg.stride = row_stride;
+  const AdvArgs adv{in->c, d_tokens, n_steps, in != out ? 1 : 0};
+  return launch_masks(s, out->c, m, out->B, d_mask, d_status, (cudaStream_t)stream, out->ev[0] ? out->ev : nullptr,
+                      lg, &adv);
 }
 
 extern "C" int grid_spec_set_work_counters(grid_spec* s, unsigned long long* d_counters) {

@@ -80,7 +80,7 @@ def lib():
         "grid_advance": (I32, [P, P, P, P, I32, P, P]),
         "grid_masks": (I32, [P, P, P, P, P]),
         "grid_masks_apply": (I32, [P, P, P, P, P, I32, I64, P]),
-        "grid_advance_masks": (I32, [P, P, P, P, I32, P, P, P, I32, I64, P]),
+        "grid_advance_masks": (I32, [P, P, P, P, P, I32, P, P, P, I32, I64, P]),
         "grid_forced_span": (I32, [P, P, I32, P, P, P, P, P, P]),
         "grid_reserve": (I32, [P, P, P, P, I32, P, P, I32, P, P]),
         "grid_cache_create": (I32, [P, I32, ctypes.POINTER(P)]),
@@ -269,11 +269,12 @@ def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
                                   _stream(stream)))
 
 
-def grid_advance_masks(spec, cin, cout, tokens, mask, status, logits=None, stream=None):
+def grid_advance_masks(spec, cin, cout, tokens, mask, status, logits=None, stream=None, cache=None):
     """grid_advance of ``tokens`` (int32 CUDA tensor [B] or [B, n_steps]) from
     cin into cout, then the masks of cout (and, with ``logits``, their -inf
-    fill) in one launch sequence; status: the advance's error for a row whose
-    token was refused, else the mask step's."""
+    fill) in one launch sequence, through ``cache`` (a Cache) if given;
+    status: the advance's error for a row whose token was refused, else the
+    mask step's."""
     import torch
     n = 1 if tokens.dim() == 1 else tokens.shape[1]
     assert tokens.is_contiguous() and tokens.dtype == torch.int32
@@ -283,7 +284,8 @@ def grid_advance_masks(spec, cin, cout, tokens, mask, status, logits=None, strea
         dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
         assert logits.stride(1) == 1
         lp, stride = _ptr(logits), logits.stride(0)
-    _check(lib().grid_advance_masks(spec, cin, cout, _ptr(tokens), n, _ptr(mask), _ptr(status), lp, dt, stride,
+    ch = ctypes.c_void_p(None) if cache is None else getattr(cache, "h", cache)
+    _check(lib().grid_advance_masks(spec, cin, cout, ch, _ptr(tokens), n, _ptr(mask), _ptr(status), lp, dt, stride,
                                     _stream(stream)))
 
 

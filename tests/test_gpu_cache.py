@@ -66,3 +66,37 @@ def test_cache_fused_logits_and_clear():
             cache.clear()
             torch.cuda.synchronize()
             assert cache.stats() == {"lookups": 0, "hits": 0, "fills": 0, "ready": 0}
+
+
+@pytest.mark.parametrize("name", ["sql_admin", "sql_select_only"])
+def test_cache_on_equals_cache_off_in_the_fused_step(name):
+    """The fused decoding step (grid_advance_masks) through a cache equals it
+    without one, over replays of several steps in place: masks, statuses,
+    configurations and the fp32 fill bit for bit, with hits from the second
+    step on."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    wl = getattr(configs, name)()
+    run_a, run_b = GpuRun(wl), GpuRun(wl)
+    assert (run_a.build_configs() == 0).all() and (run_b.build_configs() == 0).all()
+    cache = G.Cache(run_b.spec, 1024)
+    B, V = run_a.B, run_a.V
+    rng = np.random.default_rng(23)
+    words, _ = run_a.masks()
+    for step in range(4):
+        bits = unpack(words, V)
+        tok = np.array([rng.choice(np.flatnonzero(bits[b])) if bits[b].any() else -1 for b in range(B)], np.int32)
+        t = torch.from_numpy(tok).cuda()
+        lg = torch.from_numpy(configs.logits(40 + step, B, V)).cuda()
+        la, lb = lg.clone(), lg.clone()
+        st_a = torch.zeros(B, dtype=torch.int32, device="cuda")
+        st_b = torch.zeros(B, dtype=torch.int32, device="cuda")
+        G.grid_advance_masks(run_a.spec.h, run_a.cfg.h, run_a.cfg.h, t, run_a.mask, st_a, la)
+        G.grid_advance_masks(run_b.spec.h, run_b.cfg.h, run_b.cfg.h, t, run_b.mask, st_b, lb, cache=cache)
+        torch.cuda.synchronize()
+        assert torch.equal(run_a.mask, run_b.mask) and torch.equal(st_a, st_b), (name, step)
+        assert torch.equal(la.view(torch.int32), lb.view(torch.int32)), (name, step)
+        assert [G.grid_configs_export(run_a.cfg.h, b) for b in range(0, B, 5)] == \
+               [G.grid_configs_export(run_b.cfg.h, b) for b in range(0, B, 5)]
+        words = run_a.mask.cpu().numpy().view(np.uint32)
+    assert cache.stats()["hits"] > 0

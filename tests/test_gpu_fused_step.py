@@ -175,9 +175,13 @@ def test_fused_step_refuses_bad_arguments():
     lib = G.lib()
     logits = torch.zeros((4, run.V), device="cuda")
     out = G.Configs(run.spec, 4)
-    rc = lib.grid_advance_masks(run.spec.h, run.cfg.h, out.h, G._ptr(tok), 1, G._ptr(run.mask), G._ptr(st),
+    rc = lib.grid_advance_masks(run.spec.h, run.cfg.h, out.h, None, G._ptr(tok), 1, G._ptr(run.mask), G._ptr(st),
                                 G._ptr(logits), G.GRID_DTYPE_F32, run.V - 1, None)
     assert rc == -1  # GRID_E_INVALID_ARG
-    rc = lib.grid_advance_masks(run.spec.h, run.cfg.h, out.h, G._ptr(tok), 1, G._ptr(run.mask), G._ptr(st),
+    rc = lib.grid_advance_masks(run.spec.h, run.cfg.h, out.h, None, G._ptr(tok), 1, G._ptr(run.mask), G._ptr(st),
                                 G._ptr(logits), 7, run.V, None)
     assert rc == -1  # GRID_E_INVALID_ARG
+    other_spec = G.Spec(run.grammar, run.vocab)  # a cache of another spec
+    cache = G.Cache(other_spec, 64)
+    with pytest.raises(G.GridError):
+        G.grid_advance_masks(run.spec.h, run.cfg.h, out.h, tok, run.mask, st, cache=cache)
