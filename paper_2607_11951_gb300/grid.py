@@ -277,12 +277,19 @@ def grid_advance_masks(spec, cin, cout, tokens, mask, status, logits=None, strea
     mask step's."""
     import torch
     n = 1 if tokens.dim() == 1 else tokens.shape[1]
-    assert tokens.is_contiguous() and tokens.dtype == torch.int32
+    assert tokens.is_contiguous() and tokens.dtype == torch.int32 and tokens.is_cuda
     assert mask.is_contiguous() and status.is_contiguous() and mask.dtype == torch.int32
+    assert status.dtype == torch.int32 and mask.is_cuda and status.is_cuda and mask.dim() == 2
+    B, W = getattr(cout, "B", None), getattr(spec, "W", None)
+    assert B is None or (mask.shape[0] == B and tuple(status.shape) == (B,) and tokens.shape[0] == B), \
+        "tokens [B] or [B, n], mask [B, W] and status [B] expected"
+    assert W is None or mask.shape[1] == W, "mask [B, ceil(V/32)] expected"
+    spec, cin, cout = getattr(spec, "h", spec), getattr(cin, "h", cin), getattr(cout, "h", cout)
     lp, dt, stride = ctypes.c_void_p(None), GRID_DTYPE_F32, 0
     if logits is not None:
         dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
-        assert logits.stride(1) == 1
+        assert logits.is_cuda and logits.dim() == 2 and logits.stride(1) == 1
+        assert B is None or logits.shape[0] == B, "logits [B, >=V] expected"
         lp, stride = _ptr(logits), logits.stride(0)
     ch = ctypes.c_void_p(None) if cache is None else getattr(cache, "h", cache)
     _check(lib().grid_advance_masks(spec, cin, cout, ch, _ptr(tokens), n, _ptr(mask), _ptr(status), lp, dt, stride,
