@@ -64,3 +64,16 @@ def test_random_grammar_full_parity_and_step(seed, role):
     w2 = dict(wl)
     w2["prefixes"] = [list(wl["prefixes"][b]) + [int(tok[b])] for b in range(run.B)]
     _compare(w2, b2, rows, oracle_masks(w2, rows))
+
+
+@pytest.mark.parametrize("seed", range(24, 72))
+def test_random_grammar_sweep_full_parity(seed):
+    """Forty-eight more random grammars, smaller (16 rows, V = 1,500), masks
+    only; odd seeds with the role-tagged statements dropped."""
+    wl = rand_grammar_workload(seed, B=16, V=1500, role=[] if seed % 2 else None)
+    run = GpuRun(wl)
+    st = run.build_configs()
+    assert (st == 0).all(), ("grid_advance status", st)
+    words, status = run.masks()
+    assert (status == 0).all(), ("grid_masks status", status)
+    _compare(wl, unpack(words, run.V), range(run.B), oracle_masks(wl, procs=1))
