@@ -173,6 +173,36 @@ class BruteGrammar:
             pos += best
         return self.accepts_terms(sets)
 
+    def lexes_viably(self, s: bytes) -> bool:
+        """The lexing of in_L succeeds to the end of s with every picked
+        terminal scannable: the terminal string read so far is a viable
+        prefix.  For an s that ends in a blank this is s in Prefix(L) on any
+        grammar where each viable terminal string has a rendering that lexes
+        back to it."""
+        sets = self.earley_start()
+        pos, n = 0, len(s)
+        while pos < n:
+            best = 0
+            for k in range(1, n - pos + 1):
+                if any(r.fullmatch(s[pos:pos + k]) for r in self.rx):
+                    best = k
+            if best == 0:
+                return False
+            lex = s[pos:pos + best]
+            scan_ok = self.scannable(sets)
+            picked = None
+            for t in range(len(self.names)):
+                if self.rx[t].fullmatch(lex) and not (t in self.cats and lex not in self.W[t]) \
+                        and (t in self.ignored or t in scan_ok):
+                    picked = t
+                    break
+            if picked is None:
+                return False
+            if picked not in self.ignored:
+                self.scan(sets, picked)
+            pos += best
+        return True
+
     def in_prefix_L(self, s: bytes, completions) -> bool:
         return any(self.in_L(s + u) for u in completions)
 
