@@ -77,3 +77,32 @@ def test_random_grammar_sweep_full_parity(seed):
     words, status = run.masks()
     assert (status == 0).all(), ("grid_masks status", status)
     _compare(wl, unpack(words, run.V), range(run.B), oracle_masks(wl, procs=1))
+
+
+@pytest.mark.parametrize("seed", [1, 6, 14])
+def test_random_grammar_fused_fill_and_static_path(seed):
+    """On random grammars: the masks with the fused -inf fill (fp32 and bf16)
+    equal the masks followed by grid_apply_mask, bit for bit, and the
+    allocation-free entry point gives grid_masks' masks and statuses."""
+    import torch
+    from paper_2607_11951_gb300 import grid as G
+    from workloads import configs
+    from tests.test_zz_no_alloc import _masks_static, _state_arrays
+    wl = rand_grammar_workload(seed, B=32, V=3000)
+    run = GpuRun(wl)
+    assert (run.build_configs() == 0).all()
+    words, status = run.masks()
+    for dt in (torch.float32, torch.bfloat16):
+        base = torch.from_numpy(configs.logits(seed, run.B, run.V)).to(dt).cuda()
+        la, lb = base.clone(), base.clone()
+        mask = torch.zeros_like(run.mask)
+        st = torch.zeros_like(run.status)
+        G.grid_masks_apply(run.spec.h, run.cfg.h, mask, st, la)
+        G.grid_apply_mask(run.mask, lb)
+        torch.cuda.synchronize()
+        assert (mask.cpu().numpy().view(np.uint32) == words).all() and (st.cpu().numpy() == status).all()
+        iv = torch.int32 if dt == torch.float32 else torch.int16
+        assert torch.equal(la.view(iv), lb.view(iv)), dt
+    w2, s2 = _masks_static(run, torch, _state_arrays(run, torch))
+    np.testing.assert_array_equal(w2, words)
+    np.testing.assert_array_equal(s2, status)

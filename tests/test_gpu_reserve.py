@@ -8,6 +8,7 @@ import pytest
 
 from tests.harness import GpuRun
 from workloads import configs
+from workloads.randgram import rand_grammar_workload
 
 pytestmark = pytest.mark.gpu
 
@@ -20,6 +21,9 @@ def _cases():
         "sql_shared": lambda: configs.sql_shared(B=8),
         "sweep_deep": lambda: configs.sql_sweep_cell(100, 32),
         "forced_sql": configs.forced_sql,
+        # random statement grammars: keyword-led statements, lists, optional
+        # clauses, calls, nested blocks, identifier categories
+        **{"rand_%d" % k: (lambda k=k: rand_grammar_workload(k, B=16, V=1500)) for k in (0, 1, 6, 8, 14)},
     }
 
 
