@@ -53,7 +53,7 @@ class RandGrammar:
         ops = list(rng.permutation(list(OPS)))
         n_lev = int(rng.integers(1, 4))
         n_stmt = int(rng.integers(2, 5))
-        # expression ladder: e0 -> e0 op e1 | e1 ... e{L} -> u ; u -> op u | p
+        # expression ladder: e{i} -> e{i} op e{i+1} | e{i+1} for i < L; e{L} -> op e{L} | p (unary operators)
         lev_ops = [[ops.pop() for _ in range(int(rng.integers(1, 3)))] for _ in range(n_lev)]
         for i, os_ in enumerate(lev_ops):
             for o in os_:
