@@ -206,3 +206,36 @@ def test_manycat_grammars_straddle_the_class_code_space():
         for p in wl["prefixes"]:
             cfg = og.config_from_ids(p, wl["tokens"], wl["eos"], wl["specials"])
             assert cfg is not None and og.live_end(cfg)
+
+
+_VOID_FREE = ("grid_grammar_free", "grid_vocab_free", "grid_spec_free", "grid_configs_free", "grid_cache_free")
+
+
+@pytest.mark.parametrize("name", [n for n in G.EXPORTED if n != "grid_last_error" and n not in _VOID_FREE])
+def test_entry_point_refuses_null_handles_without_a_device(name):
+    """Every call with NULL handles and pointers returns GRID_E_INVALID_ARG
+    and names itself in the thread's error message, before any CUDA call (no
+    GPU in this process); the free functions accept NULL."""
+    L = G.lib()
+    f = getattr(L, name)
+    ints = (ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t, ctypes.c_uint32)
+    args = [1 if a in ints else None for a in f.argtypes]
+    assert f(*args) == -1, name
+    buf = ctypes.create_string_buffer(256)
+    L.grid_last_error(buf, 256)
+    assert buf.value.decode().startswith(name + ":"), buf.value
+    for free in _VOID_FREE:
+        getattr(L, free)(None)
+
+
+def test_apply_mask_argument_checks_on_the_host():
+    """grid_apply_mask refuses a bad row count, vocabulary size, row stride or
+    logits type, and more than 65,535 rows, before it launches anything (the
+    pointers here are never dereferenced)."""
+    L = G.lib()
+    m, lg = ctypes.c_void_p(256), ctypes.c_void_p(512)
+    F32, BF16 = G.GRID_DTYPE_F32, G.GRID_DTYPE_BF16
+    for B, V, stride, dt in [(0, 10, 10, F32), (2, 0, 10, F32), (2, 10, 9, BF16), (2, 10, 10, 7), (-1, 10, 10, F32)]:
+        assert L.grid_apply_mask(m, lg, dt, B, V, stride, None) == -1, (B, V, stride, dt)
+    assert L.grid_apply_mask(m, lg, F32, 65536, 10, 10, None) == -8  # GRID_E_TOO_LARGE
+    assert L.grid_apply_mask(None, lg, F32, 1, 10, 10, None) == -1
