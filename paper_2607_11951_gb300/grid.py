@@ -239,10 +239,16 @@ def grid_configs_reset(spec, cfg, stream=None):
 
 
 def grid_advance(spec, cin, cout, tokens, status, stream=None):
-    """tokens: int32 CUDA tensor [B] or [B, n_steps]; status: int32 CUDA tensor [B]."""
+    """tokens: int32 CUDA tensor [B] or [B, n_steps]; status: int32 CUDA tensor [B].
+    ``cin`` / ``cout`` are handles, or Configs objects (then B is checked)."""
+    import torch
     n = 1 if tokens.dim() == 1 else tokens.shape[1]
-    assert tokens.is_contiguous() and status.is_contiguous()
-    _check(lib().grid_advance(spec, cin, cout, _ptr(tokens), n, _ptr(status), _stream(stream)))
+    assert tokens.is_contiguous() and status.is_contiguous() and tokens.is_cuda and status.is_cuda
+    assert tokens.dtype == torch.int32 and status.dtype == torch.int32 and tokens.dim() in (1, 2)
+    B = getattr(cout, "B", None)
+    assert B is None or (tokens.shape[0] == B and tuple(status.shape) == (B,)), "tokens [B] or [B, n], status [B]"
+    _check(lib().grid_advance(getattr(spec, "h", spec), getattr(cin, "h", cin), getattr(cout, "h", cout),
+                              _ptr(tokens), n, _ptr(status), _stream(stream)))
 
 
 def grid_masks(spec, cfg, mask, status, stream=None):
@@ -264,9 +270,14 @@ def grid_masks_apply(spec, cfg, mask, status, logits, stream=None):
     tensor [B, >=V], unit stride along V) in the same pass."""
     import torch
     dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
-    assert mask.is_contiguous() and status.is_contiguous() and logits.stride(1) == 1
-    _check(lib().grid_masks_apply(spec, cfg, _ptr(mask), _ptr(status), _ptr(logits), dt, logits.stride(0),
-                                  _stream(stream)))
+    assert mask.is_contiguous() and status.is_contiguous() and mask.is_cuda and status.is_cuda and logits.is_cuda
+    assert mask.dtype == torch.int32 and status.dtype == torch.int32 and mask.dim() == 2 and logits.dim() == 2
+    assert logits.stride(1) == 1 and logits.shape[0] == mask.shape[0]
+    B, W = getattr(cfg, "B", None), getattr(spec, "W", None)
+    assert B is None or (mask.shape[0] == B and tuple(status.shape) == (B,)), "mask [B, W] and status [B] expected"
+    assert W is None or mask.shape[1] == W, "mask [B, ceil(V/32)] expected"
+    _check(lib().grid_masks_apply(getattr(spec, "h", spec), getattr(cfg, "h", cfg), _ptr(mask), _ptr(status),
+                                  _ptr(logits), dt, logits.stride(0), _stream(stream)))
 
 
 def grid_advance_masks(spec, cin, cout, tokens, mask, status, logits=None, stream=None, cache=None):
@@ -452,7 +463,9 @@ def grid_apply_mask(mask, logits, stream=None):
     import torch
     dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
     B, V = logits.shape
-    assert logits.stride(1) == 1
+    assert logits.stride(1) == 1 and logits.is_cuda
+    assert mask.is_contiguous() and mask.is_cuda and mask.dtype == torch.int32 and mask.dim() == 2
+    assert mask.shape[0] == B and mask.shape[1] * 32 >= V, "mask [B, >= ceil(V/32)] for logits [B, V]"
     _check(lib().grid_apply_mask(_ptr(mask), _ptr(logits), dt, B, V, logits.stride(0), _stream(stream)))
 
 
