@@ -134,6 +134,19 @@ def _ptr(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _i32(*xs):
+    """Each tensor is a contiguous int32 CUDA tensor."""
+    import torch
+    for x in xs:
+        assert x.is_contiguous() and x.is_cuda and x.dtype == torch.int32, "contiguous int32 CUDA tensor expected"
+
+
+def _u8_records(records):
+    import torch
+    assert records.is_contiguous() and records.is_cuda and records.dtype == torch.uint8 and records.shape[-1] == 80, \
+        "uint8 CUDA records [..., 80] expected"
+
+
 def _pack(items):
     """list of bytes -> (contiguous buffer, int64 offsets) kept alive by the caller."""
     import numpy as np
@@ -311,21 +324,22 @@ def grid_forced_span(spec, cfg, max_span, mask, span, span_len, status, records=
     """Jump-forward: span int32 CUDA tensor [B, max_span], span_len and status
     int32 [B], mask int32 [B, W] (the final configurations' masks); with audit
     on, records is a uint8 CUDA tensor [B, max_span, 80]."""
-    for x in (mask, span, span_len, status):
-        assert x.is_contiguous()
-    assert span.dim() == 2 and span.shape[1] == max_span
+    _i32(mask, span, span_len, status)
+    assert span.dim() == 2 and span.shape[1] == max_span and mask.dim() == 2
+    assert span.shape[0] == mask.shape[0] == span_len.shape[0] == status.shape[0], "one row per configuration"
     rp = ctypes.c_void_p(None) if records is None else _ptr(records)
     if records is not None:
-        assert records.is_contiguous() and records.numel() == span.shape[0] * max_span * 80
+        _u8_records(records)
+        assert records.numel() == span.shape[0] * max_span * 80
     _check(lib().grid_forced_span(spec, cfg, max_span, _ptr(mask), _ptr(span), _ptr(span_len), _ptr(status), rp,
                                   _stream(stream)))
 
 
 def grid_reserve(spec, cfg, cost, tokens, status, budget=None, safety=0, fire=None, stream=None):
     """cost, status (and budget, fire) int32 CUDA tensors [B]; tokens int32 [B, cap]."""
-    for x in (cost, tokens, status):
-        assert x.is_contiguous()
-    assert tokens.dim() == 2
+    _i32(cost, tokens, status, *[x for x in (budget, fire) if x is not None])
+    assert tokens.dim() == 2 and cost.shape[0] == tokens.shape[0] == status.shape[0], "one row per configuration"
+    assert all(x.shape[0] == cost.shape[0] for x in (budget, fire) if x is not None)
     nul = ctypes.c_void_p(None)
     _check(lib().grid_reserve(spec, cfg, _ptr(cost), _ptr(tokens), tokens.shape[1], _ptr(status),
                               nul if budget is None else _ptr(budget), safety, nul if fire is None else _ptr(fire),
@@ -334,12 +348,16 @@ def grid_reserve(spec, cfg, cost, tokens, status, budget=None, safety=0, fire=No
 
 def grid_masks_cached(spec, cfg, cache, mask, status, logits=None, stream=None):
     """grid_masks (logits None) or grid_masks_apply through a mask cache."""
-    assert mask.is_contiguous() and status.is_contiguous()
+    _i32(mask, status)
+    assert mask.dim() == 2 and mask.shape[0] == status.shape[0]
+    B, W = getattr(cfg, "B", None), getattr(spec, "W", None)
+    assert B is None or mask.shape[0] == B, "mask [B, W] and status [B] expected"
+    assert W is None or mask.shape[1] == W, "mask [B, ceil(V/32)] expected"
     if logits is None:
         lp, dt, stride = ctypes.c_void_p(None), GRID_DTYPE_F32, 0
     else:
         import torch
-        assert logits.stride(1) == 1
+        assert logits.stride(1) == 1 and logits.is_cuda and logits.dim() == 2 and logits.shape[0] == mask.shape[0]
         lp, stride = _ptr(logits), logits.stride(0)
         dt = {torch.float32: GRID_DTYPE_F32, torch.bfloat16: GRID_DTYPE_BF16}[logits.dtype]
     _check(lib().grid_masks_cached(getattr(spec, "h", spec), getattr(cfg, "h", cfg), getattr(cache, "h", cache),
@@ -375,12 +393,14 @@ def grid_configs_enable_audit(spec, cfg, stream=None):
 
 def grid_audit_append(spec, cfg, mask, tokens, kind, records, stream=None):
     """records: uint8 CUDA tensor [B, 80]; tokens int32 [B] (-1 = no record)."""
-    assert records.is_contiguous() and records.shape[-1] == 80 and tokens.is_contiguous()
+    _u8_records(records)
+    _i32(mask, tokens)
     _check(lib().grid_audit_append(spec, cfg, _ptr(mask), _ptr(tokens), kind, _ptr(records), _stream(stream)))
 
 
 def grid_audit_seal(spec, cfg, reason, mode_flags, records, stream=None):
-    assert records.is_contiguous() and records.shape[-1] == 80 and reason.is_contiguous()
+    _u8_records(records)
+    _i32(reason)
     _check(lib().grid_audit_seal(spec, cfg, _ptr(reason), mode_flags, _ptr(records), _stream(stream)))
 
 
