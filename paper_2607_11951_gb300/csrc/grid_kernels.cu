@@ -36,7 +36,12 @@
 //            verdict is set for each of its ids (alias ids share a spelling
 //            and so a verdict) in an id-indexed bitmap with the mask's layout
 //   k_pack   per token id: CI class selection | verdict class | walked verdict
-//            | EOS gate, packed into the id-order mask
+//            | EOS gate, packed into the id-order mask; with logits
+//            (grid_masks_apply) the -inf fill of the word's sectors as well;
+//            with a mask cache, the context-independent bits of a hit read
+//            from the cache entry (or stored into the entry the row claimed)
+// Decoding step (grid_advance_masks): the same kernels, k_row feeding each
+// row's tokens on warp 0 of its block before it prepares the row.
 // Parser step (grid_advance):  k_advance.   Masked logits:  k_apply.
 //
 // Every loop is bounded; hitting a bound writes GRID_ST_BOUND.  No kernel traps.
