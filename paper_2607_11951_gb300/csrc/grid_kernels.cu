@@ -445,7 +445,10 @@ __device__ __forceinline__ bool advance_warp(const Tables& t, const Tables& ts, 
 // ballots), and then the allowed set after that shift is A2 (walks and verdict
 // classes simulate nothing before their second shift).  Phase 2: warp 0 lays
 // out the live first-byte ranges that continue the lexeme (rows without a CI
-// table; they need A0), warps 1 .. 5 select the contexts' CI classes.
+// table; they need A0), warps 1 .. 5 select the contexts' CI classes.  Then
+// thread 0 writes the row's context for the later kernels and, with a mask
+// cache, looks the row's key up (k_pack reads a ready entry) or claims an
+// empty slot for it (k_pack fills it).
 // Clearing blocks zero both verdict bitmaps and the verdict-class bits.
 // With ADV the row's tokens are fed first (advance_warp on warp 0, from
 // adv.cin into c), and the row is masked in the configuration that leaves:
