@@ -22,6 +22,15 @@
  *   grid_apply_mask    logits <- -inf where the mask bit is 0 (Sec. 2,
  *                      "Masked decoding": masked_fill_(-inf))
  *
+ * and around them, in the paper's decoding loop: grid_masks_apply (the mask
+ * with the -inf fill in the same pass), grid_advance_masks (one decoding step:
+ * the sampled tokens fed inside the mask step), grid_masks_static (the mask
+ * with no device allocation), grid_cache_* / grid_masks_cached (the
+ * configuration-keyed mask cache, Sec. 4.3), grid_forced_span (jump-forward,
+ * Sec. 6.1 step 6), grid_reserve (the token-denominated termination reserve,
+ * Sec. 5 Prop. 9) and grid_configs_enable_audit / grid_audit_* (the audit
+ * chain, Sec. 6.4).
+ *
  * Conventions
  *   - Every call returns 0 (GRID_OK) or a negative GRID_E_* code; the message of
  *     the last failure on the calling thread is available from grid_last_error.
@@ -85,7 +94,8 @@ extern "C" {
 #define GRID_ST_NONVIABLE 1         /* the configuration is not a viable prefix      */
 #define GRID_ST_STACK_OVERFLOW 2    /* a push would exceed max_depth                 */
 #define GRID_ST_TOKEN_NOT_ALLOWED 3 /* grid_advance got a token outside the mask      */
-#define GRID_ST_EMPTY_MASK 4        /* viable row with an empty mask: a bug (Prop. 8) */
+#define GRID_ST_EMPTY_MASK 4        /* viable row, empty mask (a vocabulary that is   */
+                                    /* not byte-complete; impossible with, Prop. 8)   */
 #define GRID_ST_BOUND 5             /* a per-token overlay or reduce-chain bound hit  */
 #define GRID_ST_COMPLETE 6          /* the row accepted EOS; its mask is all zero     */
 
