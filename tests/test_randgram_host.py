@@ -52,3 +52,20 @@ def test_random_grammar_sentences_and_compilers(seed):
             cut = int(rng.integers(0, len(s)))
             c = og.feed_bytes(og.start_config(), s[:cut])
             assert c is not None and og.live_end(c), s[:cut]
+
+
+def test_random_workloads_are_seeded_and_well_formed():
+    """The same seed gives the same workload; prefixes are greedy
+    tokenizations of their texts; the vocabulary is byte-complete over the
+    grammar's alphabet with EOS last; the first row is the empty prefix."""
+    from workloads.randgram import rand_grammar_workload
+    a = rand_grammar_workload(3, B=12, V=800, role=[])
+    b = rand_grammar_workload(3, B=12, V=800, role=[])
+    assert a["grammar"] == b["grammar"] and a["tokens"] == b["tokens"] and a["prefixes"] == b["prefixes"]
+    toks = a["tokens"]
+    assert len(toks) == 800 and a["eos"] == 799 and toks[-1] == b"<eos>"
+    alpha = RandGrammar(3).alphabet()
+    assert all(bytes([c]) in toks for c in alpha)
+    assert a["prefixes"][0] == [] and a["texts"][0] == b""
+    for p, t in zip(a["prefixes"], a["texts"]):
+        assert b"".join(toks[i] for i in p) == t
